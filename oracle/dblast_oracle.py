@@ -1,0 +1,305 @@
+"""Plain fp64 CPU oracle for one DBLast draft+verify step.
+
+TEST INFRASTRUCTURE ONLY.  It exists to check the CUDA path; nothing in the
+product path imports it.  Only tests/, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may use it.  It shares no code with the CUDA
+library (no kernels, headers, helpers, tables or pre/post-processing).
+
+Everything is computed in float64 with numpy, in the direct form of the paper:
+the branch hidden states h_{i,z} are materialised and pushed through the
+vocabulary head, exactly as the definitions read; no blocking, fusion or
+reordering is done beyond converting the vocabulary head to fp64 in row chunks
+(a memory-management step of one matrix product).
+
+Definitions followed (section / equation of the paper):
+
+* Latent-mixture proposal q(x_{1:b}|y) = sum_z q(z|y) prod_i q_i(x_i|y,z)
+  (Eq. 5, cp-drafter).
+* Branch hidden states h_{i,z} = h_i + g_z(h_i) (Sec. 3.1, Architecture) with
+  the reused vocabulary head giving q_i(.|y,z).  The expander is taken as
+  rank r: g_z(h) = U_z (V_z^T h) + e_z.
+* Category prior q_{Z_T}(z|y) = softmax(l(y)/Z_T) from a linear head on the
+  block-anchor state (Sec. 3.1, "Drafter sampling during inference";
+  Appendix A: Z_T = 0 selects the highest-prior category).
+* Sampling: z-hat ~ q(z|y), then every position from q_i(.|y,z-hat) (Sec. 3.1,
+  first paragraph of "Dependent Block Drafting and Verification").  Each draw
+  is an inverse-CDF draw with one uniform (see ``inverse_cdf``).
+* Category posterior (Eq. category-posterior) and the mixture next-token
+  distribution (Eq. dep-next-token), which equal the prefix-marginal
+  conditional of Eq. 1 / Eq. dep-conditional.
+* Acceptance A_i = min(1, p/q) (Eq. 2), stop at the first rejection, residual
+  draw from norm([p - q]_+), bonus token when the whole block is accepted
+  (Algorithm 1; Appendix A, "Distributional correctness").
+* Expected accepted length of the drafted block, sum_i prod_{j<=i} A_j
+  (Eq. 3), and the overlap alpha_i = sum_v min(p_i(v), q(v|x_<i)).
+
+Readings where the paper is silent (the same list is kept in the design notes):
+the drafter's token distributions use the same temperature T as the target;
+target rows are given inputs, independent of the drafted prefix; ties in
+argmax go to the lowest index; an inverse-CDF draw takes the smallest index
+whose cumulative mass exceeds u times the total; if a rejection leaves no
+positive residual mass the replacement is drawn from p and flagged.
+"""
+
+import numpy as np
+
+from .philox import (STREAM_ACCEPT, STREAM_DRAFT, STREAM_PRIOR,
+                     STREAM_RESIDUAL, decision_uniform)
+
+# decisions whose margin to the threshold is below this are "ties"
+TIE_TOL = 1e-6
+
+
+def f64(x):
+    """Return x (torch tensor, numpy array or None) as a float64 numpy array."""
+    if x is None:
+        return None
+    if hasattr(x, "detach"):
+        import torch
+        return x.detach().to(device="cpu", dtype=torch.float64).numpy()
+    return np.asarray(x, dtype=np.float64)
+
+
+def logsumexp(s, axis=-1):
+    m = np.max(s, axis=axis, keepdims=True)
+    m = np.where(np.isfinite(m), m, 0.0)
+    with np.errstate(divide="ignore"):
+        out = np.log(np.sum(np.exp(s - m), axis=axis, keepdims=True)) + m
+    return np.squeeze(out, axis=axis)
+
+
+def category_prior(Wp, bp, anchor, z_temperature):
+    """Category logits l = Wp a (+ bp) and the prior pi = softmax(l / Z_T).
+
+    Sec. 3.1 ("Drafter sampling during inference"): q_{Z_T}(z|y) =
+    softmax(l_z(y)/Z_T).  Appendix A: for Z_T = 0 the highest-prior category is
+    selected (one-hot; the lowest index on a tie).
+    """
+    ell = Wp @ anchor
+    if bp is not None:
+        ell = ell + bp
+    if z_temperature == 0:
+        pi = np.zeros_like(ell)
+        pi[int(np.argmax(ell))] = 1.0
+        return ell, pi
+    s = ell / z_temperature
+    e = np.exp(s - np.max(s))
+    return ell, e / np.sum(e)
+
+
+def inverse_cdf(weights, u):
+    """One inverse-CDF draw from non-negative weights (not necessarily normalised).
+
+    Returns (index, margin): index is the smallest v with
+    sum_{v' <= v} w_{v'} > u * sum_v w_v; margin is the distance of u to the
+    nearest edge of the chosen index's CDF interval, in normalised units.  If
+    rounding leaves the target above every prefix sum, the last index with
+    positive weight is returned with margin 0.
+    """
+    w = np.asarray(weights, dtype=np.float64)
+    cum = np.cumsum(w)
+    total = cum[-1]
+    target = u * total
+    idx = int(np.searchsorted(cum, target, side="right"))
+    if idx >= w.shape[0]:
+        nz = np.nonzero(w > 0)[0]
+        return int(nz[-1]) if nz.size else w.shape[0] - 1, 0.0
+    lo = cum[idx - 1] if idx > 0 else 0.0
+    margin = min(target - lo, cum[idx] - target) / total
+    return idx, margin
+
+
+def branch_hidden(h, U, Vf, e):
+    """h_{i,z} = h_i + U_z (V_z^T h_i) + e_z for every position i and branch z.
+
+    Sec. 3.1 (Architecture): the category hidden expander maps h_i to K
+    category-specific offsets g_z(h_i).  h: [B, H]; U, Vf: [K, H, r];
+    e: [K, H] or None.  Returns [B, K, H].
+    """
+    B, H = h.shape
+    K = U.shape[0]
+    out = np.empty((B, K, H), dtype=np.float64)
+    for z in range(K):
+        code = h @ Vf[z]              # V_z^T h_i, [B, r]
+        g = code @ U[z].T             # U_z code, [B, H]
+        if e is not None:
+            g = g + e[z]
+        out[:, z, :] = h + g
+    return out
+
+
+def component_logits(W, hz, vbias, chunk=8192):
+    """l_{i,z,v} = W_v . h_{i,z} (+ b_v): the reused vocabulary head on each branch.
+
+    Sec. 3.1 (Architecture).  W is [V, H] (any dtype; converted to fp64 in row
+    chunks), hz is [B, K, H].  Returns [B, K, V] in fp64.
+    """
+    B, K, H = hz.shape
+    V = W.shape[0]
+    flat = hz.reshape(B * K, H)
+    out = np.empty((B * K, V), dtype=np.float64)
+    for v0 in range(0, V, chunk):
+        Wc = f64(W[v0:v0 + chunk])
+        out[:, v0:v0 + Wc.shape[0]] = flat @ Wc.T
+    if vbias is not None:
+        out += vbias[None, :]
+    return out.reshape(B, K, V)
+
+
+def posterior(log_pi, logq_at_x):
+    """Category posterior and its normaliser along the drafted prefix.
+
+    Eq. category-posterior: q(z|y,x_<i) is proportional to
+    q(z|y) prod_{j<i} q_j(x_j|y,z).  log_pi: [K]; logq_at_x: [B, K] with
+    logq_at_x[j, z] = log q_j(x_j|y,z).  Returns log w: [B, K], normalised
+    over z for every position i.
+    """
+    B, K = logq_at_x.shape
+    logw = np.empty((B, K), dtype=np.float64)
+    acc = np.array(log_pi, dtype=np.float64)
+    for i in range(B):
+        logw[i] = acc - logsumexp(acc)
+        acc = acc + logq_at_x[i]
+    return logw
+
+
+def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
+                              seed, n, pos, round_):
+    """One draft+verify step for sequence n (all arrays fp64 numpy).
+
+    head: dict with W [V,H] (any dtype), U, Vf [K,H,r], e [K,H]|None,
+    Wp [K,H], bp [K]|None, vbias [V]|None.  h: [B,H]; anchor: [H]|None
+    (None: h[0]); target: [B+has_bonus, V] target logits.
+    """
+    B, H = h.shape
+    W = head["W"]
+    a = h[0] if anchor is None else anchor
+    ties = []
+
+    # prior and latent category (Sec. 3.1; Appendix A)
+    ell, pi = category_prior(head["Wp"], head["bp"], a, Z_T)
+    u0 = decision_uniform(seed, STREAM_PRIOR, round_, n, pos)
+    zhat, m0 = inverse_cdf(pi, u0)
+    if Z_T != 0 and m0 < TIE_TOL:
+        ties.append(("zhat", -1, m0))
+    with np.errstate(divide="ignore"):
+        log_pi = np.log(pi)
+
+    # branch distributions q_i(.|y,z) = softmax(l_{i,z}/T)
+    hz = branch_hidden(h, head["U"], head["Vf"], head["e"])
+    s = component_logits(W, hz, head["vbias"]) / T          # [B, K, V]
+    lse = logsumexp(s, axis=-1)                               # [B, K]
+    logq = s - lse[:, :, None]
+
+    # draft block: every position from the z-hat branch
+    tokens = np.empty(B, dtype=np.int64)
+    for i in range(B):
+        u1 = decision_uniform(seed, STREAM_DRAFT, round_, n, pos + i)
+        tokens[i], m1 = inverse_cdf(np.exp(logq[i, zhat]), u1)
+        if m1 < TIE_TOL:
+            ties.append(("draft", i, m1))
+
+    # posterior weights and the mixture conditional q(.|y,x_<i)
+    logq_at_x = logq[np.arange(B), :, tokens]                 # [B, K]
+    logw = posterior(log_pi, logq_at_x)
+    w = np.exp(logw)
+    qmix = np.einsum("bk,bkv->bv", w, np.exp(logq))           # Eq. dep-next-token
+    q_tok = qmix[np.arange(B), tokens]
+
+    # target distributions p_i = softmax(t_i / T)
+    st = target / T
+    lse_t = logsumexp(st, axis=-1)
+    p = np.exp(st - lse_t[:, None])                           # [B+hb, V]
+    p_tok = p[np.arange(B), tokens]
+
+    alpha = np.sum(np.minimum(p[:B], qmix), axis=-1)
+    ratio = p_tok / q_tok
+    accept_prob = np.minimum(1.0, ratio)
+
+    # sequential acceptance (Eq. 2; Algorithm 1)
+    L = B
+    for i in range(B):
+        u2 = decision_uniform(seed, STREAM_ACCEPT, round_, n, pos + i)
+        m2 = abs(u2 * q_tok[i] - p_tok[i]) / q_tok[i]
+        if m2 < TIE_TOL:
+            ties.append(("accept", i, m2))
+        if not (u2 < ratio[i]):
+            L = i
+            break
+
+    emitted = list(int(x) for x in tokens[:L])
+    extra = -1
+    if L < B:
+        # residual norm([p - q]_+) at the first rejected position
+        u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + L)
+        res = np.maximum(p[L] - qmix[L], 0.0)
+        mass = float(np.sum(res))
+        if mass > 0.0:
+            extra, m3 = inverse_cdf(res, u3)
+        else:
+            extra, m3 = inverse_cdf(p[L], u3)
+        if mass < TIE_TOL:
+            ties.append(("residual_mass", L, mass))
+        if m3 < TIE_TOL:
+            ties.append(("residual", L, m3))
+    elif has_bonus:
+        u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + B)
+        extra, m3 = inverse_cdf(p[B], u3)
+        if m3 < TIE_TOL:
+            ties.append(("bonus", B, m3))
+    if extra >= 0:
+        emitted.append(int(extra))
+
+    # Eq. 3 on the drafted block, and the same sum over the overlaps
+    exp_len = float(np.sum(np.cumprod(accept_prob)))
+    alpha_len = float(np.sum(np.cumprod(alpha)))
+
+    first_tie = B + 1
+    for kind, i, _ in ties:
+        first_tie = min(first_tie, 0 if kind == "zhat" else i)
+
+    return dict(pi=pi, ell=ell, zhat=int(zhat), tokens=tokens, lse=lse,
+                logw=logw, q_tok=q_tok, p_tok=p_tok, accept_prob=accept_prob,
+                alpha=alpha, accepted=L, emitted=emitted,
+                n_emitted=len(emitted), exp_len=exp_len, alpha_len=alpha_len,
+                lse_target=lse_t, ties=ties, first_tie=first_tie)
+
+
+def prepare_head(head):
+    """fp64 copies of the small head tensors; W is left as given (chunked later)."""
+    out = {k: f64(head.get(k)) for k in ("U", "Vf", "e", "Wp", "bp", "vbias")}
+    out["W"] = head["W"]
+    return out
+
+
+def draft_and_verify(head, hidden, anchor, target, has_bonus, T, Z_T, seed,
+                     pos, round_, seqs=None):
+    """Run the step for the sequences in ``seqs`` (default: all).
+
+    hidden: [N, B, H]; anchor: [N, H] or None; target: [N, B+has_bonus, V];
+    pos: [N] int; round_: [N] int.  Returns a list of per-sequence dicts
+    (see draft_and_verify_sequence) in the order of ``seqs``.
+    """
+    hd = prepare_head(head)
+    N = hidden.shape[0]
+    seqs = range(N) if seqs is None else seqs
+    out = []
+    for n in seqs:
+        h = f64(hidden[n])
+        a = None if anchor is None else f64(anchor[n])
+        t = f64(target[n])
+        out.append(draft_and_verify_sequence(
+            hd, h, a, t, bool(has_bonus), float(T), float(Z_T), int(seed),
+            int(n), int(pos[n]), int(round_[n])))
+    return out
+
+
+def expander_parameter_count(H, K, rank=None):
+    """Parameters added by the category expander and the prior head.
+
+    Table 1 (full-rank expander, one linear layer with bias per category, plus
+    a linear prior head with bias): K H^2 + 2 K H + K.  With a rank-r expander
+    U_z V_z^T + e_z the first term becomes 2 K H r.
+    """
+    expander = K * H * H if rank is None else 2 * K * H * rank
+    return expander + K * H + (K * H + K)
