@@ -1,0 +1,368 @@
+"""Benchmark of the fused DBLast draft+verify step on GB300.
+
+One step = one dblast_draft_and_verify call over a batch of N sequences
+(prior, codes, vocabulary-head pass with fused softmax statistics, draft
+tokens, posterior, target pass, fused verify pass, acceptance and
+residual/bonus draws, state update).  Inputs are synthetic and resident in HBM
+(W 1.2 GB and target logits 165 MB exceed the 129 MB L2, so no flush is
+needed).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank runs an independent replica on its own GPU (the
+sequences are independent units; there is no data-path collective) and rank
+0 prints the aggregate.  --impl reference times the fp64 CPU oracle on a
+bounded sample (one sequence per step) on the host cores.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "draft+verify blocks/sec and accepted tokens/sec at 1 GB300; % of roofline"
+UNIT = "blocks/s"
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"],
+                    bf16_sus=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def work_model(cfg):
+    """Algorithmic FLOPs and bytes of one step (low-rank factored head)."""
+    V, H, K, r, N, B = (cfg[k] for k in ("V", "H", "K", "r", "N", "B"))
+    rr = r + (1 if cfg.get("expander_bias") else 0)
+    M = N * B
+    el = 2 if cfg["dtype"] == "bf16" else 4
+    flop_base = 2.0 * V * H * M
+    flop_corr = 2.0 * V * rr * K * M
+    flop_codes = 2.0 * M * K * r * H
+    byts = (V * H * el + N * (B + 1) * V * el + M * H * el + 2 * K * H * r * el +
+            K * H * el + M * (4 * K * 3 + 16))
+    return dict(flop=flop_base + flop_corr + flop_codes, flop_draft_pass=flop_base + flop_corr,
+                bytes=byts, flop_direct=2.0 * V * H * M * K)
+
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region (median SM clock, reasons)."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for nm, val in zip(names, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0):
+    """Time the fp64 oracle, as it stands, on one sequence of the workload."""
+    import torch
+    from oracle import dblast_oracle as orc
+    head_cpu = {k: (None if v is None else v.cpu()) for k, v in head.items()}
+    blk_cpu = {"hidden": blk["hidden"].cpu(), "anchor": None, "target": blk["target"].cpu(),
+               "has_bonus": blk["has_bonus"]}
+    pos = torch.full((cfg["N"],), 37, dtype=torch.int64)
+    rnd = torch.zeros(cfg["N"], dtype=torch.int32)
+    n_done, t0 = 0, time.perf_counter()
+    while True:
+        orc.draft_and_verify(head_cpu, blk_cpu["hidden"], None, blk_cpu["target"],
+                             blk_cpu["has_bonus"], T, Z_T, 0, pos.numpy(), rnd.numpy(),
+                             seqs=[n_done % cfg["N"]])
+        n_done += 1
+        el = time.perf_counter() - t0
+        if el > budget_s / 3 or n_done >= 4:
+            break
+    return {"value": n_done / el, "unit": UNIT, "cores": _cpu_threads(),
+            "kind": "oracle",
+            "sample": "%d sequence(s) of the %s workload (one block each), fp64 direct form"
+                      % (n_done, cfg["name"])}
+
+
+def _cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("num_threads")]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def run_reference(args, cfg, rank):
+    """--impl reference: the oracle on the host cores, one sequence per step."""
+    import torch
+    import synth
+    from oracle import dblast_oracle as orc
+    if rank != 0:
+        return
+    head = synth.make_head(cfg, "cpu")
+    blk = synth.make_block(cfg, head, 0, "cpu")
+    pos, rnd = synth.initial_state(cfg, "cpu")
+    L_total = 0
+
+    def step(i):
+        o = orc.draft_and_verify(head, blk["hidden"], None, blk["target"], blk["has_bonus"],
+                                 args.T, 1.0, i, pos.numpy(), rnd.numpy(),
+                                 seqs=[i % cfg["N"]])
+        return o[0]["accepted"]
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        L_total += step(1000 + i)
+    el = time.perf_counter() - t0
+    v = args.steps / el
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg["name"], "N": cfg["N"], "B": cfg["B"], "K": cfg["K"],
+                       "r": cfg["r"], "H": cfg["H"], "V": cfg["V"], "T": args.T,
+                       "sample": "one sequence (block) per step"},
+            "accepted_tokens_per_s": L_total / el,
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": _cpu_threads(),
+                             "kind": "oracle",
+                             "sample": "one sequence of %s per step" % cfg["name"]},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="qwen3_8b_b32")
+    ap.add_argument("--T", type=float, default=1.0)
+    ap.add_argument("--kernels", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=None)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    import synth
+    cfg = synth.config(args.config)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, cfg, rank)
+        return
+
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_05448_gb300 import (Head, Workspace, alloc_draft_out, alloc_verify_out,
+                                        dblast_draft_and_verify, dblast_stats_get,
+                                        dblast_stats_reset)
+    peaks = load_peaks()
+    dev = torch.device("cuda", local)
+    head_t = synth.make_head(cfg, dev)
+    blk = synth.make_block(cfg, head_t, 0, dev)
+    N, B = cfg["N"], cfg["B"]
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    head = Head.from_dict(head_t)
+    torch.cuda.synchronize()
+    prep_ms = 1e3 * (time.perf_counter() - t0)
+    ws = Workspace(head, N, B, blk["has_bonus"])
+    pos, rnd = synth.initial_state(cfg, dev)
+    K_steps = args.steps
+    dout = alloc_draft_out(N, B, cfg["K"], dev)
+    vouts = [alloc_verify_out(N, B, blk["has_bonus"], dev) for _ in range(K_steps)]
+    seed = 1234 + 7919 * rank
+
+    def step(vout):
+        dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, args.T, cfg["Z_T"], seed,
+                                blk["target"], blk["has_bonus"], impl=args.kernels,
+                                dout=dout, vout=vout)
+
+    for _ in range(args.warmup):
+        step(vouts[0])
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    dblast_stats_reset(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    for k in range(K_steps):
+        step(vouts[k])
+    ev1.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    st = dblast_stats_get()
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    accepted = sum(int(v["accepted"].sum()) for v in vouts)
+    emitted = sum(int(v["n_emitted"].sum()) for v in vouts)
+    if world > 1:
+        tt = torch.tensor([accepted, emitted], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt)
+        accepted, emitted = int(tt[0]), int(tt[1])
+    ms_step = ms / K_steps
+    value = N * world * K_steps / (ms / 1e3)
+
+    # end to end through the public API with host buffers (pinned), per step:
+    # H2D of hidden + target, the call, D2H of the per-sequence results
+    e2e_steps = args.e2e_steps or K_steps
+    h_host = blk["hidden"].cpu().pin_memory()
+    t_host = blk["target"].cpu().pin_memory()
+    res_host = {k: torch.empty_like(vouts[0][k], device="cpu").pin_memory()
+                for k in ("accepted", "n_emitted", "emitted", "exp_len")}
+    h_dev, t_dev = torch.empty_like(blk["hidden"]), torch.empty_like(blk["target"])
+    h2d = h_host.numel() * h_host.element_size() + t_host.numel() * t_host.element_size()
+    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for k in range(e2e_steps):
+        h_dev.copy_(h_host, non_blocking=True)
+        t_dev.copy_(t_host, non_blocking=True)
+        dblast_draft_and_verify(head, ws, h_dev, pos, rnd, args.T, cfg["Z_T"], seed, t_dev,
+                                blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0])
+        for kk, v in res_host.items():
+            v.copy_(vouts[0][kk], non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    ems = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([ems], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ems = float(tt.item())
+    e2e_value = N * world * e2e_steps / (ems / 1e3)
+
+    if rank == 0:
+        wm = work_model(cfg)
+        draft_ms = st["draft_pass_ms"] / max(1, st["timed_draft"])
+        verify_ms = st["verify_pass_ms"] / max(1, st["timed_verify"])
+        achieved = wm["flop_draft_pass"] / (draft_ms * 1e-3) / 1e12
+        t_roof = max(wm["flop"] / (peaks["bf16"] * 1e12), wm["bytes"] / (peaks["hbm"] * 1e9))
+        traffic = None
+        tr_path = os.path.join(ROOT, "profiles", "draft_pass_traffic.json")
+        if os.path.exists(tr_path):
+            d = json.load(open(tr_path))
+            if d.get("kernel_impl") == _impl_name(head, args) and d.get("workload") == cfg["name"]:
+                traffic = d.get("bytes_per_launch")
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": K_steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if cfg["dtype"] == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": cfg["name"], "N": N, "B": B, "K": cfg["K"], "r": cfg["r"],
+                       "H": cfg["H"], "V": cfg["V"], "T": args.T, "Z_T": cfg["Z_T"],
+                       "sigma": cfg["sigma"], "kernels": _impl_name(head, args),
+                       "parallelism": "replicas" if world > 1 else "single",
+                       "l2": "no flush: inputs larger than L2 (W %.2f GB, target %.0f MB)" % (
+                           cfg["V"] * cfg["H"] * 2 / 1e9,
+                           N * (B + 1) * cfg["V"] * 2 / 1e6)},
+            "accepted_tokens_per_s": accepted / (ms / 1e3),
+            "emitted_tokens_per_s": emitted / (ms / 1e3),
+            "mean_accepted_length": accepted / (N * world * K_steps),
+            "roofline_step": {"t_roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms_step,
+                              "flop": wm["flop"], "bytes": wm["bytes"],
+                              "flop_direct_form": wm["flop_direct"],
+                              "peak_source": peaks["source"]},
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"],
+                         "unit": "TFLOP/s", "frac": achieved / peaks["bf16"],
+                         "traffic": traffic, "kernel": "draft pass",
+                         "ms_per_launch": draft_ms},
+            "verify_pass_ms": verify_ms,
+            "prep_ms": prep_ms,
+            "gpu_launches": int(st["kernel_launches"]),
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "clocks": clk,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(cfg, head_t, blk, args.T, cfg["Z_T"])
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _impl_name(head, args):
+    if args.kernels != "auto":
+        return args.kernels
+    return "tcgen05" if (head.dtype.__str__() == "torch.bfloat16" and head.H % 64 == 0
+                         and _tc_available()) else "simt"
+
+
+def _tc_available():
+    try:
+        from paper_2608_05448_gb300 import binding
+        return getattr(binding, "TC_AVAILABLE", False)
+    except Exception:
+        return False
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,191 @@
+/*
+ * dblast.h - C ABI of the DBLast draft+verify step on one GPU (sm_103a).
+ *
+ * The step (paper: "DBLast: Dependent Block Drafting for Stochastic
+ * Speculative Decoding") drafts a block of B tokens from a K-component
+ * latent-mixture proposal and verifies it against given target logits:
+ *
+ *   draft   - category prior and latent draw z-hat (Sec. 3.1, "Drafter
+ *             sampling during inference"), branch distributions through the
+ *             reused vocabulary head (Sec. 3.1, Architecture; Eq. 5), one
+ *             draft token per position from the z-hat branch, the category
+ *             posterior (Eq. category-posterior) and the mixture conditional
+ *             q(x_i|x_<i) (Eq. dep-next-token, equal to Eq. 1).
+ *   verify  - acceptance with probability min(1, p/q) (Eq. 2), stop at the
+ *             first rejection, residual draw from norm([p - q]_+) or the
+ *             bonus token when all B are accepted (Algorithm 1; Appendix A,
+ *             "Distributional correctness"), the overlap
+ *             alpha_i = sum_v min(p_i(v), q(v|x_<i)) and the expected accepted
+ *             length of the drafted block sum_i prod_{j<=i} A_j (Eq. 3).
+ *
+ * The expander is rank r: h_{i,z} = h_i + U_z (V_z^T h_i) + e_z.
+ * Temperatures: q_i(.|z) = softmax(l_{i,z}/T), p_i = softmax(t_i/T),
+ * prior softmax(l/Z_T) (Z_T = 0 selects the highest-prior category).
+ *
+ * Conventions for every entry point:
+ *   - All array pointers are DEVICE pointers to caller-owned, row-major,
+ *     contiguous memory, 16-byte aligned.  The library never allocates or
+ *     frees device memory; scratch space comes from the caller ("prep" and
+ *     "workspace" buffers, sized by the *_bytes queries).
+ *   - Calls are asynchronous on `stream`.  Argument errors are returned
+ *     immediately, before any launch.  Errors found on the device (a bounded
+ *     wait that ran out) are recorded in the workspace and reported by
+ *     dblast_device_status().
+ *   - Shapes: 1 <= K <= 32, 1 <= r <= 64, 1 <= B <= 32, N >= 1, V >= 1,
+ *     H >= 8 with H % 8 == 0; T > 0; Z_T >= 0.
+ *   - Random decisions use one uniform each from Philox4x32-10 (Salmon et al.,
+ *     SC'11) with key (seed lo, seed hi) and counter
+ *     (0, pos_abs, n, (stream << 24) | (round & 0xffffff)); u = ((w0>>9)+0.5)
+ *     * 2^-23.  Streams: 0 latent category (pos_abs = pos[n]), 1 draft token,
+ *     2 acceptance, 3 residual/bonus (pos_abs = pos[n] + i).  Every draw is an
+ *     inverse-CDF draw in vocabulary order: the smallest index whose
+ *     cumulative mass exceeds u times the total.
+ */
+#ifndef DBLAST_H_
+#define DBLAST_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* dblast_stream_t; /* a cudaStream_t; NULL = legacy default stream */
+
+typedef enum {
+  DBLAST_OK = 0,
+  DBLAST_ERR_INVALID_ARG = 1,  /* NULL pointer, bad shape, bad temperature */
+  DBLAST_ERR_UNSUPPORTED = 2,  /* shape/dtype the requested implementation cannot run */
+  DBLAST_ERR_WORKSPACE = 3,    /* prep or workspace buffer too small / misaligned */
+  DBLAST_ERR_CUDA = 4,         /* a CUDA runtime call failed */
+  DBLAST_ERR_TIMEOUT = 5,      /* a device-side bounded wait ran out (see dblast_device_status) */
+  DBLAST_ERR_NO_DEVICE = 6     /* no usable sm_103 device */
+} dblast_status;
+
+typedef enum { DBLAST_BF16 = 0, DBLAST_F32 = 1 } dblast_dtype;
+
+/* Kernel family for the two vocabulary-wide passes.  AUTO picks TCGEN05 for
+ * bf16 inputs with H % 64 == 0, else SIMT (plain CUDA cores, any shape). */
+typedef enum { DBLAST_IMPL_AUTO = 0, DBLAST_IMPL_SIMT = 1, DBLAST_IMPL_TCGEN05 = 2 } dblast_impl;
+
+/* Drafter head (Sec. 3.1, Architecture; Table 1 with a rank-r expander).
+ * W is the reused vocabulary head, U/Vf the expander factors, e its optional
+ * bias, Wp/bp the category-prior head, vbias an optional vocabulary bias.
+ * W, U, Vf, e, Wp have `dtype`; bp and vbias are fp32. */
+typedef struct {
+  int V, H, K, r;
+  dblast_dtype dtype;
+  const void* W;      /* [V, H]    */
+  const void* U;      /* [K, H, r] */
+  const void* Vf;     /* [K, H, r] */
+  const void* e;      /* [K, H] or NULL */
+  const void* Wp;     /* [K, H]    */
+  const float* bp;    /* [K] or NULL */
+  const float* vbias; /* [V] or NULL */
+  void* prep;         /* device buffer, dblast_prep_bytes() bytes, filled by dblast_head_prepare() */
+  size_t prep_bytes;
+} dblast_head;
+
+/* One block per sequence n.  pos[n] is the absolute position of the first
+ * block token and round[n] counts the sequence's draft/verify rounds; both
+ * feed the Philox counters and are advanced by the verify step
+ * (pos += n_emitted, round += 1). */
+typedef struct {
+  int N, B;
+  float temperature;     /* T > 0, for drafter and target token distributions */
+  float z_temperature;   /* Z_T >= 0, category temperature */
+  uint64_t seed;
+  const void* hidden;    /* [N, B, H] block hidden states h_i (head dtype) */
+  const void* anchor;    /* [N, H] block-anchor state for the prior, or NULL = hidden[:, 0, :] */
+  int64_t* pos;          /* [N] in/out */
+  uint32_t* round;       /* [N] in/out */
+  dblast_impl impl;
+} dblast_block_args;
+
+/* Draft outputs.  Every pointer may be NULL (not written). */
+typedef struct {
+  int32_t* z_hat;  /* [N]       latent category */
+  float* pi;       /* [N, K]    tempered prior softmax(l/Z_T) */
+  int32_t* tokens; /* [N, B]    draft block */
+  float* lse;      /* [N, B, K] natural log of sum_v exp(l_{i,z,v}/T) */
+  float* logw;     /* [N, B, K] natural log of the posterior q(z|y,x_<i) */
+  float* q_tok;    /* [N, B]    q(x_i|y,x_<i) */
+} dblast_draft_out;
+
+/* Verify inputs/outputs.  target is required; every output may be NULL. */
+typedef struct {
+  const void* target;   /* [N, B + has_bonus, V] target logits (head dtype) */
+  int has_bonus;        /* 1: row B holds the bonus-position logits */
+  float* p_tok;         /* [N, B]     p_i(x_i) */
+  float* accept_prob;   /* [N, B]     A_i = min(1, p/q) (Eq. 2) */
+  float* alpha;         /* [N, B]     sum_v min(p_i(v), q(v|x_<i)) */
+  float* lse_target;    /* [N, B+has_bonus] natural log of sum_v exp(t/T) */
+  int32_t* accepted;    /* [N]        accepted draft tokens L (bonus/residual excluded) */
+  int32_t* emitted;     /* [N, B+1]   accepted tokens then the residual/bonus token, -1 padded */
+  int32_t* n_emitted;   /* [N]        number of valid entries in emitted */
+  float* exp_len;       /* [N]        sum_i prod_{j<=i} A_j (Eq. 3) */
+  float* alpha_len;     /* [N]        sum_i prod_{j<=i} alpha_j */
+  uint32_t* tie_flags;  /* [N]        bit0 z-hat, bit1 draft, bit2 accept, bit3 residual/bonus,
+                                       bit4 residual mass < 1e-6: a decision within 1e-6 of its threshold */
+} dblast_verify_out;
+
+/* Bytes of the prep buffer for this head (depends on V, K, r, e != NULL). */
+size_t dblast_prep_bytes(const dblast_head* head);
+
+/* Bytes of the per-call workspace for N sequences of block B. */
+size_t dblast_workspace_bytes(const dblast_head* head, int N, int B, int has_bonus);
+
+/* Once per weight set: fills head->prep with W U_z (and W e_z) in fp32 and in
+ * the split-fp16 operand layout of the tensor-core pass.  Asynchronous. */
+dblast_status dblast_head_prepare(const dblast_head* head, dblast_stream_t stream);
+
+/* Draft: prior, z-hat, branch statistics, draft block, posterior and q_tok.
+ * Leaves in `workspace` what dblast_verify_block needs. */
+dblast_status dblast_draft_block(const dblast_head* head, const dblast_block_args* args,
+                                 dblast_draft_out* out, void* workspace, size_t workspace_bytes,
+                                 dblast_stream_t stream);
+
+/* Verify a block drafted by dblast_draft_block with the same head, args and
+ * workspace (unmodified in between).  Advances pos and round. */
+dblast_status dblast_verify_block(const dblast_head* head, const dblast_block_args* args,
+                                  dblast_verify_out* out, void* workspace, size_t workspace_bytes,
+                                  dblast_stream_t stream);
+
+/* Both, in one call. */
+dblast_status dblast_draft_and_verify(const dblast_head* head, const dblast_block_args* args,
+                                      dblast_draft_out* dout, dblast_verify_out* vout,
+                                      void* workspace, size_t workspace_bytes,
+                                      dblast_stream_t stream);
+
+/* Synchronises `stream`, returns DBLAST_ERR_TIMEOUT if a device-side wait of
+ * a previous call on this workspace ran out (and clears the record). */
+dblast_status dblast_device_status(void* workspace, dblast_stream_t stream);
+
+/* Host-side fault injection for tests: spin limit of the device-side bounded
+ * waits of later calls (0 = default).  A limit of 1 makes waits give up. */
+void dblast_set_wait_limit(uint32_t spins);
+
+/* Measurement counters of this process.  dblast_stats_reset() zeroes them and
+ * turns per-pass timing on or off: while on, every call records CUDA events
+ * on its stream around its draft pass (the vocabulary-head contraction with
+ * its fused softmax epilogue) and its verify pass (the fused target-streaming
+ * kernel).  dblast_stats_get() waits for the recorded events and returns the
+ * summed pass times (ms), the number of timed calls and the number of kernel
+ * launches issued by the library since the reset. */
+typedef struct {
+  uint64_t calls;            /* draft/verify entry-point calls */
+  uint64_t kernel_launches;  /* kernels launched by the library */
+  uint64_t timed_draft, timed_verify;
+  double draft_pass_ms, verify_pass_ms;
+} dblast_stats;
+void dblast_stats_reset(int enable_pass_timing);
+dblast_status dblast_stats_get(dblast_stats* out);
+
+const char* dblast_status_string(dblast_status s);
+const char* dblast_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DBLAST_H_ */

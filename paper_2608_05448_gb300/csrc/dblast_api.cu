@@ -1,0 +1,362 @@
+// C ABI of libdblast: argument checks, prep/workspace layouts, launch order.
+// Every entry point is asynchronous on the caller's stream and allocates no
+// device memory.
+#include <atomic>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "dblast_internal.cuh"
+
+namespace dblast {
+
+static uint32_t g_wait_limit = 0;  // 0 = default; read by the tensor-core launchers
+uint32_t wait_limit() { return g_wait_limit; }
+
+// ------------------------------------------------------------ measurement
+static std::mutex g_stats_mu;
+static std::atomic<uint64_t> g_launches{0}, g_calls{0};
+static bool g_timing = false;
+constexpr int kMaxTimed = 4096;
+static std::vector<cudaEvent_t> g_ev[2];  // pairs (begin, end) per timed call
+static int g_n_ev[2] = {0, 0};
+
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+// DBLAST_DEBUG_SYNC=1: synchronise after every launcher and name the one that failed
+static bool debug_sync() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = getenv("DBLAST_DEBUG_SYNC");
+    v = (e && e[0] == '1') ? 1 : 0;
+  }
+  return v == 1;
+}
+void debug_kernel(const char* name, cudaStream_t s) {
+  if (!debug_sync()) return;
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  fprintf(stderr, "dblast debug kernel: %-20s %s\n", name, cudaGetErrorString(e));
+}
+
+static cudaError_t dbg(cudaError_t e, const char* what, cudaStream_t s) {
+  if (e != cudaSuccess || !debug_sync()) return e;
+  e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  fprintf(stderr, "dblast debug: %-22s %s\n", what, cudaGetErrorString(e));
+  return e;
+}
+
+static cudaEvent_t pool_event(int which, int idx) {
+  auto& v = g_ev[which];
+  while ((int)v.size() <= idx) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    v.push_back(e);
+  }
+  return v[idx];
+}
+
+void pass_event_begin(int which, cudaStream_t s) {
+  std::lock_guard<std::mutex> lk(g_stats_mu);
+  if (!g_timing || g_n_ev[which] >= kMaxTimed) return;
+  cudaEvent_t e = pool_event(which, 2 * g_n_ev[which]);
+  if (e) cudaEventRecord(e, s);
+}
+
+void pass_event_end(int which, cudaStream_t s) {
+  std::lock_guard<std::mutex> lk(g_stats_mu);
+  if (!g_timing || g_n_ev[which] >= kMaxTimed) return;
+  cudaEvent_t e = pool_event(which, 2 * g_n_ev[which] + 1);
+  if (e) {
+    cudaEventRecord(e, s);
+    ++g_n_ev[which];
+  }
+}
+
+PrepLayout prep_layout(int V, int H, int K, int r, bool has_e) {
+  (void)H;
+  PrepLayout p{};
+  p.V = V;
+  p.K = K;
+  p.rr = r + (has_e ? 1 : 0);
+  p.rp = ceil_div(p.rr, 16) * 16;
+  p.KC = K * 2 * p.rp;
+  size_t o = 0;
+  p.off_wu = o;
+  o = align_up(o + (size_t)V * K * p.rr * sizeof(float), 256);
+  p.off_wuop = o;
+  o = align_up(o + (size_t)V * p.KC * sizeof(__half), 256);
+  p.off_sw = o;
+  o = align_up(o + (size_t)K * sizeof(float), 256);
+  p.total = o;
+  return p;
+}
+
+WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus) {
+  WsLayout w{};
+  w.N = N;
+  w.B = B;
+  w.M = N * B;
+  w.Mpad = ceil_div(w.M, MTILE) * MTILE;
+  w.K = K;
+  w.rr = r + (has_e ? 1 : 0);
+  w.rp = ceil_div(w.rr, 16) * 16;
+  w.KC = K * 2 * w.rp;
+  w.V = V;
+  w.nt = ceil_div(V, TILE_V);
+  (void)has_bonus;  // the layout is the same with or without a bonus row
+  w.Rt = N * (B + 1);
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  w.off_status = take(256);
+  w.off_codes = take((size_t)w.Mpad * K * w.rr * sizeof(float));
+  w.off_cscale = take((size_t)w.Mpad * K * sizeof(float));
+  w.off_cop = take((size_t)w.Mpad * w.KC * sizeof(__half));
+  w.off_zhat = take((size_t)N * sizeof(int32_t));
+  w.off_log2pi = take((size_t)N * K * sizeof(float));
+  w.off_stash = take((size_t)w.M * V * sizeof(float));
+  w.off_partd = take((size_t)w.nt * K * w.Mpad * sizeof(float2));
+  w.off_lse2 = take((size_t)w.M * K * sizeof(double));
+  w.off_lq2 = take((size_t)w.M * K * sizeof(double));
+  w.off_w2 = take((size_t)w.M * K * sizeof(double));
+  w.off_tok = take((size_t)w.M * sizeof(int32_t));
+  w.off_partt = take((size_t)w.nt * w.Rt * sizeof(float2));
+  w.off_lse2t = take((size_t)w.Rt * sizeof(double));
+  w.off_partv = take((size_t)w.nt * w.Mpad * sizeof(float2));
+  w.off_av = take((size_t)w.M * sizeof(double2));
+  w.off_ties = take((size_t)N * sizeof(uint32_t));
+  w.total = o;
+  return w;
+}
+
+cudaError_t launch_draft_pass_tc(const StepCtx& c);
+cudaError_t launch_verify_pass_tc(const StepCtx& c);
+bool tc_supported(const dblast_head* h);
+
+}  // namespace dblast
+
+using namespace dblast;
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+static dblast_status check_head(const dblast_head* h, bool need_prep) {
+  if (!h) return DBLAST_ERR_INVALID_ARG;
+  if (h->V < 1 || h->H < 8 || (h->H % 8) != 0 || h->K < 1 || h->K > 32 || h->r < 1 || h->r > 64)
+    return DBLAST_ERR_INVALID_ARG;
+  if (h->dtype != DBLAST_BF16 && h->dtype != DBLAST_F32) return DBLAST_ERR_INVALID_ARG;
+  if (!h->W || !h->U || !h->Vf || !h->Wp) return DBLAST_ERR_INVALID_ARG;
+  const void* ptrs[] = {h->W, h->U, h->Vf, h->e, h->Wp, h->bp, h->vbias};
+  for (const void* p : ptrs)
+    if (p && !aligned16(p)) return DBLAST_ERR_INVALID_ARG;
+  if (need_prep) {
+    if (!h->prep || !aligned16(h->prep)) return DBLAST_ERR_WORKSPACE;
+    if (h->prep_bytes < dblast_prep_bytes(h)) return DBLAST_ERR_WORKSPACE;
+  }
+  return DBLAST_OK;
+}
+
+static dblast_status check_args(const dblast_head* h, const dblast_block_args* a) {
+  if (!a) return DBLAST_ERR_INVALID_ARG;
+  if (a->N < 1 || a->B < 1 || a->B > 32) return DBLAST_ERR_INVALID_ARG;
+  if (!(a->temperature > 0.f) || !(a->z_temperature >= 0.f)) return DBLAST_ERR_INVALID_ARG;
+  if (!a->hidden || !a->pos || !a->round) return DBLAST_ERR_INVALID_ARG;
+  if (!aligned16(a->hidden) || (a->anchor && !aligned16(a->anchor))) return DBLAST_ERR_INVALID_ARG;
+  if ((long long)a->N * a->B > (1LL << 24)) return DBLAST_ERR_INVALID_ARG;
+  if (a->impl == DBLAST_IMPL_TCGEN05 && !tc_supported(h)) return DBLAST_ERR_UNSUPPORTED;
+  if (a->impl != DBLAST_IMPL_AUTO && a->impl != DBLAST_IMPL_SIMT && a->impl != DBLAST_IMPL_TCGEN05)
+    return DBLAST_ERR_INVALID_ARG;
+  return DBLAST_OK;
+}
+
+static bool use_tc(const dblast_head* h, const dblast_block_args* a) {
+  if (a->impl == DBLAST_IMPL_SIMT) return false;
+  if (a->impl == DBLAST_IMPL_TCGEN05) return true;
+  return tc_supported(h);
+}
+
+static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, void* ws,
+                              size_t ws_bytes, int has_bonus, dblast_stream_t stream,
+                              StepCtx* c) {
+  if (!ws || !aligned16(ws)) return DBLAST_ERR_WORKSPACE;
+  if (ws_bytes < dblast_workspace_bytes(h, a->N, a->B, has_bonus)) return DBLAST_ERR_WORKSPACE;
+  c->head = h;
+  c->args = a;
+  c->has_e = h->e != nullptr;
+  c->pl = prep_layout(h->V, h->H, h->K, h->r, c->has_e);
+  c->wl = ws_layout(h->V, h->K, h->r, c->has_e, a->N, a->B, has_bonus);
+  c->ws = static_cast<unsigned char*>(ws);
+  c->prep = static_cast<const unsigned char*>(h->prep);
+  c->stream = reinterpret_cast<cudaStream_t>(stream);
+  c->k2 = LOG2E / a->temperature;
+  c->target = nullptr;
+  c->Bt = a->B + (has_bonus ? 1 : 0);
+  return DBLAST_OK;
+}
+
+static dblast_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return DBLAST_OK;
+  fprintf(stderr, "dblast: CUDA error %s\n", cudaGetErrorString(e));
+  return DBLAST_ERR_CUDA;
+}
+
+extern "C" {
+
+size_t dblast_prep_bytes(const dblast_head* h) {
+  if (!h || h->V < 1 || h->K < 1 || h->r < 1) return 0;
+  return prep_layout(h->V, h->H, h->K, h->r, h->e != nullptr).total;
+}
+
+size_t dblast_workspace_bytes(const dblast_head* h, int N, int B, int has_bonus) {
+  if (!h || N < 1 || B < 1 || h->V < 1 || h->K < 1 || h->r < 1) return 0;
+  return ws_layout(h->V, h->K, h->r, h->e != nullptr, N, B, has_bonus).total;
+}
+
+dblast_status dblast_head_prepare(const dblast_head* h, dblast_stream_t stream) {
+  dblast_status st = check_head(h, true);
+  if (st != DBLAST_OK) return st;
+  PrepLayout pl = prep_layout(h->V, h->H, h->K, h->r, h->e != nullptr);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(dbg(launch_prep(h, pl, s), "prep", s));
+}
+
+static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
+  g_calls.fetch_add(1, std::memory_order_relaxed);
+  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t),
+                                  c.stream);
+  if (e == cudaSuccess) e = dbg(launch_prior_codes(c), "prior_codes", c.stream);
+  if (e == cudaSuccess) {
+    pass_event_begin(0, c.stream);
+    e = use_tc(c.head, c.args) ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
+    pass_event_end(0, c.stream);
+    e = dbg(e, "draft_pass", c.stream);
+  }
+  if (e == cudaSuccess) e = dbg(launch_draft_finalize(c, out), "draft_finalize", c.stream);
+  return cuda_status(e);
+}
+
+static dblast_status verify_impl(StepCtx c, dblast_verify_out* out) {
+  c.target = out->target;
+  c.Bt = c.args->B + (out->has_bonus ? 1 : 0);
+  g_calls.fetch_add(1, std::memory_order_relaxed);
+  cudaError_t e = dbg(launch_target_stats(c, out), "target_stats", c.stream);
+  if (e == cudaSuccess) {
+    pass_event_begin(1, c.stream);
+    e = use_tc(c.head, c.args) ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
+    pass_event_end(1, c.stream);
+    e = dbg(e, "verify_pass", c.stream);
+  }
+  if (e == cudaSuccess) e = dbg(launch_verify_finalize(c, out), "verify_finalize", c.stream);
+  return cuda_status(e);
+}
+
+dblast_status dblast_draft_block(const dblast_head* h, const dblast_block_args* a,
+                                 dblast_draft_out* out, void* ws, size_t ws_bytes,
+                                 dblast_stream_t stream) {
+  dblast_status st = check_head(h, true);
+  if (st == DBLAST_OK) st = check_args(h, a);
+  if (st != DBLAST_OK) return st;
+  StepCtx c;
+  st = make_ctx(h, a, ws, ws_bytes, 1, stream, &c);
+  if (st != DBLAST_OK) return st;
+  return draft_impl(c, out);
+}
+
+dblast_status dblast_verify_block(const dblast_head* h, const dblast_block_args* a,
+                                  dblast_verify_out* out, void* ws, size_t ws_bytes,
+                                  dblast_stream_t stream) {
+  dblast_status st = check_head(h, true);
+  if (st == DBLAST_OK) st = check_args(h, a);
+  if (st != DBLAST_OK) return st;
+  if (!out || !out->target || !aligned16(out->target)) return DBLAST_ERR_INVALID_ARG;
+  StepCtx c;
+  st = make_ctx(h, a, ws, ws_bytes, out->has_bonus ? 1 : 0, stream, &c);
+  if (st != DBLAST_OK) return st;
+  return verify_impl(c, out);
+}
+
+dblast_status dblast_draft_and_verify(const dblast_head* h, const dblast_block_args* a,
+                                      dblast_draft_out* dout, dblast_verify_out* vout, void* ws,
+                                      size_t ws_bytes, dblast_stream_t stream) {
+  dblast_status st = check_head(h, true);
+  if (st == DBLAST_OK) st = check_args(h, a);
+  if (st != DBLAST_OK) return st;
+  if (!vout || !vout->target || !aligned16(vout->target)) return DBLAST_ERR_INVALID_ARG;
+  StepCtx c;
+  st = make_ctx(h, a, ws, ws_bytes, vout->has_bonus ? 1 : 0, stream, &c);
+  if (st != DBLAST_OK) return st;
+  st = draft_impl(c, dout);
+  if (st != DBLAST_OK) return st;
+  return verify_impl(c, vout);
+}
+
+dblast_status dblast_device_status(void* ws, dblast_stream_t stream) {
+  if (!ws) return DBLAST_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DevStatus hs{};
+  cudaError_t e = cudaMemcpyAsync(&hs, ws, sizeof(hs), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (hs.timeout) {
+    e = cudaMemsetAsync(ws, 0, sizeof(DevStatus), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_status(e);
+    return DBLAST_ERR_TIMEOUT;
+  }
+  return DBLAST_OK;
+}
+
+void dblast_set_wait_limit(uint32_t spins) { g_wait_limit = spins; }
+
+void dblast_stats_reset(int enable_pass_timing) {
+  std::lock_guard<std::mutex> lk(g_stats_mu);
+  g_launches = 0;
+  g_calls = 0;
+  g_n_ev[0] = g_n_ev[1] = 0;
+  g_timing = enable_pass_timing != 0;
+}
+
+dblast_status dblast_stats_get(dblast_stats* out) {
+  if (!out) return DBLAST_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_stats_mu);
+  out->calls = g_calls.load();
+  out->kernel_launches = g_launches.load();
+  double ms[2] = {0.0, 0.0};
+  for (int w = 0; w < 2; ++w) {
+    for (int i = 0; i < g_n_ev[w]; ++i) {
+      cudaError_t e = cudaEventSynchronize(g_ev[w][2 * i + 1]);
+      float t = 0.f;
+      if (e == cudaSuccess) e = cudaEventElapsedTime(&t, g_ev[w][2 * i], g_ev[w][2 * i + 1]);
+      if (e != cudaSuccess) return cuda_status(e);
+      ms[w] += t;
+    }
+  }
+  out->timed_draft = (uint64_t)g_n_ev[0];
+  out->timed_verify = (uint64_t)g_n_ev[1];
+  out->draft_pass_ms = ms[0];
+  out->verify_pass_ms = ms[1];
+  return DBLAST_OK;
+}
+
+const char* dblast_status_string(dblast_status s) {
+  switch (s) {
+    case DBLAST_OK: return "ok";
+    case DBLAST_ERR_INVALID_ARG: return "invalid argument";
+    case DBLAST_ERR_UNSUPPORTED: return "unsupported shape or dtype for the requested implementation";
+    case DBLAST_ERR_WORKSPACE: return "prep or workspace buffer too small or misaligned";
+    case DBLAST_ERR_CUDA: return "CUDA runtime error";
+    case DBLAST_ERR_TIMEOUT: return "device-side wait ran out";
+    case DBLAST_ERR_NO_DEVICE: return "no usable device";
+  }
+  return "unknown status";
+}
+
+const char* dblast_version(void) { return "dblast 0.1 (sm_103a)"; }
+
+}  // extern "C"

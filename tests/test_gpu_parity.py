@@ -1,0 +1,141 @@
+"""GPU parity: the CUDA step through the C ABI against the fp64 oracle.
+
+Every case draws seeded synthetic inputs (synth/), runs
+dblast_draft_and_verify on cuda:0 and the oracle on the CPU, and compares
+with tests/parity.py's rules: integer decisions bit-exact except counted
+threshold ties, probabilities / overlaps / expected lengths within 1e-4
+relative.
+"""
+import pytest
+import torch
+
+import synth
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+IMPLS = ["simt"]
+
+
+def _case(cfg, T, Z_T, seed, impl, seqs=None, round_idx=0, device="cuda"):
+    head = synth.make_head(cfg, device)
+    blk = synth.make_block(cfg, head, round_idx, device)
+    pos, rnd = synth.initial_state(cfg, device)
+    pos0, rnd0 = pos.clone(), rnd.clone()
+    gpu = parity.run_gpu(head, blk, T, Z_T, seed, pos, rnd, impl=impl)
+    seqs = list(range(cfg["N"])) if seqs is None else seqs
+    orc = parity.run_oracle(head, blk, T, Z_T, seed, pos0, rnd0, seqs)
+    stats = parity.compare(gpu, orc, seqs)
+    # state update: pos += n_emitted, round += 1
+    assert torch.equal(pos.cpu(), pos0.cpu() + gpu["n_emitted"].long())
+    assert torch.equal(rnd.cpu(), rnd0.cpu() + 1)
+    return stats
+
+
+def _skip_unsupported(cfg, impl):
+    if impl == "tcgen05" and not (cfg["dtype"] == "bf16" and cfg["H"] % 64 == 0):
+        pytest.skip("tensor-core path needs bf16 and H % 64 == 0")
+
+
+@pytest.mark.parametrize("T,Z_T", [(1.0, 1.0), (0.6, 1.0), (1.5, 0.0)])
+def test_tiny_config_all_sequences(T, Z_T):
+    cfg = synth.config("tiny")
+    st = _case(cfg, T, Z_T, seed=0, impl="auto")
+    assert st["sequences"] == 8
+
+
+SMALL = {
+    # ragged vocabulary tail, expander bias, Zipf bias
+    "ragged_e": dict(base="qwen3_8b_b32", V=1000, H=64, K=3, r=4, B=5, N=6,
+                     expander_bias=True, sigma=0.7),
+    # argmax prior, block of 16, 8 components
+    "zt0": dict(base="qwen3_8b_b32", V=4099, H=128, K=8, r=16, B=16, N=3),
+    # independent baseline K = 1 with B = 1
+    "k1_b1": dict(base="qwen3_8b_b32", V=2048, H=64, K=1, r=8, B=1, N=5),
+    # fp32, no bonus row, B = 32
+    "f32_b32": dict(base="tiny", V=777, H=32, K=2, r=2, B=32, N=2, bonus=False),
+    # many components, rank 32
+    "k16_r32": dict(base="sweep_k16", V=3000, H=128, B=4, N=4),
+}
+SMALL_T = {"ragged_e": (0.8, 1.0), "zt0": (1.0, 0.0), "k1_b1": (1.5, 1.0),
+           "f32_b32": (1.0, 0.7), "k16_r32": (0.7, 1.0)}
+
+
+@pytest.mark.parametrize("impl", IMPLS)
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_small_shapes(name, impl):
+    over = dict(SMALL[name])
+    cfg = synth.config(over.pop("base"), **over)
+    _skip_unsupported(cfg, impl)
+    T, Z_T = SMALL_T[name]
+    for seed in (1, 2):
+        _case(cfg, T, Z_T, seed=seed, impl=impl)
+
+
+@pytest.mark.parametrize("impl", IMPLS)
+def test_four_rounds_carry_state(impl):
+    from paper_2608_05448_gb300 import Head, Workspace
+    cfg = synth.config("qwen3_8b_b32", V=2500, H=128, K=4, r=8, B=6, N=7)
+    _skip_unsupported(cfg, impl)
+    head_t = synth.make_head(cfg, "cuda")
+    head = Head.from_dict(head_t)
+    ws = Workspace(head, cfg["N"], cfg["B"], True)
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    for rd in range(4):
+        blk = synth.make_block(cfg, head_t, rd, "cuda")
+        pos0, rnd0 = pos.clone(), rnd.clone()
+        gpu = parity.run_gpu(head_t, blk, 1.0, 1.0, 11, pos, rnd, impl=impl, head=head, ws=ws)
+        orc = parity.run_oracle(head_t, blk, 1.0, 1.0, 11, pos0, rnd0, list(range(cfg["N"])))
+        parity.compare(gpu, orc, list(range(cfg["N"])))
+        assert torch.equal(pos.cpu(), pos0.cpu() + gpu["n_emitted"].long())
+        assert torch.equal(rnd.cpu(), rnd0.cpu() + 1)
+    assert int(rnd[0]) == 4
+
+
+def test_target_equal_to_drafter_accepts_every_token():
+    """K = 1 and t = drafter logits (fp32): p = q, alpha = 1, all B accepted."""
+    from oracle import dblast_oracle as orc
+    cfg = synth.config("tiny", V=500, H=32, K=1, r=2, B=6, N=4)
+    head = synth.make_head(cfg, "cuda")
+    blk = synth.make_block(cfg, head, 0, "cuda")
+    hd = orc.prepare_head(head)
+    rows = []
+    for n in range(cfg["N"]):
+        h = orc.f64(blk["hidden"][n])
+        l = orc.component_logits(head["W"], orc.branch_hidden(h, hd["U"], hd["Vf"], None),
+                                 None)[:, 0, :]
+        rows.append(torch.cat([torch.tensor(l), torch.tensor(l[:1])], 0))
+    blk["target"] = torch.stack(rows).float().cuda().contiguous()
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    gpu = parity.run_gpu(head, blk, 0.9, 1.0, 5, pos, rnd)
+    assert (gpu["accepted"] == cfg["B"]).all()
+    assert torch.allclose(gpu["alpha"], torch.ones_like(gpu["alpha"]), atol=1e-5)
+    assert torch.allclose(gpu["exp_len"], torch.full_like(gpu["exp_len"], cfg["B"]), atol=1e-4)
+
+
+def test_disjoint_target_rejects_first_token():
+    cfg = synth.config("qwen3_8b_b32", V=1500, H=64, K=2, r=4, B=4, N=6)
+    head = synth.make_head(cfg, "cuda")
+    blk = synth.make_block(cfg, head, 0, "cuda")
+    blk["target"] = (-4.0 * blk["target"].float()).to(torch.bfloat16).contiguous()
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    pos0, rnd0 = pos.clone(), rnd.clone()
+    gpu = parity.run_gpu(head, blk, 1.0, 1.0, 3, pos, rnd)
+    assert (gpu["accepted"] == 0).sum() >= 4
+    orc = parity.run_oracle(head, blk, 1.0, 1.0, 3, pos0, rnd0, list(range(cfg["N"])))
+    parity.compare(gpu, orc, list(range(cfg["N"])))
+
+
+@pytest.mark.parametrize("impl", IMPLS)
+def test_qwen3_4b_single_sequence_full(impl):
+    cfg = synth.config("qwen3_4b_b1")
+    _skip_unsupported(cfg, impl)
+    _case(cfg, 1.0, 1.0, seed=0, impl=impl)
+
+
+@pytest.mark.parametrize("impl", IMPLS)
+@pytest.mark.parametrize("T", [1.0, 0.6])
+def test_qwen3_8b_batched_sampled(impl, T):
+    cfg = synth.config("qwen3_8b_b32")
+    _skip_unsupported(cfg, impl)
+    _case(cfg, T, 1.0, seed=0, impl=impl, seqs=[0, 31])

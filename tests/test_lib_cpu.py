@@ -1,0 +1,101 @@
+"""Host-side checks of libdblast that need no GPU: it builds, loads, exports
+every entry point declared in include/dblast.h, sizes its buffers and rejects
+bad arguments before any CUDA call."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_05448_gb300 import binding as bd
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "dblast.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dblast_[a-z_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_function():
+    names = header_functions()
+    assert len(names) >= 10
+    lib = bd.lib()
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(bd.EXPORTS)
+    assert lib.dblast_version().startswith(b"dblast")
+
+
+def fake_head(V=151936, H=4096, K=8, r=16, e=False):
+    p = ctypes.c_void_p(1 << 20)  # 16-byte aligned placeholder, never dereferenced
+    return bd.CHead(V, H, K, r, 0, p, p, p, p if e else None, p, None, None, p, 0)
+
+
+def test_prep_and_workspace_sizes():
+    lib = bd.lib()
+    h = fake_head()
+    prep = lib.dblast_prep_bytes(ctypes.byref(h))
+    V, K, rr = 151936, 8, 16
+    assert prep >= V * K * rr * 4 + V * K * 2 * 16 * 2
+    he = fake_head(e=True)
+    assert lib.dblast_prep_bytes(ctypes.byref(he)) > prep   # r+1 -> padded to 32
+    ws = lib.dblast_workspace_bytes(ctypes.byref(h), 32, 16, 1)
+    assert ws >= 32 * 16 * V * 4            # fp32 stash of the base logits
+    assert ws < 32 * 16 * V * 4 * 1.35      # everything else is small next to it
+    assert lib.dblast_workspace_bytes(ctypes.byref(h), 32, 16, 0) == ws
+
+
+def _args(N=2, B=3, T=1.0, zt=1.0):
+    p = ctypes.c_void_p(1 << 20)
+    return bd.CBlockArgs(N, B, T, zt, 0, p, None, p, p, 0)
+
+
+@pytest.mark.parametrize("mutate,status", [
+    (lambda h, a: setattr(h, "K", 0), 1),
+    (lambda h, a: setattr(h, "K", 33), 1),
+    (lambda h, a: setattr(h, "r", 65), 1),
+    (lambda h, a: setattr(h, "H", 12), 1),
+    (lambda h, a: setattr(h, "W", None), 1),
+    (lambda h, a: setattr(h, "W", 1 << 20 | 4), 1),
+    (lambda h, a: setattr(a, "B", 33), 1),
+    (lambda h, a: setattr(a, "N", 0), 1),
+    (lambda h, a: setattr(a, "temperature", 0.0), 1),
+    (lambda h, a: setattr(a, "z_temperature", -1.0), 1),
+    (lambda h, a: setattr(a, "hidden", None), 1),
+    (lambda h, a: setattr(h, "prep_bytes", 0), 3),
+])
+def test_bad_arguments_are_rejected_before_launch(mutate, status):
+    lib = bd.lib()
+    h = fake_head(V=1000, H=64, K=4, r=8)
+    h.prep_bytes = lib.dblast_prep_bytes(ctypes.byref(h))
+    a = _args()
+    mutate(h, a)
+    d = bd.CDraftOut()
+    ws = ctypes.c_void_p(1 << 20)
+    got = lib.dblast_draft_block(ctypes.byref(h), ctypes.byref(a), ctypes.byref(d), ws,
+                                 1 << 40, None)
+    assert got == status
+
+
+def test_workspace_too_small_is_rejected():
+    lib = bd.lib()
+    h = fake_head(V=1000, H=64, K=4, r=8)
+    h.prep_bytes = lib.dblast_prep_bytes(ctypes.byref(h))
+    a = _args()
+    need = lib.dblast_workspace_bytes(ctypes.byref(h), 2, 3, 1)
+    d = bd.CDraftOut()
+    got = lib.dblast_draft_block(ctypes.byref(h), ctypes.byref(a), ctypes.byref(d),
+                                 ctypes.c_void_p(1 << 20), need - 1, None)
+    assert got == 3
+    v = bd.CVerifyOut()
+    got = lib.dblast_verify_block(ctypes.byref(h), ctypes.byref(a), ctypes.byref(v),
+                                  ctypes.c_void_p(1 << 20), need, None)
+    assert got == 1   # verify needs target logits
+
+
+def test_status_strings():
+    lib = bd.lib()
+    for s in range(7):
+        assert lib.dblast_status_string(s)
