@@ -182,6 +182,29 @@ typedef struct {
 void dblast_stats_reset(int enable_pass_timing);
 dblast_status dblast_stats_get(dblast_stats* out);
 
+/* No-allocation variant of the target log-sum-exp pass.  The paper has no
+ * counterpart; this is a service for callers that cannot allocate device
+ * memory when they call in, such as a plugin run inside another engine's
+ * enqueue step (cudaMalloc would synchronise the device and bypass that
+ * engine's memory pool) or code with a fixed device-memory budget.
+ *
+ *   lse_out[row] = log sum_v exp(target[row, v] / temperature)
+ *
+ * target: [rows, V] logits of `dtype` (device); lse_out: [rows] fp32 (device).
+ * Its only scratch is a static device array of DBLAST_NOALLOC_MAX_RECORDS
+ * 8-byte records (8 MiB on every GPU that loads the library, held until the
+ * process exits); rows * ceil(V / 128) must not exceed it, otherwise
+ * DBLAST_ERR_WORKSPACE is returned and nothing is launched.  It calls no
+ * allocation routine.  The first call on a device, with that device current,
+ * looks up the array's device address (cudaGetSymbolAddress); make that first
+ * call before any stream capture.  `stream` must belong to the current
+ * device.  Every call reuses the same array, so calls that overlap on the GPU
+ * (other streams or threads) race; serialise them. */
+#define DBLAST_NOALLOC_MAX_RECORDS (1u << 20)
+dblast_status dblast_target_lse_noalloc(const void* target, int rows, int V, dblast_dtype dtype,
+                                        float temperature, float* lse_out,
+                                        dblast_stream_t stream);
+
 const char* dblast_status_string(dblast_status s);
 const char* dblast_version(void);
 

@@ -67,7 +67,7 @@ class CVerifyOut(ctypes.Structure):
 EXPORTS = ["dblast_prep_bytes", "dblast_workspace_bytes", "dblast_head_prepare",
            "dblast_draft_block", "dblast_verify_block", "dblast_draft_and_verify",
            "dblast_device_status", "dblast_set_wait_limit", "dblast_stats_reset",
-           "dblast_stats_get", "dblast_status_string",
+           "dblast_stats_get", "dblast_target_lse_noalloc", "dblast_status_string",
            "dblast_version"]
 
 
@@ -105,6 +105,10 @@ def load_library(path=None, build_if_missing=True):
     lib.dblast_stats_reset.restype = None
     lib.dblast_stats_get.argtypes = [P(CStats)]
     lib.dblast_stats_get.restype = ctypes.c_int
+    lib.dblast_target_lse_noalloc.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_int, ctypes.c_float, ctypes.c_void_p,
+                                              ctypes.c_void_p]
+    lib.dblast_target_lse_noalloc.restype = ctypes.c_int
     lib.dblast_status_string.argtypes = [ctypes.c_int]
     lib.dblast_status_string.restype = ctypes.c_char_p
     lib.dblast_version.argtypes = []
@@ -311,3 +315,21 @@ def dblast_stats_get():
     st = CStats()
     _check(lib().dblast_stats_get(ctypes.byref(st)), "dblast_stats_get")
     return {k: getattr(st, k) for k, _ in CStats._fields_}
+
+
+NOALLOC_MAX_RECORDS = 1 << 20
+
+
+def dblast_target_lse_noalloc(target, temperature, lse_out):
+    """Natural log-sum-exp of target / T per row through the no-allocation
+    entry point: its only scratch is the library's static device array, and
+    the caller provides the output.  target: CUDA [..., V] bf16/fp32 logits;
+    lse_out: CUDA fp32 with one entry per row.  Returns the C status code."""
+    _cuda_contig(target, "target")
+    _cuda_contig(lse_out, "lse_out", torch.float32)
+    V = target.shape[-1]
+    rows = target.numel() // V
+    if lse_out.numel() != rows:
+        raise ValueError("lse_out must have one entry per row")
+    return lib().dblast_target_lse_noalloc(_ptr(target), rows, V, DTYPES[target.dtype],
+                                           float(temperature), _ptr(lse_out), _stream())
