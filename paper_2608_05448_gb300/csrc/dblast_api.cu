@@ -77,7 +77,6 @@ void pass_event_end(int which, cudaStream_t s) {
 }
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e) {
-  (void)H;
   PrepLayout p{};
   p.V = V;
   p.K = K;
@@ -91,6 +90,10 @@ PrepLayout prep_layout(int V, int H, int K, int r, bool has_e) {
   o = align_up(o + (size_t)V * p.KC * sizeof(__half), 256);
   p.off_sw = o;
   o = align_up(o + (size_t)K * sizeof(float), 256);
+  p.off_ut = o;
+  o = align_up(o + (size_t)ceil_div(K * p.rr, MTILE) * MTILE * H * 2, 256);
+  p.off_status = o;
+  o = align_up(o + sizeof(DevStatus), 256);
   p.total = o;
   return p;
 }
@@ -138,7 +141,6 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
 
 cudaError_t launch_draft_pass_tc(const StepCtx& c);
 cudaError_t launch_verify_pass_tc(const StepCtx& c);
-bool tc_supported(const dblast_head* h);
 
 }  // namespace dblast
 

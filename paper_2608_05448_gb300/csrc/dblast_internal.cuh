@@ -30,10 +30,12 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 // ---------------------------------------------------------------- layouts
 struct PrepLayout {
   int V, K, rr, rp, KC;    // rr = r + (e != NULL); rp = rr rounded up to 16; KC = K*2*rp
-  size_t off_wu, off_wuop, off_sw, total;
+  size_t off_wu, off_wuop, off_sw, off_ut, off_status, total;
   // WU   fp32 [V, K, rr]: (W U_z)_v and, if e, (W e_z)_v in column r
   // WUop fp16 [V, KC]   : per z, [hi(rp) | lo(rp)] of WU_z * sw[z]
   // sw   fp32 [K]       : power-of-two scale of WUop's z block
+  // ut   bf16 [rows_pad, H]: [U_z | e_z]^T, the A operand of the tensor-core prep
+  // status DevStatus      : bounded-wait record of the tensor-core prep
 };
 
 // Workspace regions (each 256-byte aligned), with their element types:
@@ -158,6 +160,8 @@ void pass_event_begin(int which, cudaStream_t s);  // which: 0 draft pass, 1 ver
 void pass_event_end(int which, cudaStream_t s);
 
 cudaError_t launch_prep(const dblast_head* head, const PrepLayout& pl, cudaStream_t s);
+cudaError_t launch_prep_tc(const dblast_head* head, const PrepLayout& pl, cudaStream_t s);
+bool tc_supported(const dblast_head* h);
 cudaError_t launch_prior_codes(const StepCtx& c);
 cudaError_t launch_draft_pass_simt(const StepCtx& c);
 cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* out);

@@ -8,6 +8,8 @@
 // as split-fp16 operands for the tensor-core correction GEMM: for every z the
 // operand row is [hi(rp) | lo(rp)] of WU_z * sw_z, sw_z a power of two that
 // brings max|WU_z| near 2^14 (hi + lo carries 22 bits of mantissa).
+#include <cstdlib>
+
 #include "dblast_internal.cuh"
 
 namespace dblast {
@@ -133,11 +135,18 @@ static cudaError_t prep_typed(const dblast_head* h, const PrepLayout& pl, cudaSt
   const int Nb = h->K * pl.rr;
   ExpanderCols<Tin> bf{static_cast<const Tin*>(h->U), static_cast<const Tin*>(h->e), h->H, h->r,
                        pl.rr};
-  dim3 grid(ceil_div(h->V, 64), ceil_div(Nb, 64), 1);
-  k_gemm_simt<Tin><<<grid, 256, 0, s>>>(static_cast<const Tin*>(h->W), h->V, h->H, bf, Nb, h->H,
-                                        wu, 0);
-  debug_kernel("k_gemm_simt", s);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = cudaSuccess;
+  const char* force_simt = getenv("DBLAST_PREP_SIMT");  // test hook: compare the two prep GEMMs
+  if (tc_supported(h) && !(force_simt && force_simt[0] == '1')) {
+    e = launch_prep_tc(h, pl, s);
+  } else {
+    dim3 grid(ceil_div(h->V, 64), ceil_div(Nb, 64), 1);
+    k_gemm_simt<Tin><<<grid, 256, 0, s>>>(static_cast<const Tin*>(h->W), h->V, h->H, bf, Nb,
+                                          h->H, wu, 0);
+    debug_kernel("k_gemm_simt", s);
+    count_launches(1);
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess) return e;
   e = cudaMemsetAsync(sw, 0, h->K * sizeof(float), s);
   if (e != cudaSuccess) return e;
@@ -148,7 +157,7 @@ static cudaError_t prep_typed(const dblast_head* h, const PrepLayout& pl, cudaSt
   debug_kernel("k_prep_split", s);
   k_prep_scale<<<1, 32, 0, s>>>(sw, h->K);
   debug_kernel("k_prep_scale", s);
-  count_launches(4);
+  count_launches(3);
   return cudaGetLastError();
 }
 

@@ -1,21 +1,679 @@
-// Tensor-core (tcgen05 / TMEM / TMA) passes for sm_103a.
+// Tensor-core passes for sm_103a: tcgen05.mma with fp32 accumulators in TMEM,
+// operands staged in shared memory by TMA (cp.async.bulk.tensor, 128-byte
+// swizzle), mbarrier pipelines, one persistent CTA per SM.
+//
+// Draft pass (rows a2+a3 of the step).  For a tile of 128 positions (TMEM
+// lanes) x 128 vocabulary tokens (TMEM columns):
+//   base    D_b  = h . W^T                        (bf16 x bf16, K = H)
+//   branch  D_z  = c_z . WU_z^T   for z < K        (split fp16: hi.hi + hi.lo + lo.hi)
+//   l_{m,z,v} = D_b + D_z / (sc_{m,z} sw_z) + b_v, s = l log2(e) / T
+// and the epilogue warps reduce every (m, z) row of the tile to a (max, sum)
+// record of 2^s, stash W h + b in fp32 and never write the branch logits.
+// The branch GEMMs of tile t are interleaved with the base GEMM of tile t+1
+// so the epilogue of one tile overlaps the main loop of the next.
+//
+// Prep pass (row a0): the same machinery with only the base GEMM computes
+// WU = [U_z | e_z]^T . W^T and stores it as fp32 [V, K, rr].
+#include <cuda.h>
+
 #include "dblast_internal.cuh"
 
 namespace dblast {
 
+uint32_t wait_limit();
+
+namespace tc {
+
+constexpr int BM = 128;            // rows per tile (TMEM lanes)
+constexpr int BN = 128;            // vocabulary tokens per tile (TMEM columns)
+constexpr int BK = 64;             // elements per stage row (128 bytes, SW128 atom)
+constexpr int STAGES = 5;
+constexpr int STAGE_A = BM * BK * 2;   // 16 KB
+constexpr int STAGE_B = BN * BK * 2;   // 16 KB
+constexpr int STAGE_BYTES = STAGE_A + STAGE_B;
+constexpr int KMAX = 16;           // components supported by the tensor-core path
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int NUM_THREADS = 32 * (2 + NUM_EPI_WARPS);
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int RED_BYTES = KMAX * 2 * BM * 8;   // [z][half][row] (max, sum)
+
+enum Mode { MODE_PREP = 0, MODE_DRAFT = 1 };
+
+// ------------------------------------------------------------------ PTX
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Shared state of the roles: every wait is bounded; a wait that runs out
+// raises `abort` so that the other roles leave their loops too.
+struct Ctl {
+  uint32_t spin_limit;        // 0: time bound only
+  volatile int* abort;        // shared flag
+  DevStatus* status;          // global status word
+};
+
+__device__ __noinline__ void record_timeout(const Ctl& c, uint32_t where) {
+  *c.abort = 1;
+  atomicExch(&c.status->timeout, 1u);
+  atomicExch(&c.status->where, where);
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const Ctl& c,
+                                          uint32_t where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*c.abort) return false;
+    if ((c.spin_limit && i >= c.spin_limit) || (globaltimer() - t0) > 2000000000ull) {
+      record_timeout(c, where);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// K-major operand in a 128-byte-swizzled tile: rows of 128 bytes, 8-row
+// groups 1024 bytes apart; the start address moves by 32 bytes per 16-element
+// K step inside the row.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1) << 16;                 // leading byte offset (unused here)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;         // stride byte offset: 8 rows
+  d |= static_cast<uint64_t>(1) << 46;                 // descriptor version for tcgen05
+  d |= static_cast<uint64_t>(2) << 61;                 // 128-byte swizzle
+  return d;
+}
+
+// instruction descriptor, kind::f16: fp32 accumulate, A/B both bf16 or both
+// fp16, both K-major, M = 128, N = BN
+__host__ __device__ constexpr uint32_t idesc_f16(bool bf16) {
+  return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) |
+         (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                     uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ------------------------------------------------------------ parameters
+struct Params {
+  int mode;
+  int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles
+  int nb;                    // base stages per tile (H / BK)
+  int ncs;                   // branch stages per tile (KC / BK); 0 in prep mode
+  int K, rp, zps;            // components, padded rank, components per branch stage
+  int M, V, Mpad;            // valid rows, vocabulary, padded rows
+  float k2;                  // log2(e) / T
+  const float* vbias;        // [V] or null
+  const float* cscale;       // [Mpad, K]
+  const float* sw;           // [K]
+  float* stash;              // [M, V]
+  float2* partd;             // [nt, K, Mpad]
+  float* wu;                 // prep output [V, rows_total]
+  int prep_rows;             // K * rr in prep mode
+  DevStatus* status;
+  uint32_t spin_limit;
+};
+
+// The item sequence consumed by the MMA warp and produced by the TMA warp:
+// for tile slot s = 0 .. my_tiles, base stages of tile s with the branch
+// stages of tile s-1 spread between them (after the last tile: the branch
+// stages of the last tile).
+__device__ __forceinline__ int ins_point(int c, int nb, int ncs) {
+  return ((c + 1) * nb) / (ncs + 1);
+}
+
+__device__ __forceinline__ void tile_of(const Params& P, int slot, int* mt, int* vt) {
+  const int t = (int)blockIdx.x + slot * (int)gridDim.x;
+  *vt = t / P.n_mt;
+  *mt = t - *vt * P.n_mt;
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+              const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
+              const Params P) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* stage_base = smem;
+  float2* red = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + RED_BYTES);
+  uint64_t* full = bars;                 // [STAGES]
+  uint64_t* empty = bars + STAGES;       // [STAGES]
+  uint64_t* bfull = bars + 2 * STAGES;   // [2] base accumulator ready
+  uint64_t* bempty = bfull + 2;          // [2] base accumulator free
+  uint64_t* cfull = bfull + 4;           // [2] branch accumulator ready
+  uint64_t* cempty = bfull + 6;          // [2] branch accumulator free
+  uint64_t* done = bfull + 8;            // [1] all MMAs of this CTA finished
+  uint64_t* redw = bfull + 9;            // [1] all epilogue records of a tile written
+  uint64_t* redm = bfull + 10;           // [1] all records of a tile merged
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 11);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int my_tiles = (P.n_tiles > (int)blockIdx.x)
+                           ? (P.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
+                           : 0;
+  Ctl ctl{P.spin_limit, abort_flag, P.status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bfull[b], 1);
+      mbar_init(&bempty[b], NUM_EPI_WARPS);
+      mbar_init(&cfull[b], 1);
+      mbar_init(&cempty[b], NUM_EPI_WARPS);
+    }
+    mbar_init(done, 1);
+    mbar_init(redw, 32 * NUM_EPI_WARPS);
+    mbar_init(redm, 32 * NUM_EPI_WARPS);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0u, issued_phase = 0u;  // per stage: issued at least once / its parity
+      bool ok = true;
+      for (int slot = 0; slot <= my_tiles && ok; ++slot) {
+        const int nbv = (slot < my_tiles) ? P.nb : 0;
+        const int ncv = (slot >= 1) ? P.ncs : 0;
+        int mt = 0, vt = 0, pmt = 0, pvt = 0;
+        if (slot < my_tiles) tile_of(P, slot, &mt, &vt);
+        if (slot >= 1) tile_of(P, slot - 1, &pmt, &pvt);
+        int c = 0;
+        for (int j = 0; j < nbv + ncv && ok; ++j) {
+          // decide the next item: base stage or branch stage
+          bool is_base;
+          int jb = j - c;  // base stages emitted so far
+          if (jb >= nbv) is_base = false;
+          else if (c < ncv && jb == ins_point(c, nbv, ncv) && nbv > 0) is_base = false;
+          else is_base = true;
+          if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) { ok = false; break; }
+          unsigned char* sa = stage_base + stage * STAGE_BYTES;
+          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          if (is_base) {
+            tma_load_2d(sa, &tm_a, &full[stage], jb * BK, mt * BM);
+            tma_load_2d(sa + STAGE_A, &tm_b, &full[stage], jb * BK, vt * BN);
+          } else {
+            tma_load_2d(sa, &tm_ca, &full[stage], c * BK, pmt * BM);
+            tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, pvt * BN);
+            ++c;
+          }
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // copies still in flight after an abort: wait (bounded) before leaving
+      for (int s = 0; s < STAGES; ++s)
+        if (issued_mask & (1u << s)) {
+          const uint64_t t0 = globaltimer();
+          while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
+                 (globaltimer() - t0) < 2000000000ull) {
+          }
+        }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t id_base = idesc_f16(true);
+      const uint32_t id_corr = idesc_f16(false);
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t cuse0 = 0u, cuse1 = 0u;  // uses of the two branch accumulators
+      bool ok = true;
+      for (int slot = 0; slot <= my_tiles && ok; ++slot) {
+        const int nbv = (slot < my_tiles) ? P.nb : 0;
+        const int ncv = (slot >= 1) ? P.ncs : 0;
+        const int bb = slot & 1;
+        const uint32_t bcol = tmem + (uint32_t)(bb * BN);
+        int c = 0;
+        for (int j = 0; j < nbv + ncv && ok; ++j) {
+          bool is_base;
+          const int jb = j - c;
+          if (jb >= nbv) is_base = false;
+          else if (c < ncv && jb == ins_point(c, nbv, ncv) && nbv > 0) is_base = false;
+          else is_base = true;
+          if (is_base && jb == 0) {
+            if (!mbar_wait(&bempty[bb], (((uint32_t)slot >> 1) & 1u) ^ 1u, ctl, 2)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          if (!mbar_wait(&full[stage], phase, ctl, 3)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(stage_base + stage * STAGE_BYTES);
+          const uint32_t sb = sa + STAGE_A;
+          if (is_base) {
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              umma(bcol, sdesc(sa + k * 32), sdesc(sb + k * 32), id_base,
+                   (jb > 0 || k > 0) ? 1u : 0u);
+            umma_commit(&empty[stage]);
+            if (jb == nbv - 1) umma_commit(&bfull[bb]);
+          } else {
+            // branch stage c of the previous tile: components z0 .. z0+zps-1
+            const int z0 = c * P.zps;
+            for (int zz = 0; zz < P.zps && z0 + zz < P.K && ok; ++zz) {
+              const int z = z0 + zz;
+              const int cs = z & 1;
+              const uint32_t use = cs ? cuse1 : cuse0;
+              if (!mbar_wait(&cempty[cs], (use & 1u) ^ 1u, ctl, 4)) { ok = false; break; }
+              tc_fence_after();
+              const uint32_t ccol = tmem + 2u * BN + (uint32_t)(cs * BN);
+              const int o = zz * 2 * P.rp;  // element offset of this component in the stage
+              int first = 1;
+              for (int kk = 0; kk < P.rp; kk += 16) {
+                const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
+                umma(ccol, sdesc(sa + hi), sdesc(sb + hi), id_corr, first ? 0u : 1u);
+                umma(ccol, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
+                umma(ccol, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
+                first = 0;
+              }
+              umma_commit(&cfull[cs]);
+              if (cs) ++cuse1; else ++cuse0;
+            }
+            umma_commit(&empty[stage]);
+            ++c;
+          }
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // wait (bounded) for every MMA this thread issued before TMEM is freed
+      umma_commit(done);
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
+      }
+    }
+  } else {
+    // ------------------------------------------------------ epilogue warps
+    const int ew = warp - 2;
+    const int q = warp & 3;          // TMEM lane quarter of this warp
+    const int half = ew >> 2;        // which 64 columns of the tile
+    const int row = q * 32 + lane;   // row of the tile
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint32_t cuse0 = 0u, cuse1 = 0u;
+    for (int slot = 0; slot < my_tiles; ++slot) {
+      int mt, vt;
+      tile_of(P, slot, &mt, &vt);
+      const int bb = slot & 1;
+      if (!mbar_wait(&bfull[bb], ((uint32_t)slot >> 1) & 1u, ctl, 5)) break;
+      tc_fence_after();
+      const int m = mt * BM + row;
+      const int v0 = vt * BN + half * 64;
+      float bk[64];
+      {
+        float t[32];
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          tmem_ld32(tmem + lane_off + (uint32_t)(bb * BN + half * 64 + cc * 32), t);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) bk[cc * 32 + j] = t[j];
+        }
+      }
+      // base accumulator is in registers: hand the TMEM buffer back
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bempty[bb]);
+
+      if (P.mode == MODE_PREP) {
+        // WU[v][row] for rows < prep_rows
+        if (m < P.prep_rows) {
+#pragma unroll
+          for (int j = 0; j < 64; ++j) {
+            const int v = v0 + j;
+            if (v < P.V) P.wu[(size_t)v * P.prep_rows + m] = bk[j];
+          }
+        }
+        continue;
+      }
+
+      // draft: b_v, stash, scale by log2(e)/T
+      const bool full_vec = (v0 + 64 <= P.V) && ((P.V & 3) == 0);
+#pragma unroll
+      for (int j = 0; j < 64; ++j) {
+        const int v = v0 + j;
+        if (P.vbias && v < P.V) bk[j] += __ldg(P.vbias + v);
+      }
+      if (m < P.M) {
+        float* srow = P.stash + (size_t)m * P.V + v0;
+        if (full_vec) {
+#pragma unroll
+          for (int j = 0; j < 64; j += 4)
+            *reinterpret_cast<float4*>(srow + j) = make_float4(bk[j], bk[j + 1], bk[j + 2], bk[j + 3]);
+        } else {
+          for (int j = 0; j < 64; ++j)
+            if (v0 + j < P.V) srow[j] = bk[j];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 64; ++j) bk[j] = (v0 + j < P.V) ? bk[j] * P.k2 : -INFINITY;
+
+      // the previous tile's records must be merged before they are overwritten
+      if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 7)) break;
+      bool ok = true;
+      for (int z = 0; z < P.K; ++z) {
+        const int cs = z & 1;
+        const uint32_t use = cs ? cuse1 : cuse0;
+        if (!mbar_wait(&cfull[cs], use & 1u, ctl, 6)) { ok = false; break; }
+        if (cs) ++cuse1; else ++cuse0;
+        tc_fence_after();
+        const float a = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
+        float M2 = -INFINITY, S = 0.f;
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          float cr[32];
+          tmem_ld32(tmem + lane_off + (uint32_t)(2 * BN + cs * BN + half * 64 + cc * 32), cr);
+          float mx = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            cr[j] = fmaf(cr[j], a, bk[cc * 32 + j]);
+            mx = fmaxf(mx, cr[j]);
+          }
+          const float Mn = fmaxf(M2, mx);
+          if (Mn != -INFINITY) {
+            float acc = 0.f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) acc += exp2f(cr[j] - Mn);
+            S = S * exp2f(M2 - Mn) + acc;
+            M2 = Mn;
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&cempty[cs]);
+        red[((size_t)z * 2 + half) * BM + row] = make_float2(M2, S);
+      }
+      if (!ok) break;
+      // merge the two column halves of every (row, z) and write the records
+      mbar_arrive(redw);
+      if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 8)) break;
+      for (int z = half; z < P.K; z += 2) {
+        const float2 p0 = red[((size_t)z * 2) * BM + row];
+        const float2 p1 = red[((size_t)z * 2 + 1) * BM + row];
+        const float mz = fmaxf(p0.x, p1.x);
+        float2 out = make_float2(-INFINITY, 0.f);
+        if (mz != -INFINITY)
+          out = make_float2(mz, p0.y * exp2f(p0.x - mz) + p1.y * exp2f(p1.x - mz));
+        P.partd[((size_t)vt * P.K + z) * P.Mpad + m] = out;
+      }
+      mbar_arrive(redm);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(TMEM_COLS));
+  }
+}
+
+// --------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D K-major tile map: rows x cols elements of 2 bytes, box 128 rows x 64
+static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, bool bf16) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
+                  const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+static int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+static size_t smem_bytes() { return STAGES * STAGE_BYTES + RED_BYTES + 256 + 1024; }
+
+static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
+                          const CUtensorMap& cb, const Params& P, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_tc_pass, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem_bytes());
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
+  if (grid <= 0) return cudaSuccess;
+  k_tc_pass<<<grid, NUM_THREADS, smem_bytes(), s>>>(a, b, ca, cb, P);
+  debug_kernel("k_tc_pass", s);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace tc
+
 bool tc_supported(const dblast_head* h) {
-  (void)h;
-  return false;
+  if (!h || h->dtype != DBLAST_BF16 || (h->H % tc::BK) != 0) return false;
+  const int rr = h->r + (h->e ? 1 : 0);
+  if (rr > 32 || h->K > tc::KMAX) return false;
+  return tc::encode_fn() != nullptr;
+}
+
+// transposed expander [U_z | e_z]^T as bf16 [rows_pad, H] for the prep GEMM
+__global__ void k_prep_transpose(const __nv_bfloat16* __restrict__ U,
+                                 const __nv_bfloat16* __restrict__ e, int H, int K, int r, int rr,
+                                 int rows_pad, __nv_bfloat16* __restrict__ ut) {
+  const size_t n = (size_t)rows_pad * H;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const int hh = (int)(i % H);
+    const int row = (int)(i / H);
+    __nv_bfloat16 v = __float2bfloat16(0.f);
+    if (row < K * rr) {
+      const int z = row / rr, k = row - z * rr;
+      if (k < r) v = U[((size_t)z * H + hh) * r + k];
+      else if (e) v = e[(size_t)z * H + hh];
+    }
+    ut[i] = v;
+  }
+}
+
+cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStream_t s) {
+  unsigned char* prep = static_cast<unsigned char*>(h->prep);
+  void* ut = prep + pl.off_ut;
+  const int rows = h->K * pl.rr;
+  const int rows_pad = ceil_div(rows, tc::BM) * tc::BM;
+  auto* utp = static_cast<__nv_bfloat16*>(ut);
+  k_prep_transpose<<<1024, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(h->U),
+                                        static_cast<const __nv_bfloat16*>(h->e), h->H, h->K, h->r,
+                                        pl.rr, rows_pad, utp);
+  debug_kernel("k_prep_transpose", s);
+  count_launches(1);
+  CUtensorMap ma, mb;
+  if (!tc::make_map(&ma, utp, h->H, rows_pad, true) || !tc::make_map(&mb, h->W, h->H, h->V, true))
+    return cudaErrorInvalidValue;
+  tc::Params P{};
+  P.mode = tc::MODE_PREP;
+  P.n_mt = rows_pad / tc::BM;
+  P.n_vt = ceil_div(h->V, tc::BN);
+  P.n_tiles = P.n_mt * P.n_vt;
+  P.nb = h->H / tc::BK;
+  P.ncs = 0;
+  P.K = h->K;
+  P.rp = pl.rp;
+  P.zps = 1;
+  P.M = rows;
+  P.V = h->V;
+  P.Mpad = rows_pad;
+  P.wu = reinterpret_cast<float*>(prep + pl.off_wu);
+  P.prep_rows = rows;
+  P.status = reinterpret_cast<DevStatus*>(prep + pl.off_status);
+  P.spin_limit = wait_limit();
+  return tc::launch(ma, mb, ma, mb, P, s);
 }
 
 cudaError_t launch_draft_pass_tc(const StepCtx& c) {
-  (void)c;
-  return cudaErrorNotSupported;
+  const dblast_head* h = c.head;
+  const WsLayout& w = c.wl;
+  CUtensorMap ma, mb, mca, mcb;
+  const unsigned char* prep = c.prep;
+  if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true) ||
+      !tc::make_map(&mb, h->W, h->H, h->V, true) ||
+      !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false) ||
+      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false))
+    return cudaErrorInvalidValue;
+  tc::Params P{};
+  P.mode = tc::MODE_DRAFT;
+  P.n_mt = w.Mpad / tc::BM;
+  P.n_vt = ceil_div(h->V, tc::BN);
+  P.n_tiles = P.n_mt * P.n_vt;
+  P.nb = h->H / tc::BK;
+  P.ncs = ceil_div(w.KC, tc::BK);
+  P.K = h->K;
+  P.rp = w.rp;
+  P.zps = tc::BK / (2 * w.rp);
+  P.M = w.M;
+  P.V = h->V;
+  P.Mpad = w.Mpad;
+  P.k2 = c.k2;
+  P.vbias = h->vbias;
+  P.cscale = wsp<float>(c, w.off_cscale);
+  P.sw = prp<float>(c, c.pl.off_sw);
+  P.stash = wsp<float>(c, w.off_stash);
+  P.partd = wsp<float2>(c, w.off_partd);
+  P.status = wsp<DevStatus>(c, w.off_status);
+  P.spin_limit = wait_limit();
+  return tc::launch(ma, mb, mca, mcb, P, c.stream);
 }
 
 cudaError_t launch_verify_pass_tc(const StepCtx& c) {
-  (void)c;
-  return cudaErrorNotSupported;
+  // the fused verify pass runs on CUDA cores for now
+  return launch_verify_pass_simt(c);
 }
 
 }  // namespace dblast

@@ -14,7 +14,7 @@ from tests import parity
 
 pytestmark = pytest.mark.gpu
 
-IMPLS = ["simt"]
+IMPLS = ["simt", "tcgen05"]
 
 
 def _case(cfg, T, Z_T, seed, impl, seqs=None, round_idx=0, device="cuda"):
