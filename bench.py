@@ -310,7 +310,8 @@ def main():
         tr_path = os.path.join(ROOT, "profiles", "draft_pass_traffic.json")
         if os.path.exists(tr_path):
             d = json.load(open(tr_path))
-            if d.get("kernel_impl") == _impl_name(head, args) and d.get("workload") == cfg["name"]:
+            if d.get("kernel_impl") == ("tcgen05" if st["tc_launches"] > 0 else "simt") and \
+                    d.get("workload") == cfg["name"]:
                 traffic = d.get("bytes_per_launch")
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
@@ -319,7 +320,8 @@ def main():
             "dtype": "bf16" if cfg["dtype"] == "bf16" else "f32", "data": "synthetic",
             "config": {"workload": cfg["name"], "N": N, "B": B, "K": cfg["K"], "r": cfg["r"],
                        "H": cfg["H"], "V": cfg["V"], "T": args.T, "Z_T": cfg["Z_T"],
-                       "sigma": cfg["sigma"], "kernels": _impl_name(head, args),
+                       "sigma": cfg["sigma"],
+                       "kernels": "tcgen05" if st["tc_launches"] > 0 else "simt",
                        "parallelism": "replicas" if world > 1 else "single",
                        "l2": "no flush: inputs larger than L2 (W %.2f GB, target %.0f MB)" % (
                            cfg["V"] * cfg["H"] * 2 / 1e9,
@@ -347,21 +349,6 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
-
-
-def _impl_name(head, args):
-    if args.kernels != "auto":
-        return args.kernels
-    return "tcgen05" if (head.dtype.__str__() == "torch.bfloat16" and head.H % 64 == 0
-                         and _tc_available()) else "simt"
-
-
-def _tc_available():
-    try:
-        from paper_2608_05448_gb300 import binding
-        return getattr(binding, "TC_AVAILABLE", False)
-    except Exception:
-        return False
 
 
 if __name__ == "__main__":

@@ -176,6 +176,7 @@ void dblast_set_wait_limit(uint32_t spins);
 typedef struct {
   uint64_t calls;            /* draft/verify entry-point calls */
   uint64_t kernel_launches;  /* kernels launched by the library */
+  uint64_t tc_launches;      /* of which tensor-core (tcgen05) kernels */
   uint64_t timed_draft, timed_verify;
   double draft_pass_ms, verify_pass_ms;
 } dblast_stats;

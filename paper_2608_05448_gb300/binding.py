@@ -53,6 +53,7 @@ class CDraftOut(ctypes.Structure):
 
 class CStats(ctypes.Structure):
     _fields_ = [("calls", ctypes.c_uint64), ("kernel_launches", ctypes.c_uint64),
+                ("tc_launches", ctypes.c_uint64),
                 ("timed_draft", ctypes.c_uint64), ("timed_verify", ctypes.c_uint64),
                 ("draft_pass_ms", ctypes.c_double), ("verify_pass_ms", ctypes.c_double)]
 

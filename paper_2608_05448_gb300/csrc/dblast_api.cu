@@ -17,13 +17,14 @@ uint32_t wait_limit() { return g_wait_limit; }
 
 // ------------------------------------------------------------ measurement
 static std::mutex g_stats_mu;
-static std::atomic<uint64_t> g_launches{0}, g_calls{0};
+static std::atomic<uint64_t> g_launches{0}, g_calls{0}, g_tc_launches{0};
 static bool g_timing = false;
 constexpr int kMaxTimed = 4096;
 static std::vector<cudaEvent_t> g_ev[2];  // pairs (begin, end) per timed call
 static int g_n_ev[2] = {0, 0};
 
 void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+void count_tc_launch() { g_tc_launches.fetch_add(1, std::memory_order_relaxed); }
 
 // DBLAST_DEBUG_SYNC=1: synchronise after every launcher and name the one that failed
 static bool debug_sync() {
@@ -320,6 +321,7 @@ void dblast_stats_reset(int enable_pass_timing) {
   std::lock_guard<std::mutex> lk(g_stats_mu);
   g_launches = 0;
   g_calls = 0;
+  g_tc_launches = 0;
   g_n_ev[0] = g_n_ev[1] = 0;
   g_timing = enable_pass_timing != 0;
 }
@@ -329,6 +331,7 @@ dblast_status dblast_stats_get(dblast_stats* out) {
   std::lock_guard<std::mutex> lk(g_stats_mu);
   out->calls = g_calls.load();
   out->kernel_launches = g_launches.load();
+  out->tc_launches = g_tc_launches.load();
   double ms[2] = {0.0, 0.0};
   for (int w = 0; w < 2; ++w) {
     for (int i = 0; i < g_n_ev[w]; ++i) {

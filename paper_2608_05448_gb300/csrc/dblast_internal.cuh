@@ -154,6 +154,7 @@ template <typename T> const T* prp(const StepCtx& c, size_t off) {
 
 // measurement hooks (dblast_api.cu)
 void count_launches(int n);
+void count_tc_launch();
 // with DBLAST_DEBUG_SYNC=1: synchronise and report the kernel just launched
 void debug_kernel(const char* name, cudaStream_t s);
 void pass_event_begin(int which, cudaStream_t s);  // which: 0 draft pass, 1 verify pass

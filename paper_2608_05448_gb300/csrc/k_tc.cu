@@ -509,6 +509,294 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ------------------------------------------------------------ verify pass
+// For a tile of 128 positions x 128 tokens: branch GEMMs D_z = c_z . WU_z^T
+// (two components per TMEM slot, two slots), then per (m, v)
+//   q(v|x_<i) = 2^{bk_v - B0} sum_z 2^{D_z a_{m,z} + log2 w_{m,z} - L_{m,z} + B0},
+//   p(v)      = 2^{t_v log2(e)/T - Lt_m},
+// and the tile records (sum min(p, q), sum [p - q]_+).  bk = stash log2(e)/T;
+// B0 = floor(max_z L_{m,z}) keeps both factors inside the fp32 range.
+struct VParams {
+  int n_mt, n_vt, n_tiles, ncs, K, rp, zps, M, V, Mpad, B, Bt;
+  float k2;
+  const float* cscale;   // [Mpad, K]
+  const float* sw;       // [K]
+  const double* lse2;    // [M, K]
+  const double* w2;      // [M, K]
+  const double* lse2t;   // [N (B+1)]
+  const float* stash;    // [M, V]
+  const __nv_bfloat16* target;  // [N, Bt, V]
+  float2* partv;         // [nt, Mpad]
+  DevStatus* status;
+  uint32_t spin_limit;
+};
+
+__device__ __forceinline__ void vtile_of(const VParams& P, int slot, int* mt, int* vt) {
+  const int t = (int)blockIdx.x + slot * (int)gridDim.x;
+  *vt = t / P.n_mt;
+  *mt = t - *vt * P.n_mt;
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    k_tc_verify(const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
+                const VParams P) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* stage_base = smem;
+  float2* red = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES);   // [2][BM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + 2 * BM * 8);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* sfull = bars + 2 * STAGES;   // [2] TMEM slot ready
+  uint64_t* sempty = sfull + 2;          // [2] TMEM slot free
+  uint64_t* done = sfull + 4;
+  uint64_t* redw = sfull + 5;
+  uint64_t* redm = sfull + 6;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 7);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int my_tiles = (P.n_tiles > (int)blockIdx.x)
+                           ? (P.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
+                           : 0;
+  const int ngroups = (P.K + 1) / 2;     // two components per TMEM slot
+  Ctl ctl{P.spin_limit, abort_flag, P.status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sfull[b], 1);
+      mbar_init(&sempty[b], NUM_EPI_WARPS);
+    }
+    mbar_init(done, 1);
+    mbar_init(redw, 32 * NUM_EPI_WARPS);
+    mbar_init(redm, 32 * NUM_EPI_WARPS);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
+      bool ok = true;
+      for (int slot = 0; slot < my_tiles && ok; ++slot) {
+        int mt, vt;
+        vtile_of(P, slot, &mt, &vt);
+        for (int c = 0; c < P.ncs; ++c) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 11)) { ok = false; break; }
+          unsigned char* sa = stage_base + stage * STAGE_BYTES;
+          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          tma_load_2d(sa, &tm_ca, &full[stage], c * BK, mt * BM);
+          tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, vt * BN);
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      for (int s = 0; s < STAGES; ++s)
+        if (issued_mask & (1u << s)) {
+          const uint64_t t0 = globaltimer();
+          while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
+                 (globaltimer() - t0) < 2000000000ull) {
+          }
+        }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id_corr = idesc_f16(false);
+      int stage = 0;
+      uint32_t phase = 0, guse0 = 0u, guse1 = 0u;
+      bool ok = true;
+      for (int slot = 0; slot < my_tiles && ok; ++slot) {
+        int c = 0;  // next stage of this tile
+        for (int g = 0; g < ngroups && ok; ++g) {
+          const int gs = g & 1;
+          const uint32_t use = gs ? guse1 : guse0;
+          if (!mbar_wait(&sempty[gs], (use & 1u) ^ 1u, ctl, 12)) { ok = false; break; }
+          tc_fence_after();
+          const int z0 = 2 * g, z1 = min(P.K, z0 + 2);
+          // stages holding components z0 .. z1-1
+          while (ok && c < P.ncs && c * P.zps < z1) {
+            if (!mbar_wait(&full[stage], phase, ctl, 13)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(stage_base + stage * STAGE_BYTES);
+            const uint32_t sb = sa + STAGE_A;
+            for (int zz = 0; zz < P.zps; ++zz) {
+              const int z = c * P.zps + zz;
+              if (z >= z1) break;
+              const uint32_t col = tmem + (uint32_t)(gs * 2 * BN + (z - z0) * BN);
+              const int o = zz * 2 * P.rp;
+              int first = 1;
+              for (int kk = 0; kk < P.rp; kk += 16) {
+                const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
+                umma(col, sdesc(sa + hi), sdesc(sb + hi), id_corr, first ? 0u : 1u);
+                umma(col, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
+                umma(col, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
+                first = 0;
+              }
+            }
+            umma_commit(&empty[stage]);
+            if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+            ++c;
+          }
+          if (!ok) break;
+          umma_commit(&sfull[gs]);
+          if (gs) ++guse1; else ++guse0;
+        }
+      }
+      umma_commit(done);
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
+      }
+    }
+  } else {
+    const int ew = warp - 2;
+    const int q = warp & 3;
+    const int half = ew >> 2;
+    const int row = q * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint32_t guse0 = 0u, guse1 = 0u;
+    for (int slot = 0; slot < my_tiles; ++slot) {
+      int mt, vt;
+      vtile_of(P, slot, &mt, &vt);
+      const int m = mt * BM + row;
+      const bool mok = m < P.M;
+      const int v0 = vt * BN + half * 64;
+      // per-row constants
+      float a[KMAX], cz[KMAX];
+      double B0 = 0.0;
+      if (mok) {
+        double mx = -INFINITY;
+        for (int z = 0; z < P.K; ++z) mx = fmax(mx, P.lse2[(size_t)m * P.K + z]);
+        B0 = floor(mx);
+      }
+#pragma unroll
+      for (int z = 0; z < KMAX; ++z) {
+        a[z] = 0.f;
+        cz[z] = -INFINITY;
+        if (z < P.K && mok) {
+          a[z] = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
+          const double wz = P.w2[(size_t)m * P.K + z];
+          cz[z] = (wz == -INFINITY) ? -INFINITY
+                                    : (float)(wz - P.lse2[(size_t)m * P.K + z] + B0);
+        }
+      }
+      float acc[64];
+#pragma unroll
+      for (int j = 0; j < 64; ++j) acc[j] = 0.f;
+      bool ok = true;
+      for (int g = 0; g < ngroups; ++g) {
+        const int gs = g & 1;
+        const uint32_t use = gs ? guse1 : guse0;
+        if (!mbar_wait(&sfull[gs], use & 1u, ctl, 14)) { ok = false; break; }
+        if (gs) ++guse1; else ++guse0;
+        tc_fence_after();
+#pragma unroll
+        for (int zz = 0; zz < 2; ++zz) {
+          const int z = 2 * g + zz;
+          if (z < P.K) {
+            float az = 0.f, cc_z = -INFINITY;
+#pragma unroll
+            for (int k = 0; k < KMAX; ++k)
+              if (k == z) { az = a[k]; cc_z = cz[k]; }
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+              float cr[32];
+              tmem_ld32(tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + half * 64 + cc * 32),
+                        cr);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) acc[cc * 32 + j] += exp2f(fmaf(cr[j], az, cc_z));
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sempty[gs]);
+      }
+      if (!ok) break;
+      float As = 0.f, Rs = 0.f;
+      if (mok) {
+        const int n = m / P.B, i = m - n * P.B;
+        const float Lt = (float)P.lse2t[(size_t)n * (P.B + 1) + i];
+        const float B0f = (float)B0;
+        const float* srow = P.stash + (size_t)m * P.V + v0;
+        const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
+        const bool vec = (v0 + 64 <= P.V) && ((P.V & 7) == 0);
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc) {
+          float sv[8], tv[8];
+          if (vec) {
+            const float4 s0 = *reinterpret_cast<const float4*>(srow + cc * 8);
+            const float4 s1 = *reinterpret_cast<const float4*>(srow + cc * 8 + 4);
+            sv[0] = s0.x; sv[1] = s0.y; sv[2] = s0.z; sv[3] = s0.w;
+            sv[4] = s1.x; sv[5] = s1.y; sv[6] = s1.z; sv[7] = s1.w;
+            const uint4 t8 = *reinterpret_cast<const uint4*>(trow + cc * 8);
+            const __nv_bfloat162* tp = reinterpret_cast<const __nv_bfloat162*>(&t8);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const float2 f = __bfloat1622float2(tp[u]);
+              tv[2 * u] = f.x;
+              tv[2 * u + 1] = f.y;
+            }
+          } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              const int v = v0 + cc * 8 + u;
+              sv[u] = (v < P.V) ? srow[cc * 8 + u] : 0.f;
+              tv[u] = (v < P.V) ? __bfloat162float(trow[cc * 8 + u]) : 0.f;
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int j = cc * 8 + u;
+            if (v0 + j < P.V) {
+              const float qv = exp2f(fmaf(sv[u], P.k2, -B0f)) * acc[j];
+              const float pv = exp2f(fmaf(tv[u], P.k2, -Lt));
+              const float mn = fminf(pv, qv);
+              As += mn;
+              Rs += pv - mn;
+            }
+          }
+        }
+      }
+      // the other column half of this row, then one record per (tile, row)
+      if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 15)) break;
+      red[half * BM + row] = make_float2(As, Rs);
+      mbar_arrive(redw);
+      if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 16)) break;
+      if (half == 0) {
+        const float2 o = red[BM + row];
+        P.partv[(size_t)vt * P.Mpad + m] = make_float2(As + o.x, Rs + o.y);
+      }
+      mbar_arrive(redm);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(TMEM_COLS));
+  }
+}
+
 // --------------------------------------------------------------- host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -572,6 +860,7 @@ static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUte
   k_tc_pass<<<grid, NUM_THREADS, smem_bytes(), s>>>(a, b, ca, cb, P);
   debug_kernel("k_tc_pass", s);
   count_launches(1);
+  count_tc_launch();
   return cudaGetLastError();
 }
 
@@ -672,8 +961,50 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
 }
 
 cudaError_t launch_verify_pass_tc(const StepCtx& c) {
-  // the fused verify pass runs on CUDA cores for now
-  return launch_verify_pass_simt(c);
+  const dblast_head* h = c.head;
+  const WsLayout& w = c.wl;
+  CUtensorMap mca, mcb;
+  if (!tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false) ||
+      !tc::make_map(&mcb, c.prep + c.pl.off_wuop, w.KC, h->V, false))
+    return cudaErrorInvalidValue;
+  tc::VParams P{};
+  P.n_mt = w.Mpad / tc::BM;
+  P.n_vt = ceil_div(h->V, tc::BN);
+  P.n_tiles = P.n_mt * P.n_vt;
+  P.ncs = ceil_div(w.KC, tc::BK);
+  P.K = h->K;
+  P.rp = w.rp;
+  P.zps = tc::BK / (2 * w.rp);
+  P.M = w.M;
+  P.V = h->V;
+  P.Mpad = w.Mpad;
+  P.B = w.B;
+  P.Bt = c.Bt;
+  P.k2 = c.k2;
+  P.cscale = wsp<float>(c, w.off_cscale);
+  P.sw = prp<float>(c, c.pl.off_sw);
+  P.lse2 = wsp<double>(c, w.off_lse2);
+  P.w2 = wsp<double>(c, w.off_w2);
+  P.lse2t = wsp<double>(c, w.off_lse2t);
+  P.stash = wsp<float>(c, w.off_stash);
+  P.target = static_cast<const __nv_bfloat16*>(c.target);
+  P.partv = wsp<float2>(c, w.off_partv);
+  P.status = wsp<DevStatus>(c, w.off_status);
+  P.spin_limit = wait_limit();
+  static bool attr = false;
+  const size_t smem = tc::STAGES * tc::STAGE_BYTES + 2 * tc::BM * 8 + 256 + 1024;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(tc::k_tc_verify,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int grid = P.n_tiles < tc::num_sms() ? P.n_tiles : tc::num_sms();
+  tc::k_tc_verify<<<grid, tc::NUM_THREADS, smem, c.stream>>>(mca, mcb, P);
+  debug_kernel("k_tc_verify", c.stream);
+  count_launches(1);
+  count_tc_launch();
+  return cudaGetLastError();
 }
 
 }  // namespace dblast
