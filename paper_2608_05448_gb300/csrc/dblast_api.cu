@@ -93,6 +93,8 @@ PrepLayout prep_layout(int V, int H, int K, int r, bool has_e) {
   o = align_up(o + (size_t)K * sizeof(float), 256);
   p.off_ut = o;
   o = align_up(o + (size_t)ceil_div(K * p.rr, MTILE) * MTILE * H * 2, 256);
+  p.off_vt = o;
+  o = align_up(o + (size_t)ceil_div(K * p.rr, MTILE) * MTILE * H * 2, 256);
   p.off_status = o;
   o = align_up(o + sizeof(DevStatus), 256);
   p.total = o;
@@ -127,14 +129,18 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_log2pi = take((size_t)N * K * sizeof(float));
   w.off_stash = take((size_t)w.M * V * sizeof(float));
   w.off_partd = take((size_t)w.nt * K * w.Mpad * sizeof(float2));
-  w.off_lse2 = take((size_t)w.M * K * sizeof(double));
-  w.off_lq2 = take((size_t)w.M * K * sizeof(double));
-  w.off_w2 = take((size_t)w.M * K * sizeof(double));
+  w.off_lsep = take((size_t)LSE_SPLIT * w.M * K * sizeof(float4));
+  w.off_lse2 = take((size_t)w.M * K * sizeof(float2));
+  w.off_lq2 = take((size_t)w.M * K * sizeof(float2));
+  w.off_w2 = take((size_t)w.M * K * sizeof(float2));
+  w.off_qtok = take((size_t)w.M * sizeof(float));
   w.off_tok = take((size_t)w.M * sizeof(int32_t));
+  w.off_vcz = take((size_t)w.M * K * sizeof(float2));
+  w.off_vb0 = take((size_t)w.M * sizeof(float));
   w.off_partt = take((size_t)w.nt * w.Rt * sizeof(float2));
-  w.off_lse2t = take((size_t)w.Rt * sizeof(double));
+  w.off_lt2 = take((size_t)w.Rt * sizeof(float2));
   w.off_partv = take((size_t)w.nt * w.Mpad * sizeof(float2));
-  w.off_av = take((size_t)w.M * sizeof(double2));
+  w.off_av = take((size_t)AV_SPLIT * w.M * sizeof(float4));
   w.off_ties = take((size_t)N * sizeof(uint32_t));
   w.total = o;
   return w;
@@ -198,6 +204,7 @@ static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, 
   c->prep = static_cast<const unsigned char*>(h->prep);
   c->stream = reinterpret_cast<cudaStream_t>(stream);
   c->k2 = LOG2E / a->temperature;
+  c->tc = use_tc(h, a);
   c->target = nullptr;
   c->Bt = a->B + (has_bonus ? 1 : 0);
   return DBLAST_OK;
@@ -236,7 +243,7 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   if (e == cudaSuccess) e = dbg(launch_prior_codes(c), "prior_codes", c.stream);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
-    e = use_tc(c.head, c.args) ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
+    e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
     pass_event_end(0, c.stream);
     e = dbg(e, "draft_pass", c.stream);
   }
@@ -251,7 +258,7 @@ static dblast_status verify_impl(StepCtx c, dblast_verify_out* out) {
   cudaError_t e = dbg(launch_target_stats(c, out), "target_stats", c.stream);
   if (e == cudaSuccess) {
     pass_event_begin(1, c.stream);
-    e = use_tc(c.head, c.args) ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
+    e = c.tc ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
     pass_event_end(1, c.stream);
     e = dbg(e, "verify_pass", c.stream);
   }

@@ -30,24 +30,29 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 // ---------------------------------------------------------------- layouts
 struct PrepLayout {
   int V, K, rr, rp, KC;    // rr = r + (e != NULL); rp = rr rounded up to 16; KC = K*2*rp
-  size_t off_wu, off_wuop, off_sw, off_ut, off_status, total;
+  size_t off_wu, off_wuop, off_sw, off_ut, off_vt, off_status, total;
   // WU   fp32 [V, K, rr]: (W U_z)_v and, if e, (W e_z)_v in column r
   // WUop fp16 [V, KC]   : per z, [hi(rp) | lo(rp)] of WU_z * sw[z]
   // sw   fp32 [K]       : power-of-two scale of WUop's z block
   // ut   bf16 [rows_pad, H]: [U_z | e_z]^T, the A operand of the tensor-core prep
+  // vt   bf16 [rows_pad, H]: [V_z | 0]^T, the A operand of the tensor-core codes GEMM
   // status DevStatus      : bounded-wait record of the tensor-core prep
 };
 
-// Workspace regions (each 256-byte aligned), with their element types:
+// Workspace regions (each 256-byte aligned), with their element types (ff: a
+// float pair hi + lo, see FF below):
 //   status DevStatus | codes f32 [Mpad,K,rr] | cscale f32 [Mpad,K] | cop f16 [Mpad,KC]
 //   zhat i32 [N] | log2pi f32 [N,K] | stash f32 [M,V] | partd float2 [nt,K,Mpad]
-//   lse2, lq2, w2 f64 [M,K] | tok i32 [M] | partt float2 [nt,Rt] | lse2t f64 [Rt]
-//   partv float2 [nt,Mpad] | av double2 [M] | ties u32 [N]
+//   lsep float4 [LSE_SPLIT,M,K] | lse2, lq2, w2 ff [M,K] | qtok f32 [M] | tok i32 [M]
+//   vcz float2 [M,K] | vb0 f32 [M] | partt float2 [nt,Rt] | lt2 ff [Rt]
+//   partv float2 [nt,Mpad] | av float4 [AV_SPLIT,M] | ties u32 [N]
+constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
+constexpr int AV_SPLIT = 8;   // partial sums of the verify records per row
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
-      off_partd, off_lse2, off_lq2, off_w2, off_tok, off_partt, off_lse2t, off_partv,
-      off_av, off_ties, total;
+      off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
+      off_partt, off_lt2, off_partv, off_av, off_ties, total;
 };
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
@@ -87,6 +92,41 @@ template <> __device__ __forceinline__ float ldf<__nv_bfloat16>(const __nv_bfloa
   return __bfloat162float(*p);
 }
 
+// 8 consecutive values of a row starting at v0 (v0 % 8 == 0), -inf past V.
+// `vec` (16-byte aligned rows, V % 8 == 0): one unconditional load from an
+// in-bounds offset, then a select, so loads of consecutive calls can overlap.
+__device__ __forceinline__ void load8(const __nv_bfloat16* row, int v0, int V, bool vec,
+                                      float (&x)[8]) {
+  if (vec) {
+    const bool in = v0 < V;
+    const uint4 u = *reinterpret_cast<const uint4*>(row + (in ? v0 : 0));
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(h[j]);
+      x[2 * j] = in ? f.x : -INFINITY;
+      x[2 * j + 1] = in ? f.y : -INFINITY;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) x[j] = (v0 + j < V) ? __bfloat162float(row[v0 + j]) : -INFINITY;
+  }
+}
+__device__ __forceinline__ void load8(const float* row, int v0, int V, bool vec, float (&x)[8]) {
+  if (vec) {
+    const bool in = v0 < V;
+    const float4 a = *reinterpret_cast<const float4*>(row + (in ? v0 : 0));
+    const float4 b = *reinterpret_cast<const float4*>(row + (in ? v0 : 0) + 4);
+    x[0] = in ? a.x : -INFINITY; x[1] = in ? a.y : -INFINITY;
+    x[2] = in ? a.z : -INFINITY; x[3] = in ? a.w : -INFINITY;
+    x[4] = in ? b.x : -INFINITY; x[5] = in ? b.y : -INFINITY;
+    x[6] = in ? b.z : -INFINITY; x[7] = in ? b.w : -INFINITY;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) x[j] = (v0 + j < V) ? row[v0 + j] : -INFINITY;
+  }
+}
+
 // ------------------------------------------------- (max, sum) pairs in base 2
 // A pair (m, s) stands for s * 2^m; the empty pair is (-inf, 0).
 __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
@@ -121,15 +161,61 @@ __device__ __forceinline__ float warp_max(float v) {
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
-// inclusive prefix sum over lanes
-__device__ __forceinline__ double warp_incl_scan_d(double v) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const double t = __shfl_up_sync(0xffffffffu, v, o);
-    if (lane >= o) v += t;
+// ------------------------------------------------------------ float-float
+// This GPU issues double-precision arithmetic at a small fraction of the fp32
+// rate and with long latency, so the device path carries extended precision
+// as an unevaluated pair of floats (TwoSum / TwoProd, about 44 significant
+// bits) and never uses doubles.
+struct FF {
+  float hi, lo;  // value hi + lo, |lo| <= ulp(hi) / 2
+};
+__device__ __forceinline__ FF ff_add(FF a, FF b) {
+  const float s = a.hi + b.hi;
+  const float bb = s - a.hi;
+  const float e = ((a.hi - (s - bb)) + (b.hi - bb)) + (a.lo + b.lo);
+  const float hi = s + e;
+  return FF{hi, e - (hi - s)};
+}
+__device__ __forceinline__ FF ff_neg(FF a) { return FF{-a.hi, -a.lo}; }
+__device__ __forceinline__ FF ff_sub(FF a, FF b) { return ff_add(a, ff_neg(b)); }
+__device__ __forceinline__ FF ff_addf(FF a, float b) { return ff_add(a, FF{b, 0.f}); }
+// exact product of two floats as a pair
+__device__ __forceinline__ FF ff_prod(float a, float b) {
+  const float p = a * b;
+  return FF{p, fmaf(a, b, -p)};
+}
+__device__ __forceinline__ FF ff_mulf(FF a, float b) {
+  const float p = a.hi * b;
+  const float e = fmaf(a.hi, b, -p) + a.lo * b;
+  const float hi = p + e;
+  return FF{hi, e - (hi - p)};
+}
+__device__ __forceinline__ bool ff_gt(FF a, FF b) {
+  return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo);
+}
+__device__ __forceinline__ float ff_f(FF a) { return a.hi + a.lo; }
+__device__ __forceinline__ FF ff_ld(const float2* p) {
+  const float2 v = *p;
+  return FF{v.x, v.y};
+}
+__device__ __forceinline__ float2 ff_st(FF a) { return make_float2(a.hi, a.lo); }
+// 2^a: exp2f of the high part times the first-order factor of the low part
+__device__ __forceinline__ float ff_exp2(FF a) { return exp2f(a.hi) * fmaf(a.lo, LN2, 1.f); }
+// log2 of a positive pair: exact binary exponent, log2f of the mantissa in
+// [1, 2) (absolute error about 1e-7), and a first-order term for lo / hi
+__device__ __forceinline__ FF ff_log2(FF a) {
+  if (!(a.hi > 0.f)) return FF{-INFINITY, 0.f};
+  if (a.hi == INFINITY) return FF{INFINITY, 0.f};
+  float x = a.hi;
+  int bias = 0;
+  if (x < 0x1p-100f) {
+    x *= 0x1p64f;
+    bias = 64;
   }
-  return v;
+  const unsigned b = __float_as_uint(x);
+  const int e = (int)((b >> 23) & 0xffu) - 127 - bias;
+  const float m = __uint_as_float((b & 0x7fffffu) | 0x3f800000u);
+  return ff_add(FF{(float)e, 0.f}, FF{log2f(m) + (a.lo / a.hi) * LOG2E, 0.f});
 }
 
 // ------------------------------------------------------------ launchers
@@ -143,6 +229,7 @@ struct StepCtx {
   cudaStream_t stream;
   float k2;  // log2(e) / T
   bool has_e;
+  bool tc;   // tensor-core passes
   const void* target;  // verify only: [N, Bt, V]
   int Bt;              // target rows per sequence (B + has_bonus)
 };
@@ -162,6 +249,7 @@ void pass_event_end(int which, cudaStream_t s);
 
 cudaError_t launch_prep(const dblast_head* head, const PrepLayout& pl, cudaStream_t s);
 cudaError_t launch_prep_tc(const dblast_head* head, const PrepLayout& pl, cudaStream_t s);
+cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit);
 bool tc_supported(const dblast_head* h);
 cudaError_t launch_prior_codes(const StepCtx& c);
 cudaError_t launch_draft_pass_simt(const StepCtx& c);

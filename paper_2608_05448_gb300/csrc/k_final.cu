@@ -1,0 +1,791 @@
+// Finalize kernels of the step, shared by the CUDA-core and tensor-core
+// vocabulary passes.  They merge the per-tile records of the passes
+//   draft  : partd[t][z][m] = (m2, s), s * 2^m2 = sum_v 2^{l_{m,z,v} log2(e)/T}
+//   target : partt[t][row]  = (tmax, s), s = sum_v 2^{(t_v - tmax) log2(e)/T}
+//   verify : partv[t][m]    = (sum_v min(p, q), sum_v [p - q]_+)
+// and take every decision of the step: the draft tokens (Sec. 3.1), the
+// category posterior and q(x_i|x_<i) (Eqs. category-posterior and
+// dep-next-token), acceptance with min(1, p/q) (Eq. 2), the residual or bonus
+// token (Algorithm 1, App. A) and the expected lengths (Eq. 3).
+//
+// Every token draw is an inverse CDF over the vocabulary in two levels: a
+// block-wide scan of the tile masses finds the tile, then the tile's TILE_V
+// masses are recomputed and scanned.
+//
+// Precision without FP64: sums, scans, log-sum-exps and log-weights are
+// float-float pairs (FF); exponents subtract a normaliser held as a pair, so
+// the rounded part of every exponent is the small difference, not the large
+// logit.
+#include "dblast_internal.cuh"
+
+namespace dblast {
+
+constexpr unsigned FULLMASK = 0xffffffffu;
+
+// ------------------------------------------------------------ float-float
+__device__ __forceinline__ FF ff_shfl_up(FF a, int o) {
+  return FF{__shfl_up_sync(FULLMASK, a.hi, o), __shfl_up_sync(FULLMASK, a.lo, o)};
+}
+__device__ __forceinline__ FF ff_shfl_xor(FF a, int o) {
+  return FF{__shfl_xor_sync(FULLMASK, a.hi, o), __shfl_xor_sync(FULLMASK, a.lo, o)};
+}
+
+// ------------------------------------------------------------ block helpers
+struct BlockScan {
+  FF excl, incl, total;  // excl of thread j equals incl of thread j-1 bit for bit
+};
+
+template <int NT> __device__ BlockScan block_scan_ff(FF v, FF* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  FF wi = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const FF t = ff_shfl_up(wi, o);
+    if (lane >= o) wi = ff_add(t, wi);
+  }
+  FF we = ff_shfl_up(wi, 1);
+  if (lane == 0) we = FF{0.f, 0.f};
+  if (lane == 31) sh[warp] = wi;
+  __syncthreads();
+  FF off{0.f, 0.f}, tot{0.f, 0.f};
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) {
+    if (w == warp) off = tot;
+    tot = ff_add(tot, sh[w]);
+  }
+  __syncthreads();
+  return BlockScan{ff_add(off, we), ff_add(off, wi), tot};
+}
+
+template <int NT> __device__ int block_min_i(int v, int* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(FULLMASK, v, o));
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+  __syncthreads();
+  int r = sh[0];
+#pragma unroll
+  for (int w = 1; w < NT / 32; ++w) r = min(r, sh[w]);
+  __syncthreads();
+  return r;
+}
+
+template <int NT> __device__ int block_max_i(int v, int* sh) {
+  return -block_min_i<NT>(-v, sh);
+}
+
+__device__ __forceinline__ float corr_at(const float* __restrict__ wu, const float* __restrict__ c,
+                                         int v, int z, int K, int rr) {
+  const float* wr = wu + ((size_t)v * K + z) * rr;
+  float acc = 0.f;
+  for (int k = 0; k < rr; ++k) acc = fmaf(wr[k], c[k], acc);
+  return acc;
+}
+
+// 2^{(x k2 - C)} for a float logit x and a split normaliser C = c.hi + c.lo:
+// the product is exact inside the fma, so only the small difference rounds.
+__device__ __forceinline__ float exp2_rel(float x, float k2, FF c) {
+  return exp2f(fmaf(x, k2, -c.hi) - c.lo);
+}
+// 2^{(base + corr) k2 - C} with the same care for the two-term logit
+__device__ __forceinline__ float exp2_rel2(float base, float corr, float k2, FF c) {
+  return exp2f(fmaf(corr, k2, fmaf(base, k2, -c.hi)) - c.lo);
+}
+
+// ------------------------------------------------------- two-level draw
+template <int NT> struct FindShared {
+  FF d[NT / 32];
+  int i[NT / 32];
+  FF before;
+  int tile, x, tie;
+};
+
+struct FindOut {
+  int x;     // chosen token, -1 if no token has mass
+  bool tie;  // the decision is within TIE_TOL of its threshold, or rounding forced a fallback
+};
+
+// Smallest token whose cumulative mass (in vocabulary order) exceeds `target`.
+// tmass(t): mass of tile t; emass(v): mass of token v (floats); `total` scales
+// the decision margin.
+template <int NT, typename TM, typename EM>
+__device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF target,
+                              float total, FindShared<NT>& fs) {
+  static_assert(NT >= TILE_V, "one thread per token of a tile");
+  const int tid = threadIdx.x, lane = tid & 31;
+  const int chunk = ceil_div(nt, NT);
+  const int t0 = min(nt, tid * chunk), t1 = min(nt, t0 + chunk);
+  // level 1: this thread's chunk of tiles, loads issued eight at a time
+  FF loc{0.f, 0.f};
+  int lastp = -1;
+  for (int c0 = 0; c0 < chunk; c0 += 8) {
+    float w[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int t = t0 + c0 + j;
+      w[j] = tmass(t < t1 ? t : 0);  // tile 0 always exists
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int t = t0 + c0 + j;
+      if (t < t1) {
+        loc = ff_addf(loc, w[j]);
+        if (w[j] > 0.f) lastp = t;
+      }
+    }
+  }
+  const BlockScan sc = block_scan_ff<NT>(loc, fs.d);
+  const int first = block_min_i<NT>(ff_gt(sc.incl, target) ? tid : NT, fs.i);
+  const int lastall = block_max_i<NT>(lastp, fs.i);
+  if (first < NT) {
+    // the warp holding thread `first` rescans its chunk, 32 tiles per round,
+    // starting from that thread's exclusive prefix
+    if ((tid >> 5) == (first >> 5)) {
+      const FF ex{__shfl_sync(FULLMASK, sc.excl.hi, first & 31),
+                  __shfl_sync(FULLMASK, sc.excl.lo, first & 31)};
+      const int f0 = first * chunk, f1 = min(nt, f0 + chunk);
+      FF base = ex, lastlo{0.f, 0.f};
+      int tt = -1, lp = -1;
+      FF before{0.f, 0.f};
+      for (int r0 = f0; r0 < f1 && tt < 0; r0 += 32) {
+        const int t = r0 + lane;
+        const float w = (t < f1) ? tmass(t) : 0.f;
+        FF incl{w, 0.f};
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const FF u = ff_shfl_up(incl, o);
+          if (lane >= o) incl = ff_add(u, incl);
+        }
+        FF ex1 = ff_shfl_up(incl, 1);
+        if (lane == 0) ex1 = FF{0.f, 0.f};
+        const FF hi = ff_add(base, incl), lo = ff_add(base, ex1);
+        const unsigned hit = __ballot_sync(FULLMASK, t < f1 && ff_gt(hi, target));
+        const unsigned pos = __ballot_sync(FULLMASK, t < f1 && w > 0.f);
+        if (pos) {
+          const int l = 31 - __clz(pos);
+          lp = r0 + l;
+          lastlo = FF{__shfl_sync(FULLMASK, lo.hi, l), __shfl_sync(FULLMASK, lo.lo, l)};
+        }
+        if (hit) {
+          const int l = __ffs(hit) - 1;
+          tt = r0 + l;
+          before = FF{__shfl_sync(FULLMASK, lo.hi, l), __shfl_sync(FULLMASK, lo.lo, l)};
+        }
+        base = FF{__shfl_sync(FULLMASK, hi.hi, 31), __shfl_sync(FULLMASK, hi.lo, 31)};
+      }
+      if (lane == 0) {
+        const bool miss = tt < 0;  // the rescan rounded below the target
+        fs.tile = miss ? lp : tt;
+        fs.before = miss ? lastlo : before;
+        fs.tie = miss ? 1 : 0;
+      }
+    }
+  } else if (tid == 0) {  // rounding left the target at or above the total
+    fs.tile = lastall;
+    fs.before = lastall >= 0 ? ff_add(sc.total, FF{-tmass(lastall), 0.f}) : FF{0.f, 0.f};
+    fs.tie = 1;
+  }
+  __syncthreads();
+  const int tt = fs.tile;
+  const FF before = fs.before;
+  float e = 0.f;
+  const int v = tt * TILE_V + tid;
+  if (tt >= 0 && tid < TILE_V && v < V) e = emass(v);
+  const BlockScan es = block_scan_ff<NT>(FF{e, 0.f}, fs.d);
+  const FF lo = ff_add(before, es.excl), hi = ff_add(before, es.incl);
+  const int fj = block_min_i<NT>((tt >= 0 && ff_gt(hi, target)) ? tid : NT, fs.i);
+  const int lastv = block_max_i<NT>(e > 0.f ? tid : -1, fs.i);
+  if (fj < NT) {
+    if (tid == fj) {
+      fs.x = tt * TILE_V + fj;
+      const float margin = fminf(ff_f(ff_sub(target, lo)), ff_f(ff_sub(hi, target))) / total;
+      if (margin < TIE_TOL) fs.tie = 1;
+    }
+  } else if (tid == 0) {
+    fs.x = (tt >= 0 && lastv >= 0) ? tt * TILE_V + lastv : -1;
+    fs.tie = 1;
+  }
+  __syncthreads();
+  const FindOut r{fs.x, fs.tie != 0};
+  __syncthreads();
+  return r;
+}
+
+// Mass functors (data by value).
+struct DraftTileMass {  // s 2^(m2 - L) of a draft record
+  const float2* rec;
+  size_t stride;
+  FF L;
+  __device__ float operator()(int t) const {
+    const float2 q = rec[(size_t)t * stride];
+    return q.y > 0.f ? q.y * exp2f((q.x - L.hi) - L.lo) : 0.f;
+  }
+};
+struct TargetTileMass {  // s 2^(tmax k2 - Lt) of a target record
+  const float2* rec;
+  size_t stride;
+  float k2;
+  FF Lt;
+  __device__ float operator()(int t) const {
+    const float2 q = rec[(size_t)t * stride];
+    return q.y > 0.f ? q.y * exp2_rel(q.x, k2, Lt) : 0.f;
+  }
+};
+struct ResidTileMass {  // residual mass record, clamped at 0
+  const float2* rec;
+  size_t stride;
+  __device__ float operator()(int t) const { return fmaxf(rec[(size_t)t * stride].y, 0.f); }
+};
+struct BranchTokenProb {  // q_i(v|z) = 2^{(base_v + corr_z(v)) k2 - L_z}
+  const float* srow;
+  const float* wu;
+  const float* cz;
+  int z, K, rr;
+  float k2;
+  FF L;
+  __device__ float operator()(int v) const {
+    return exp2_rel2(srow[v], corr_at(wu, cz, v, z, K, rr), k2, L);
+  }
+};
+template <typename Tin> struct TargetTokenProb {  // p_i(v) = 2^{t_v k2 - Lt}
+  const Tin* trow;
+  float k2;
+  FF Lt;
+  __device__ float operator()(int v) const { return exp2_rel(ldf(trow + v), k2, Lt); }
+};
+template <typename Tin> struct ResidualTokenMass {  // [p(v) - q(v|x_<i)]_+
+  TargetTokenProb<Tin> p;
+  const float* srow;
+  const float* wu;
+  const float* cm;  // codes of row m, [K, rr]
+  const FF* C;      // [K] in shared memory: L_z - log2 w_z (+inf if w_z = 0)
+  int K, rr;
+  float k2;
+  __device__ float operator()(int v) const {
+    float q = 0.f;
+    const float base = srow[v];
+    for (int z = 0; z < K; ++z) {
+      const FF c = C[z];
+      if (c.hi == INFINITY) continue;
+      q += exp2_rel2(base, corr_at(wu, cm + z * rr, v, z, K, rr), k2, c);
+    }
+    return fmaxf(p(v) - q, 0.f);
+  }
+};
+
+// ---------------------------------------------------------------- draft side
+// Partial log-sum-exps of the draft records: block (row group of 32, z, split);
+// lane = row, warps and splits interleave over the tiles.
+// lsep[sp][m][z] = (max, sum.hi, sum.lo, 0) with sum * 2^max the partial mass.
+constexpr int LSE_WARPS = 16;
+__global__ void __launch_bounds__(LSE_WARPS * 32)
+    k_draft_lse(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
+                float4* __restrict__ lsep) {
+  __shared__ float smx[LSE_WARPS][32];
+  __shared__ FF ssum[LSE_WARPS][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int m = blockIdx.x * 32 + lane, z = blockIdx.y, sp = blockIdx.z;
+  const int step = LSE_WARPS * LSE_SPLIT;
+  float mx = -INFINITY;
+  FF s{0.f, 0.f};
+  auto merge = [&](float2 q) {
+    if (q.y > 0.f) {
+      if (q.x > mx) {
+        s = ff_mulf(s, exp2f(mx - q.x));
+        mx = q.x;
+      }
+      s = ff_addf(s, q.y * exp2f(q.x - mx));
+    }
+  };
+  if (m < M) {
+    const float2* p = partd + (size_t)z * Mpad + m;
+    const size_t st = (size_t)K * Mpad;
+    int t = sp * LSE_WARPS + warp;
+    for (; t + 3 * step < nt; t += 4 * step) {
+      const float2 q0 = p[(size_t)t * st], q1 = p[(size_t)(t + step) * st];
+      const float2 q2 = p[(size_t)(t + 2 * step) * st], q3 = p[(size_t)(t + 3 * step) * st];
+      merge(q0);
+      merge(q1);
+      merge(q2);
+      merge(q3);
+    }
+    for (; t < nt; t += step) merge(p[(size_t)t * st]);
+  }
+  smx[warp][lane] = mx;
+  ssum[warp][lane] = s;
+  __syncthreads();
+  if (warp == 0 && m < M) {
+    float M2 = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < LSE_WARPS; ++w) M2 = fmaxf(M2, smx[w][lane]);
+    FF S{0.f, 0.f};
+    if (M2 != -INFINITY)
+#pragma unroll
+      for (int w = 0; w < LSE_WARPS; ++w) S = ff_add(S, ff_mulf(ssum[w][lane], exp2f(smx[w][lane] - M2)));
+    lsep[((size_t)sp * M + m) * K + z] = make_float4(M2, S.hi, S.lo, 0.f);
+  }
+}
+
+// One block per row m = (n, i): lse2 of every branch, the draft token
+// x_i ~ q_i(.|z-hat) (stream 1), and log2 q_z(x_i) for every branch.
+constexpr int DT_NT = 128;
+__global__ void __launch_bounds__(DT_NT)
+    k_draft_token(const float2* __restrict__ partd, const float4* __restrict__ lsep,
+                  const float* __restrict__ stash, const float* __restrict__ wu,
+                  const float* __restrict__ codes, const int32_t* __restrict__ zhat, int nt, int V,
+                  int K, int rr, int B, int M, int Mpad, float k2, uint64_t seed,
+                  const int64_t* __restrict__ pos, const uint32_t* __restrict__ rnd,
+                  float2* __restrict__ lse2, int32_t* __restrict__ tok, float2* __restrict__ lq2,
+                  uint32_t* __restrict__ ties) {
+  __shared__ FindShared<DT_NT> fs;
+  __shared__ FF sL[32];
+  const int m = blockIdx.x, tid = threadIdx.x;
+  const int n = m / B, i = m - n * B;
+  if (tid < K) {
+    float mx = -INFINITY;
+    for (int sp = 0; sp < LSE_SPLIT; ++sp) mx = fmaxf(mx, lsep[((size_t)sp * M + m) * K + tid].x);
+    FF S{0.f, 0.f};
+    if (mx != -INFINITY)
+      for (int sp = 0; sp < LSE_SPLIT; ++sp) {
+        const float4 q = lsep[((size_t)sp * M + m) * K + tid];
+        S = ff_add(S, ff_mulf(FF{q.y, q.z}, exp2f(q.x - mx)));
+      }
+    const FF L = (mx == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
+                                                   : ff_add(FF{mx, 0.f}, ff_log2(S));
+    sL[tid] = L;
+    lse2[(size_t)m * K + tid] = ff_st(L);
+  }
+  __syncthreads();
+  const int z = zhat[n];
+  const FF L = sL[z];
+  const float u = decision_uniform(seed, 1u, rnd[n], (uint32_t)n, (uint32_t)(pos[n] + i));
+  const float* cm = codes + (size_t)m * K * rr;
+  const float* srow = stash + (size_t)m * V;
+  const DraftTileMass tm{partd + (size_t)z * Mpad + m, (size_t)K * Mpad, L};
+  const BranchTokenProb em{srow, wu, cm + z * rr, z, K, rr, k2, L};
+  const FindOut f = block_find<DT_NT>(nt, V, tm, em, FF{u, 0.f}, 1.f, fs);
+  const int x = f.x >= 0 ? f.x : 0;
+  if (tid == 0) {
+    tok[m] = x;
+    if (f.tie || f.x < 0) atomicOr(&ties[n], (uint32_t)TIE_DRAFT);
+  }
+  if (tid < K) {  // log2 q_z(x) = (base_x + corr_z(x)) k2 - L_z, products exact
+    const FF s = ff_add(ff_prod(srow[x], k2), ff_prod(corr_at(wu, cm + tid * rr, x, tid, K, rr), k2));
+    lq2[(size_t)m * K + tid] = ff_st(ff_sub(s, sL[tid]));
+  }
+}
+
+// One block per sequence, thread t = (i, z) with i = t / K: the category
+// posterior log2 w_{i,z} (Eq. category-posterior) from prefix sums over i of
+// log2 q_z(x_j), q(x_i|x_<i) (Eq. dep-next-token), the per-row constants of
+// the tensor-core verify pass, and the user-visible draft outputs.
+__global__ void __launch_bounds__(1024)
+    k_posterior(const float2* __restrict__ lq2, const float2* __restrict__ lse2,
+                const float* __restrict__ log2pi, const int32_t* __restrict__ zhat,
+                const int32_t* __restrict__ tok, const float* __restrict__ cscale,
+                const float* __restrict__ sw, float k2, int B, int K, float2* __restrict__ w2,
+                float* __restrict__ qtok, float2* __restrict__ vcz, float* __restrict__ vb0,
+                dblast_draft_out out) {
+  __shared__ FF A[1024];
+  __shared__ FF rowv[32];
+  __shared__ float rowb[32];
+  __shared__ float E[1024];
+  const int n = blockIdx.x, t = threadIdx.x;
+  const int i = t / K, z = t - i * K;
+  const bool ok = i < B;
+  const size_t m = (size_t)n * B + (ok ? i : 0);
+  const FF lq = ok ? ff_ld(lq2 + m * K + z) : FF{0.f, 0.f};
+  // exclusive prefix over positions: A[i][z] = sum_{j<i} log2 q_z(x_j)
+  A[t] = (ok && i > 0) ? ff_ld(lq2 + (m - 1) * K + z) : FF{0.f, 0.f};
+  __syncthreads();
+  for (int o = 1; o < B; o <<= 1) {
+    const FF v = (ok && i >= o) ? A[t - o * K] : FF{0.f, 0.f};
+    __syncthreads();
+    if (ok) A[t] = ff_add(v, A[t]);
+    __syncthreads();
+  }
+  const float lp = ok ? log2pi[n * K + z] : -INFINITY;
+  const FF acc = (lp == -INFINITY || A[t].hi == -INFINITY) ? FF{-INFINITY, 0.f}
+                                                           : ff_addf(A[t], lp);
+  __syncthreads();
+  A[t] = acc;
+  __syncthreads();
+  if (ok && z == 0) {
+    float mx = -INFINITY, lmx = -INFINITY;
+    for (int k = 0; k < K; ++k) {
+      mx = fmaxf(mx, A[t + k].hi);
+      lmx = fmaxf(lmx, lse2[m * K + k].x);
+    }
+    FF S{0.f, 0.f};
+    if (mx != -INFINITY)
+      for (int k = 0; k < K; ++k)
+        if (A[t + k].hi != -INFINITY) S = ff_addf(S, ff_exp2(ff_addf(A[t + k], -mx)));
+    rowv[i] = (mx == -INFINITY) ? FF{-INFINITY, 0.f} : ff_add(FF{mx, 0.f}, ff_log2(S));
+    rowb[i] = floorf(lmx);  // B0 of the verify pass: keeps its two factors in range
+  }
+  __syncthreads();
+  const FF lz = ok ? rowv[i] : FF{-INFINITY, 0.f};
+  const bool wdead = acc.hi == -INFINITY || lz.hi == -INFINITY;
+  const FF wz = wdead ? FF{-INFINITY, 0.f} : ff_sub(acc, lz);
+  E[t] = (wdead || lq.hi == -INFINITY) ? 0.f : ff_exp2(ff_add(wz, lq));
+  __syncthreads();
+  if (ok) {
+    const FF Lz = ff_ld(lse2 + m * K + z);
+    w2[m * K + z] = ff_st(wz);
+    const float b0 = rowb[i];
+    vcz[m * K + z] = make_float2(k2 / (cscale[m * K + z] * sw[z]),
+                                 wdead ? -INFINITY : ff_f(ff_addf(ff_sub(wz, Lz), b0)));
+    if (out.logw) out.logw[m * K + z] = wdead ? -INFINITY : ff_f(wz) * LN2;
+    if (out.lse) out.lse[m * K + z] = ff_f(Lz) * LN2;
+    if (z == 0) {
+      FF qt{0.f, 0.f};
+      for (int k = 0; k < K; ++k) qt = ff_addf(qt, E[t + k]);
+      qtok[m] = ff_f(qt);
+      vb0[m] = b0;
+      if (out.q_tok) out.q_tok[m] = ff_f(qt);
+      if (out.tokens) out.tokens[m] = tok[m];
+    }
+  }
+  if (t < K) {
+    if (out.pi) out.pi[n * K + t] = exp2f(log2pi[n * K + t]);
+    if (out.z_hat && t == 0) out.z_hat[n] = zhat[n];
+  }
+}
+
+cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp) {
+  const WsLayout& w = c.wl;
+  const dblast_block_args* a = c.args;
+  const int K = c.head->K;
+  k_draft_lse<<<dim3(ceil_div(w.M, 32), K, LSE_SPLIT), LSE_WARPS * 32, 0, c.stream>>>(
+      wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+  debug_kernel("k_draft_lse", c.stream);
+  k_draft_token<<<w.M, DT_NT, 0, c.stream>>>(
+      wsp<float2>(c, w.off_partd), wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_stash),
+      prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<int32_t>(c, w.off_zhat), w.nt,
+      w.V, K, w.rr, w.B, w.M, w.Mpad, c.k2, a->seed, a->pos, a->round, wsp<float2>(c, w.off_lse2),
+      wsp<int32_t>(c, w.off_tok), wsp<float2>(c, w.off_lq2), wsp<uint32_t>(c, w.off_ties));
+  debug_kernel("k_draft_token", c.stream);
+  dblast_draft_out out{};
+  if (outp) out = *outp;
+  const int pt = ceil_div(w.B * K, 32) * 32;
+  k_posterior<<<w.N, pt, 0, c.stream>>>(
+      wsp<float2>(c, w.off_lq2), wsp<float2>(c, w.off_lse2), wsp<float>(c, w.off_log2pi),
+      wsp<int32_t>(c, w.off_zhat), wsp<int32_t>(c, w.off_tok), wsp<float>(c, w.off_cscale),
+      prp<float>(c, c.pl.off_sw), c.k2, w.B, K, wsp<float2>(c, w.off_w2),
+      wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_vcz), wsp<float>(c, w.off_vb0), out);
+  debug_kernel("k_posterior", c.stream);
+  count_launches(3);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- target side
+// One block per target row: a half-warp per tile of 128 tokens (8 per lane),
+// the tile records partt and the row's lse2t = log2 sum_v 2^{t_v k2} (also as
+// a float pair lt2 for the verify pass).
+constexpr int TS_NT = 256;
+constexpr int TS_HW = TS_NT / 16;  // half-warps per block
+constexpr int TS_NF = 4;           // tiles in flight per half-warp
+static_assert(TS_HW <= 32, "one warp merges the half-warp partials");
+template <typename Tin>
+__global__ void __launch_bounds__(TS_NT)
+    k_target_stats(const Tin* __restrict__ target, int V, int nt, int B, int Bt, int Rt, float k2,
+                   bool vec, float2* __restrict__ partt, float2* __restrict__ lt2,
+                   float* __restrict__ lse_out) {
+  __shared__ float smx[TS_HW];
+  __shared__ FF ssum[TS_HW];
+  const int row = blockIdx.x;
+  const int n = row / Bt, i = row - n * Bt;
+  const int rl = n * (B + 1) + i;
+  const Tin* tr = target + (size_t)row * V;
+  const int hw = threadIdx.x >> 4, hl = threadIdx.x & 15;
+  float rmax = -INFINITY;
+  FF rsum{0.f, 0.f};
+  // every lane of both half-warps runs the shuffles; `valid` gates the results
+  auto tile = [&](int t, const float (&x)[8], bool valid) {
+    float mx = x[0];
+#pragma unroll
+    for (int j = 1; j < 8; ++j) mx = fmaxf(mx, x[j]);
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(FULLMASK, mx, o));
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s += exp2f((x[j] - mx) * k2);
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(FULLMASK, s, o);
+    if (!valid) return;
+    if (hl == 0) partt[(size_t)t * Rt + rl] = make_float2(mx, s);
+    if (mx > rmax) {
+      rsum = ff_mulf(rsum, exp2f((rmax - mx) * k2));
+      rmax = mx;
+    }
+    rsum = ff_addf(rsum, s * exp2f((mx - rmax) * k2));
+  };
+  // TS_NF tiles in flight per half-warp; the loop bounds are uniform over the block
+  const int iters = ceil_div(nt, TS_HW);
+  for (int k = 0; k < iters; k += TS_NF) {
+    float x[TS_NF][8];
+#pragma unroll
+    for (int f = 0; f < TS_NF; ++f) {
+      const int tf = (k + f) * TS_HW + hw;
+      load8(tr, tf * TILE_V + hl * 8, (k + f < iters && tf < nt) ? V : 0, vec, x[f]);
+    }
+#pragma unroll
+    for (int f = 0; f < TS_NF; ++f) {
+      const int tf = (k + f) * TS_HW + hw;
+      tile(tf, x[f], k + f < iters && tf < nt);
+    }
+  }
+  if (hl == 0) {
+    smx[hw] = rmax;
+    ssum[hw] = rsum;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int l = threadIdx.x;
+    const float ml = l < TS_HW ? smx[l] : -INFINITY;
+    float M2 = ml;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M2 = fmaxf(M2, __shfl_xor_sync(FULLMASK, M2, o));
+    FF S{0.f, 0.f};
+    if (M2 != -INFINITY && ml != -INFINITY) S = ff_mulf(ssum[l], exp2f((ml - M2) * k2));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) S = ff_add(S, ff_shfl_xor(S, o));
+    if (l == 0) {
+      const FF L = (M2 == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
+                                                     : ff_add(ff_prod(M2, k2), ff_log2(S));
+      lt2[rl] = ff_st(L);
+      if (lse_out) lse_out[row] = ff_f(L) * LN2;
+    }
+  }
+}
+
+template <typename Tin>
+static cudaError_t target_typed(const StepCtx& c, const dblast_verify_out* o) {
+  const WsLayout& w = c.wl;
+  const int Bt = w.B + (o->has_bonus ? 1 : 0);
+  const int rows = w.N * Bt;
+  const bool vec = (w.V % 8) == 0 && (reinterpret_cast<uintptr_t>(o->target) & 15u) == 0;
+  k_target_stats<Tin><<<rows, TS_NT, 0, c.stream>>>(
+      static_cast<const Tin*>(o->target), w.V, w.nt, w.B, Bt, w.Rt, c.k2, vec,
+      wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), o->lse_target);
+  debug_kernel("k_target_stats", c.stream);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_target_stats(const StepCtx& c, const dblast_verify_out* o) {
+  return c.head->dtype == DBLAST_F32 ? target_typed<float>(c, o)
+                                     : target_typed<__nv_bfloat16>(c, o);
+}
+
+// ---------------------------------------------------------------- verify side
+// Partial sums of the verify records: block (row group of 32, split), lane =
+// row.  avp[sp][m] = (alpha.hi, alpha.lo, R.hi, R.lo).
+constexpr int AVM_WARPS = 16;
+__global__ void __launch_bounds__(AVM_WARPS * 32)
+    k_verify_merge(const float2* __restrict__ partv, int nt, int M, int Mpad,
+                   float4* __restrict__ avp) {
+  __shared__ FF sa[AVM_WARPS][32], sr[AVM_WARPS][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int m = blockIdx.x * 32 + lane, sp = blockIdx.y;
+  const int step = AVM_WARPS * AV_SPLIT;
+  FF a{0.f, 0.f}, r{0.f, 0.f};
+  if (m < M) {
+    int t = sp * AVM_WARPS + warp;
+    for (; t + step < nt; t += 2 * step) {
+      const float2 q0 = partv[(size_t)t * Mpad + m], q1 = partv[(size_t)(t + step) * Mpad + m];
+      a = ff_addf(ff_addf(a, q0.x), q1.x);
+      r = ff_addf(ff_addf(r, q0.y), q1.y);
+    }
+    for (; t < nt; t += step) {
+      const float2 q = partv[(size_t)t * Mpad + m];
+      a = ff_addf(a, q.x);
+      r = ff_addf(r, q.y);
+    }
+  }
+  sa[warp][lane] = a;
+  sr[warp][lane] = r;
+  __syncthreads();
+  if (warp == 0 && m < M) {
+    FF A{0.f, 0.f}, R{0.f, 0.f};
+#pragma unroll
+    for (int w = 0; w < AVM_WARPS; ++w) {
+      A = ff_add(A, sa[w][lane]);
+      R = ff_add(R, sr[w][lane]);
+    }
+    avp[(size_t)sp * M + m] = make_float4(A.hi, A.lo, R.hi, R.lo);
+  }
+}
+
+// One block per sequence: acceptance (stream 2), residual or bonus draw
+// (stream 3), expected lengths, emitted tokens, state update.
+constexpr int VF_NT = 256;
+template <typename Tin>
+__global__ void __launch_bounds__(VF_NT)
+    k_verify_final(const Tin* __restrict__ target, const float* __restrict__ stash,
+                   const float* __restrict__ wu, const float* __restrict__ codes,
+                   const float2* __restrict__ lse2, const float2* __restrict__ w2,
+                   const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
+                   const float2* __restrict__ partv, const float2* __restrict__ partt,
+                   const float4* __restrict__ avp, const int32_t* __restrict__ tok,
+                   const uint32_t* __restrict__ ties_draft, int V, int K, int rr, int B, int Bt,
+                   int nt, int M, int Mpad, int Rt, float k2, uint64_t seed,
+                   int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
+                   dblast_verify_out out) {
+  __shared__ FindShared<VF_NT> fs;
+  __shared__ FF sC[32];
+  __shared__ int sL;
+  __shared__ uint32_t sties;
+  __shared__ FF sR;
+  const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
+  const int64_t p0 = pos[n];
+  const uint32_t rd = rnd[n];
+  if (tid < 32) {
+    // lane i: p(x_i), q(x_i|x_<i), acceptance
+    uint32_t ties = ties_draft[n];
+    float A = 0.f, alpha = 0.f, ptok = 0.f, qtok = 1.f, u2 = 0.f;
+    bool acc_ok = false;
+    if (lane < B) {
+      const int m = n * B + lane;
+      const int x = min(max(tok[m], 0), V - 1);
+      const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
+      const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
+      ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
+      qtok = qtok_ws[m];
+      const float ratio = ptok / qtok;
+      A = fminf(1.f, ratio);
+      FF al{0.f, 0.f};
+      for (int sp = 0; sp < AV_SPLIT; ++sp) {
+        const float4 q = avp[(size_t)sp * M + m];
+        al = ff_add(al, FF{q.x, q.y});
+      }
+      alpha = ff_f(al);
+      u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
+      acc_ok = u2 < ratio;
+      if (out.p_tok) out.p_tok[m] = ptok;
+      if (out.accept_prob) out.accept_prob[m] = A;
+      if (out.alpha) out.alpha[m] = alpha;
+    }
+    const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
+    const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
+    const int L = rej ? (__ffs(rej) - 1) : B;
+    // acceptance ties only for the positions that were tested (i <= L)
+    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha (products in lane order)
+    float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float ta = __shfl_up_sync(FULLMASK, cA, o);
+      const float tl = __shfl_up_sync(FULLMASK, cAl, o);
+      if (lane >= o) {
+        cA *= ta;
+        cAl *= tl;
+      }
+    }
+    FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
+    FF R{0.f, 0.f};
+    if (L < B && lane < AV_SPLIT) {
+      const float4 q = avp[(size_t)lane * M + n * B + L];
+      R = FF{q.z, q.w};
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      R = ff_add(R, ff_shfl_xor(R, o));
+      el = ff_add(el, ff_shfl_xor(el, o));
+      ea = ff_add(ea, ff_shfl_xor(ea, o));
+    }
+    if (L < B && lane < K) {  // normalisers of the rejected row: L_z - log2 w_z
+      const size_t mz = (size_t)(n * B + L) * K + lane;
+      const FF wz = ff_ld(w2 + mz);
+      sC[lane] = (wz.hi == -INFINITY) ? FF{INFINITY, 0.f} : ff_sub(ff_ld(lse2 + mz), wz);
+    }
+    if (lane == 0) {
+      if (out.exp_len) out.exp_len[n] = ff_f(el);
+      if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
+      sL = L;
+      sties = ties;
+      sR = R;
+    }
+  }
+  __syncthreads();
+  const int L = sL;
+  const FF Rm = sR;
+  int extra = -1;
+  bool tie = false;
+  uint32_t tbits = 0;
+  const int irow = (L < B) ? L : B;  // target row of the extra token
+  if ((L < B) || (Bt > B)) {
+    const float u3 = decision_uniform(seed, 3u, rd, (uint32_t)n, (uint32_t)(p0 + irow));
+    const int rl = n * (B + 1) + irow;
+    const FF Lt = ff_ld(lt2 + rl);
+    const TargetTokenProb<Tin> pv{target + ((size_t)n * Bt + irow) * V, k2, Lt};
+    bool from_p = (L >= B);
+    if (L < B) {
+      const int m = n * B + L;
+      const float Rf = ff_f(Rm);
+      if (Rf < TIE_TOL) tbits |= TIE_RMASS;
+      if (Rf > 0.f) {
+        const ResidualTokenMass<Tin> rm{pv, stash + (size_t)m * V, wu,
+                                        codes + (size_t)m * K * rr, sC, K, rr, k2};
+        const FindOut f = block_find<VF_NT>(nt, V, ResidTileMass{partv + m, (size_t)Mpad}, rm,
+                                            ff_mulf(Rm, u3), Rf, fs);
+        extra = f.x;
+        tie = f.tie;
+      }
+      if (extra < 0) {  // no positive residual mass left by rounding: draw from p
+        from_p = true;
+        tie = true;
+        tbits |= TIE_RMASS;
+      }
+    }
+    if (from_p) {
+      const FindOut f = block_find<VF_NT>(nt, V, TargetTileMass{partt + rl, (size_t)Rt, k2, Lt},
+                                          pv, FF{u3, 0.f}, 1.f, fs);
+      extra = f.x >= 0 ? f.x : 0;
+      tie = tie || f.tie || f.x < 0;
+    }
+  }
+  if (tid == 0) {
+    const uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u);
+    const int ne = L + (extra >= 0 ? 1 : 0);
+    if (out.accepted) out.accepted[n] = L;
+    if (out.n_emitted) out.n_emitted[n] = ne;
+    if (out.tie_flags) out.tie_flags[n] = ties;
+    pos[n] = p0 + ne;
+    rnd[n] = rd + 1u;
+  }
+  if (out.emitted) {
+    for (int j = tid; j < B + 1; j += VF_NT) {
+      int val = -1;
+      if (j < L) val = tok[n * B + j];
+      else if (j == L && extra >= 0) val = extra;
+      out.emitted[(size_t)n * (B + 1) + j] = val;
+    }
+  }
+}
+
+template <typename Tin>
+static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out* o) {
+  const int Bt = c.Bt;
+  const WsLayout& w = c.wl;
+  k_verify_merge<<<dim3(ceil_div(w.M, 32), AV_SPLIT), AVM_WARPS * 32, 0, c.stream>>>(
+      wsp<float2>(c, w.off_partv), w.nt, w.M, w.Mpad, wsp<float4>(c, w.off_av));
+  debug_kernel("k_verify_merge", c.stream);
+  k_verify_final<Tin><<<w.N, VF_NT, 0, c.stream>>>(
+      static_cast<const Tin*>(o->target), wsp<float>(c, w.off_stash), prp<float>(c, c.pl.off_wu),
+      wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2), wsp<float2>(c, w.off_w2),
+      wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
+      wsp<float2>(c, w.off_partt), wsp<float4>(c, w.off_av), wsp<int32_t>(c, w.off_tok),
+      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, Bt, w.nt, w.M, w.Mpad, w.Rt, c.k2,
+      c.args->seed, c.args->pos, c.args->round, *o);
+  debug_kernel("k_verify_final", c.stream);
+  count_launches(2);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {
+  return c.head->dtype == DBLAST_F32 ? verify_final_typed<float>(c, o)
+                                     : verify_final_typed<__nv_bfloat16>(c, o);
+}
+
+}  // namespace dblast

@@ -166,68 +166,84 @@ cudaError_t launch_prep(const dblast_head* h, const PrepLayout& pl, cudaStream_t
 }
 
 // ------------------------------------------------------------- prior
-// One CTA per sequence: l = Wp a + bp, pi = softmax(l / Z_T) (Z_T = 0: one-hot
-// argmax, lowest index on ties), z-hat by an inverse-CDF draw (stream 0).
+// One CTA per sequence: l = Wp a + bp (a warp per category, 16-byte loads),
+// then warp 0 with lane z: pi = softmax(l / Z_T) (Z_T = 0: one-hot argmax,
+// lowest index on ties) and z-hat by an inverse-CDF draw (stream 0).
 template <typename Tin>
-__global__ void k_prior(const Tin* __restrict__ Wp, const float* __restrict__ bp,
-                        const Tin* __restrict__ anchor, const Tin* __restrict__ hidden, int H,
-                        int K, int B, float zt, uint64_t seed, const int64_t* __restrict__ pos,
-                        const uint32_t* __restrict__ rnd, int32_t* __restrict__ zhat_ws,
-                        float* __restrict__ log2pi_ws, uint32_t* __restrict__ ties,
-                        int32_t* __restrict__ zhat_out, float* __restrict__ pi_out) {
-  // zhat_out / pi_out may be null: the draft finalize kernel also writes them
+__global__ void __launch_bounds__(256)
+    k_prior(const Tin* __restrict__ Wp, const float* __restrict__ bp,
+            const Tin* __restrict__ anchor, const Tin* __restrict__ hidden, int H, int K, int B,
+            float zt, uint64_t seed, const int64_t* __restrict__ pos,
+            const uint32_t* __restrict__ rnd, int32_t* __restrict__ zhat_ws,
+            float* __restrict__ log2pi_ws, uint32_t* __restrict__ ties) {
   __shared__ float ell[32];
   const int n = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const Tin* a = anchor ? anchor + (size_t)n * H : hidden + (size_t)n * B * H;
   for (int z = warp; z < K; z += blockDim.x >> 5) {
+    const Tin* w = Wp + (size_t)z * H;
     float acc = 0.f;
-    for (int hh = lane; hh < H; hh += 32) acc = fmaf(ldf(Wp + (size_t)z * H + hh), ldf(a + hh), acc);
+#pragma unroll 4
+    for (int h0 = lane * 8; h0 < H; h0 += 256) {
+      float w8[8], a8[8];
+      load8(w, h0, H, true, w8);
+      load8(a, h0, H, true, a8);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], a8[j], acc);
+    }
     acc = warp_sum(acc);
     if (lane == 0) ell[z] = acc + (bp ? bp[z] : 0.f);
   }
   __syncthreads();
-  if (threadIdx.x != 0) return;
-  double pi[32];
+  if (warp != 0) return;
+  const bool on = lane < K;
+  const float lz = on ? ell[lane] : -INFINITY;
+  float pz;
   if (zt == 0.f) {
-    int best = 0;
-    for (int z = 1; z < K; ++z)
-      if (ell[z] > ell[best]) best = z;
-    for (int z = 0; z < K; ++z) pi[z] = (z == best) ? 1.0 : 0.0;
+    float best = lz;
+    int bi = on ? lane : 32;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ob > best || (ob == best && oi < bi)) {
+        best = ob;
+        bi = oi;
+      }
+    }
+    pz = (lane == bi) ? 1.f : 0.f;
   } else {
-    double mx = -INFINITY, tot = 0.0;
-    for (int z = 0; z < K; ++z) mx = fmax(mx, (double)ell[z] / zt);
-    for (int z = 0; z < K; ++z) {
-      pi[z] = exp((double)ell[z] / zt - mx);
-      tot += pi[z];
-    }
-    for (int z = 0; z < K; ++z) pi[z] /= tot;
+    const float x = on ? lz / zt : -INFINITY;
+    const float mx = warp_max(x);
+    const float e = on ? exp2f((x - mx) * LOG2E) : 0.f;
+    pz = e / warp_sum(e);
   }
-  const double u = decision_uniform(seed, 0u, rnd[n], (uint32_t)n, (uint32_t)pos[n]);
-  double cum = 0.0, tot = 0.0;
-  for (int z = 0; z < K; ++z) tot += pi[z];
-  const double target = u * tot;
-  int zh = -1;
-  double margin = 1.0;
-  for (int z = 0; z < K; ++z) {
-    const double lo = cum;
-    cum += pi[z];
-    if (zh < 0 && cum > target) {
-      zh = z;
-      margin = fmin(target - lo, cum - target) / tot;
-    }
+  // inverse CDF over the categories in index order (float-pair prefix sums)
+  const float u = decision_uniform(seed, 0u, rnd[n], (uint32_t)n, (uint32_t)pos[n]);
+  FF cum{pz, 0.f};
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const FF t{__shfl_up_sync(0xffffffffu, cum.hi, o), __shfl_up_sync(0xffffffffu, cum.lo, o)};
+    if (lane >= o) cum = ff_add(t, cum);
   }
-  if (zh < 0) {
-    for (int z = K - 1; z >= 0; --z)
-      if (pi[z] > 0.0) { zh = z; break; }
-    margin = 0.0;
+  const FF tot{__shfl_sync(0xffffffffu, cum.hi, 31), __shfl_sync(0xffffffffu, cum.lo, 31)};
+  const FF target = ff_mulf(tot, u);
+  const unsigned hit = __ballot_sync(0xffffffffu, on && ff_gt(cum, target));
+  const unsigned posm = __ballot_sync(0xffffffffu, on && pz > 0.f);
+  int zh;
+  float margin = 0.f;
+  if (hit) {
+    zh = __ffs(hit) - 1;
+    const FF c{__shfl_sync(0xffffffffu, cum.hi, zh), __shfl_sync(0xffffffffu, cum.lo, zh)};
+    const float p = __shfl_sync(0xffffffffu, pz, zh);
+    margin = fminf(ff_f(ff_sub(target, ff_addf(c, -p))), ff_f(ff_sub(c, target))) / ff_f(tot);
+  } else {
+    zh = posm ? 31 - __clz(posm) : 0;
   }
-  if (zt != 0.f && margin < (double)TIE_TOL) atomicOr(&ties[n], TIE_ZHAT);
-  zhat_ws[n] = zh;
-  if (zhat_out) zhat_out[n] = zh;
-  for (int z = 0; z < K; ++z) {
-    log2pi_ws[n * K + z] = pi[z] > 0.0 ? (float)log2(pi[z]) : -INFINITY;
-    if (pi_out) pi_out[n * K + z] = (float)pi[z];
+  if (lane == 0) {
+    if (zt != 0.f && margin < TIE_TOL) atomicOr(&ties[n], TIE_ZHAT);
+    zhat_ws[n] = zh;
   }
+  if (on) log2pi_ws[n * K + lane] = pz > 0.f ? log2f(pz) : -INFINITY;
 }
 
 // Deterministic split-K reduction of the codes, the constant code for e, the
@@ -281,25 +297,33 @@ template <typename Tin> static cudaError_t prior_codes_typed(const StepCtx& c) {
       static_cast<const Tin*>(h->Wp), h->bp, static_cast<const Tin*>(a->anchor),
       static_cast<const Tin*>(a->hidden), h->H, h->K, a->B, a->z_temperature, a->seed, a->pos,
       a->round, wsp<int32_t>(c, w.off_zhat), wsp<float>(c, w.off_log2pi),
-      wsp<uint32_t>(c, w.off_ties), nullptr, nullptr);
+      wsp<uint32_t>(c, w.off_ties));
   debug_kernel("k_prior", s);
   // codes: split-K partials go to the stash region (not yet written by this call)
   const int Nb = h->K * w.rr;
-  int nsplit = max(1, min(16, h->H / 256));
-  nsplit = max(1, min(nsplit, (int)(((size_t)w.M * h->V) / ((size_t)w.M * Nb))));
-  const int hchunk = ceil_div(ceil_div(h->H, nsplit), 32) * 32;
   float* part = wsp<float>(c, w.off_stash);
-  ExpanderCols<Tin> bf{static_cast<const Tin*>(h->Vf), nullptr, h->H, h->r, w.rr};
-  dim3 grid(ceil_div(w.M, 64), ceil_div(Nb, 64), ceil_div(h->H, hchunk));
-  k_gemm_simt<Tin><<<grid, 256, 0, s>>>(static_cast<const Tin*>(a->hidden), w.M, h->H, bf, Nb,
-                                        hchunk, part, (size_t)w.M * Nb);
-  debug_kernel("k_gemm_simt", s);
+  int nsplit = 1;
+  if (c.tc) {
+    cudaError_t e = launch_codes_tc(c, part, &nsplit);
+    if (e != cudaSuccess) return e;
+  } else {
+    nsplit = max(1, min(16, h->H / 256));
+    nsplit = max(1, min(nsplit, (int)(((size_t)w.M * h->V) / ((size_t)w.M * Nb))));
+    const int hchunk = ceil_div(ceil_div(h->H, nsplit), 32) * 32;
+    ExpanderCols<Tin> bf{static_cast<const Tin*>(h->Vf), nullptr, h->H, h->r, w.rr};
+    dim3 grid(ceil_div(w.M, 64), ceil_div(Nb, 64), ceil_div(h->H, hchunk));
+    k_gemm_simt<Tin><<<grid, 256, 0, s>>>(static_cast<const Tin*>(a->hidden), w.M, h->H, bf, Nb,
+                                          hchunk, part, (size_t)w.M * Nb);
+    debug_kernel("k_gemm_simt", s);
+    count_launches(1);
+    nsplit = (int)grid.z;
+  }
   const int warps = w.Mpad * h->K;
   k_codes_finish<<<ceil_div(warps * 32, 256), 256, 0, s>>>(
-      part, (int)grid.z, w.M, w.Mpad, h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes),
+      part, nsplit, w.M, w.Mpad, h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes),
       wsp<float>(c, w.off_cscale), wsp<__half>(c, w.off_cop));
   debug_kernel("k_codes_finish", s);
-  count_launches(3);
+  count_launches(2);
   return cudaGetLastError();
 }
 

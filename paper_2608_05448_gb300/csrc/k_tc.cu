@@ -129,10 +129,10 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
 }
 
 // instruction descriptor, kind::f16: fp32 accumulate, A/B both bf16 or both
-// fp16, both K-major, M = 128, N = BN
-__host__ __device__ constexpr uint32_t idesc_f16(bool bf16) {
+// fp16, both K-major, M = 128, N = n
+__host__ __device__ constexpr uint32_t idesc_f16(bool bf16, int n) {
   return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) |
-         (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
+         (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
 }
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -173,82 +173,402 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// ------------------------------------------------------------ parameters
+// ------------------------------------------------------------ draft pass
+// 128 x 256 tiles: TMEM columns [0, 256) hold the base accumulator, [256, 512)
+// the branch accumulator of one component.  12 warps: warp 0 issues TMA, warp
+// 1 issues MMAs and owns TMEM, warps 4-11 are the epilogue (two per TMEM lane
+// quarter, 128 columns each).  Warpgroup 0 gives registers to the epilogue
+// warpgroups with setmaxnreg (56 + 2 x 224 = 3 x 168 per thread).
+constexpr int DBN = 256;                     // vocabulary tokens per tile
+constexpr int DSTAGES = 4;
+constexpr int DSTAGE_A = BM * BK * 2;        // 16 KB
+constexpr int DSTAGE_B = DBN * BK * 2;       // 32 KB
+constexpr int DSTAGE = DSTAGE_A + DSTAGE_B;  // 48 KB
+constexpr int DCOLS = DBN / 2;               // columns per epilogue thread
+constexpr int D_THREADS = 384;
+constexpr int DREG = 168, DREG_LO = 56, DREG_HI = 224;
+static_assert(4 * DREG_LO + 8 * DREG_HI == 12 * DREG, "register split must equal the launch pool");
+constexpr int D_EPI = 256;                   // epilogue threads
+constexpr int DAZ_BYTES = KMAX * D_EPI * 4;  // per-thread branch scales
+constexpr size_t DSMEM = (size_t)DSTAGES * DSTAGE + DAZ_BYTES + 256 + 1024;
+
 struct Params {
   int mode;
-  int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles
-  int nb;                    // base stages per tile (H / BK)
-  int ncs;                   // branch stages per tile (KC / BK); 0 in prep mode
-  int K, rp, zps;            // components, padded rank, components per branch stage
-  int M, V, Mpad;            // valid rows, vocabulary, padded rows
+  int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles, tiles (x ksplit in prep mode)
+  int nb;                    // base stages per tile
+  int K, rp, zps;            // components, padded rank, components per 64-wide block
+  int M, V, Mpad;            // valid rows, vocabulary (B-operand rows), padded rows
   float k2;                  // log2(e) / T
   const float* vbias;        // [V] or null
   const float* cscale;       // [Mpad, K]
   const float* sw;           // [K]
   float* stash;              // [M, V]
   float2* partd;             // [nt, K, Mpad]
-  float* wu;                 // prep output [V, rows_total]
-  int prep_rows;             // K * rr in prep mode
+  float* wu;                 // prep output [ksplit][V, prep_rows]
+  int prep_rows;             // valid A rows in prep mode
+  size_t split_stride;       // elements between the split-K partial outputs
   DevStatus* status;
   uint32_t spin_limit;
 };
 
-// The item sequence consumed by the MMA warp and produced by the TMA warp:
-// for tile slot s = 0 .. my_tiles, base stages of tile s with the branch
-// stages of tile s-1 spread between them (after the last tile: the branch
-// stages of the last tile).
-__device__ __forceinline__ int ins_point(int c, int nb, int ncs) {
-  return ((c + 1) * nb) / (ncs + 1);
-}
-
-__device__ __forceinline__ void tile_of(const Params& P, int slot, int* mt, int* vt) {
+// tile `slot` of this CTA: split (prep mode), M tile, vocabulary tile; the
+// order is vocabulary-major so concurrent CTAs share the B tile through L2
+__device__ __forceinline__ void tile_of(const Params& P, int slot, int* sp, int* mt, int* vt) {
   const int t = (int)blockIdx.x + slot * (int)gridDim.x;
-  *vt = t / P.n_mt;
-  *mt = t - *vt * P.n_mt;
+  const int per = P.n_mt * P.n_vt;
+  *sp = t / per;
+  const int r = t - *sp * per;
+  *vt = r / P.n_mt;
+  *mt = r - *vt * P.n_mt;
 }
 
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+// The item sequence of slot s (consumed by the MMA thread, produced by the TMA
+// thread): the base stages of tile s, with the branch items (one per
+// component) of tile s-1 inserted before base stage ins_point(z).  The last
+// slot (s == my_tiles) holds only the branch items of the last tile.
+__device__ __forceinline__ int ins_point(int z, int nb, int nz) { return ((z + 1) * nb) / (nz + 2); }
+__device__ __forceinline__ bool is_branch(int jb, int zd, int nbv, int nzv) {
+  return zd < nzv && (jb >= nbv || jb == ins_point(zd, nbv, nzv));
+}
+
+__device__ __noinline__ void draft_producer(const Params& P, const CUtensorMap* tm_a,
+                                            const CUtensorMap* tm_b, const CUtensorMap* tm_ca,
+                                            const CUtensorMap* tm_cb, unsigned char* stages,
+                                            uint64_t* full, uint64_t* empty, const Ctl& ctl,
+                                            int my_tiles) {
+  int stage = 0;
+  uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
+  bool ok = true;
+  const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
+  for (int slot = 0; slot <= my_tiles && ok; ++slot) {
+    const int nbv = (slot < my_tiles) ? P.nb : 0;
+    const int nzv = (slot >= 1) ? nzK : 0;
+    int sp = 0, mt = 0, vt = 0, psp = 0, pmt = 0, pvt = 0;
+    if (slot < my_tiles) tile_of(P, slot, &sp, &mt, &vt);
+    if (slot >= 1) tile_of(P, slot - 1, &psp, &pmt, &pvt);
+    int zd = 0;
+    for (int j = 0; j < nbv + nzv; ++j) {
+      const int jb = j - zd;
+      const bool br = is_branch(jb, zd, nbv, nzv);
+      if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) {
+        ok = false;
+        break;
+      }
+      unsigned char* sa = stages + stage * DSTAGE;
+      mbar_arrive_expect_tx(&full[stage], DSTAGE);
+      if (!br) {
+        const int kx = (sp * P.nb + jb) * BK;
+        tma_load_2d(sa, tm_a, &full[stage], kx, mt * BM);
+        tma_load_2d(sa + DSTAGE_A, tm_b, &full[stage], kx, vt * DBN);
+      } else {
+        const int kx = (zd / P.zps) * BK;
+        tma_load_2d(sa, tm_ca, &full[stage], kx, pmt * BM);
+        tma_load_2d(sa + DSTAGE_A, tm_cb, &full[stage], kx, pvt * DBN);
+        ++zd;
+      }
+      issued_mask |= 1u << stage;
+      issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+      if (++stage == DSTAGES) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  // copies still in flight after an abort: wait (bounded) before leaving
+  for (int s = 0; s < DSTAGES; ++s)
+    if (issued_mask & (1u << s)) {
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
+             (globaltimer() - t0) < 2000000000ull) {
+      }
+    }
+}
+
+__device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned char* stages,
+                                       uint64_t* full, uint64_t* empty, uint64_t* bfull,
+                                       uint64_t* bempty, uint64_t* cfull, uint64_t* cempty,
+                                       uint64_t* done, const Ctl& ctl, int my_tiles) {
+  const uint32_t id_base = idesc_f16(true, DBN);
+  const uint32_t id_corr = idesc_f16(false, DBN);
+  int stage = 0;
+  uint32_t phase = 0, cuse = 0;
+  bool ok = true;
+  const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
+  for (int slot = 0; slot <= my_tiles && ok; ++slot) {
+    const int nbv = (slot < my_tiles) ? P.nb : 0;
+    const int nzv = (slot >= 1) ? nzK : 0;
+    int zd = 0;
+    for (int j = 0; j < nbv + nzv; ++j) {
+      const int jb = j - zd;
+      const bool br = is_branch(jb, zd, nbv, nzv);
+      if (!br && jb == 0) {  // the epilogue has taken the previous base accumulator
+        if (!mbar_wait(bempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 2)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+      }
+      if (br) {  // the epilogue has taken the previous branch accumulator
+        if (!mbar_wait(cempty, (cuse & 1u) ^ 1u, ctl, 4)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+      }
+      if (!mbar_wait(&full[stage], phase, ctl, 3)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t sa = smem_u32(stages + stage * DSTAGE);
+      const uint32_t sb = sa + DSTAGE_A;
+      if (!br) {
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          umma(tmem, sdesc(sa + k * 32), sdesc(sb + k * 32), id_base, (jb > 0 || k > 0) ? 1u : 0u);
+        umma_commit(&empty[stage]);
+        if (jb == nbv - 1) umma_commit(bfull);
+      } else {
+        // component zd of the previous tile: hi.hi + hi.lo + lo.hi
+        const uint32_t dcol = tmem + (uint32_t)DBN;
+        const int o = (zd % P.zps) * 2 * P.rp;
+        for (int kk = 0; kk < P.rp; kk += 16) {
+          const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
+          umma(dcol, sdesc(sa + hi), sdesc(sb + hi), id_corr, kk > 0 ? 1u : 0u);
+          umma(dcol, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
+          umma(dcol, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
+        }
+        umma_commit(cfull);
+        umma_commit(&empty[stage]);
+        ++cuse;
+        ++zd;
+      }
+      if (++stage == DSTAGES) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  // wait (bounded) for every MMA this thread issued before TMEM is freed
+  umma_commit(done);
+  const uint64_t t0 = globaltimer();
+  while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
+  }
+}
+
+__device__ __forceinline__ void tmem_ld16_raw(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// Volatile on purpose: the math on one TMEM chunk must stay ahead of the
+// next chunk's tcgen05.ld, or the compiler keeps every chunk live at once.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ void pin(float& x) { asm volatile("" : "+f"(x)); }
+
+// Epilogue: per tile, the base accumulator plus b_v becomes the stash; then
+// for every component z the record (ref, sum 2^{t_v}) of this thread's 128
+// columns, t_v = D_z a_z + (base_v + b_v) k2 - ref, with ref = k2 max_v
+// (base_v + b_v) taken once per tile.  A sum outside [2^-100, 2^100] (a branch
+// offset far from the base logits) is redone against the exact maximum.
+__device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, int warp, int lane,
+                                            float* az, uint64_t* bfull, uint64_t* bempty,
+                                            uint64_t* cfull, uint64_t* cempty, const Ctl& ctl,
+                                            int my_tiles) {
+  const int ew = warp - 4;
+  const int q = warp & 3;        // TMEM lane quarter of this warp
+  const int half = ew >> 2;      // which 128 columns of the tile
+  const int row = q * 32 + lane;
+  const int et = ew * 32 + lane;
+  const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+  uint32_t cuse = 0;
+  for (int slot = 0; slot < my_tiles; ++slot) {
+    int sp, mt, vt;
+    tile_of(P, slot, &sp, &mt, &vt);
+    const int m = mt * BM + row;
+    const int v0 = vt * DBN + half * DCOLS;
+    float bk[DCOLS];
+    if (P.mode == MODE_DRAFT) {
+      // branch scales and vocabulary bias while the main loop still runs
+      for (int z = 0; z < P.K; ++z) az[z * D_EPI + et] = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
+      if (P.vbias && v0 + DCOLS <= P.V) {
+        const float4* vb = reinterpret_cast<const float4*>(P.vbias + v0);
+#pragma unroll
+        for (int j = 0; j < DCOLS / 4; ++j) {
+          const float4 t = __ldg(vb + j);
+          bk[4 * j] = t.x;
+          bk[4 * j + 1] = t.y;
+          bk[4 * j + 2] = t.z;
+          bk[4 * j + 3] = t.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < DCOLS; ++j) bk[j] = (P.vbias && v0 + j < P.V) ? __ldg(P.vbias + v0 + j) : 0.f;
+      }
+    }
+    if (!mbar_wait(bfull, (uint32_t)slot & 1u, ctl, 5)) break;
+    tc_fence_after();
+#pragma unroll
+    for (int cc = 0; cc < DCOLS / 16; ++cc) {
+      uint32_t r[16];
+      tmem_ld16_raw(tmem + lane_off + (uint32_t)(half * DCOLS + cc * 16), r);
+      tmem_wait_ld();
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        bk[cc * 16 + j] = (P.mode == MODE_DRAFT) ? bk[cc * 16 + j] + __uint_as_float(r[j])
+                                                 : __uint_as_float(r[j]);
+        pin(bk[cc * 16 + j]);
+      }
+    }
+    // the base accumulator is in registers: hand TMEM back to the MMA thread
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bempty);
+
+    if (P.mode == MODE_PREP) {
+      if (m < P.prep_rows) {
+        float* out = P.wu + (size_t)sp * P.split_stride;
+#pragma unroll
+        for (int j = 0; j < DCOLS; ++j) {
+          const int v = v0 + j;
+          if (v < P.V) out[(size_t)v * P.prep_rows + m] = bk[j];
+        }
+      }
+      continue;
+    }
+
+    // stash W h + b
+    if (m < P.M) {
+      float* srow = P.stash + (size_t)m * P.V + v0;
+      if (v0 + DCOLS <= P.V && (P.V & 3) == 0) {
+#pragma unroll
+        for (int j = 0; j < DCOLS; j += 4)
+          *reinterpret_cast<float4*>(srow + j) = make_float4(bk[j], bk[j + 1], bk[j + 2], bk[j + 3]);
+      } else {
+        for (int j = 0; j < DCOLS; ++j)
+          if (v0 + j < P.V) srow[j] = bk[j];
+      }
+    }
+    // reference and scaled base: bk_j <- (base_j + b_j) k2 - ref (-inf past V)
+    float bmax = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < DCOLS; ++j)
+      if (v0 + j < P.V) bmax = fmaxf(bmax, bk[j]);
+    const bool live = v0 < P.V;
+    const float ref = live ? bmax * P.k2 : 0.f;
+#pragma unroll
+    for (int j = 0; j < DCOLS; ++j) bk[j] = (v0 + j < P.V) ? fmaf(bk[j], P.k2, -ref) : -INFINITY;
+
+    const int rec = vt * 2 + half;
+    bool ok = true;
+    for (int z = 0; z < P.K; ++z) {
+      if (!mbar_wait(cfull, cuse & 1u, ctl, 6)) {
+        ok = false;
+        break;
+      }
+      ++cuse;
+      tc_fence_after();
+      const float a = az[z * D_EPI + et];
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+      for (int cc = 0; cc < DCOLS / 16; ++cc) {
+        uint32_t r[16];
+        tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 16; j += 4) {
+          s0 += ex2(fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]));
+          s1 += ex2(fmaf(__uint_as_float(r[j + 1]), a, bk[cc * 16 + j + 1]));
+          s2 += ex2(fmaf(__uint_as_float(r[j + 2]), a, bk[cc * 16 + j + 2]));
+          s3 += ex2(fmaf(__uint_as_float(r[j + 3]), a, bk[cc * 16 + j + 3]));
+        }
+      }
+      float sum = (s0 + s1) + (s2 + s3);
+      float rz = ref;
+      const bool bad = live && !(sum >= 0x1p-100f && sum <= 0x1p100f);
+      if (__any_sync(0xffffffffu, bad)) {
+        // exact maximum of this thread's values, then the sum against it
+        float mx = -INFINITY;
+#pragma unroll
+        for (int cc = 0; cc < DCOLS / 16; ++cc) {
+          uint32_t r[16];
+          tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) mx = fmaxf(mx, fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]));
+          pin(mx);
+        }
+        float s = 0.f;
+#pragma unroll
+        for (int cc = 0; cc < DCOLS / 16; ++cc) {
+          uint32_t r[16];
+          tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) s += ex2(fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]) - mx);
+        }
+        if (bad) {
+          sum = s;
+          rz = ref + mx;
+        }
+      }
+      // the branch accumulator is read: hand it back
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(cempty);
+      if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(rz, sum);
+    }
+    if (!ok) break;
+  }
+}
+
+__global__ void __launch_bounds__(D_THREADS, 1)
     k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
               const Params P) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* stage_base = smem;
-  float2* red = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + RED_BYTES);
-  uint64_t* full = bars;                 // [STAGES]
-  uint64_t* empty = bars + STAGES;       // [STAGES]
-  uint64_t* bfull = bars + 2 * STAGES;   // [2] base accumulator ready
-  uint64_t* bempty = bfull + 2;          // [2] base accumulator free
-  uint64_t* cfull = bfull + 4;           // [2] branch accumulator ready
-  uint64_t* cempty = bfull + 6;          // [2] branch accumulator free
-  uint64_t* done = bfull + 8;            // [1] all MMAs of this CTA finished
-  uint64_t* redw = bfull + 9;            // [1] all epilogue records of a tile written
-  uint64_t* redm = bfull + 10;           // [1] all records of a tile merged
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 11);
+  unsigned char* stages = smem;
+  float* az = reinterpret_cast<float*>(smem + DSTAGES * DSTAGE);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DSTAGES * DSTAGE + DAZ_BYTES);
+  uint64_t* full = bars;                 // [DSTAGES]
+  uint64_t* empty = bars + DSTAGES;      // [DSTAGES]
+  uint64_t* bfull = bars + 2 * DSTAGES;  // base accumulator ready
+  uint64_t* bempty = bfull + 1;          // base accumulator taken (8 epilogue warps)
+  uint64_t* cfull = bfull + 2;           // branch accumulator ready
+  uint64_t* cempty = bfull + 3;          // branch accumulator taken (8 epilogue warps)
+  uint64_t* done = bfull + 4;            // every MMA of this CTA finished
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 5);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int my_tiles = (P.n_tiles > (int)blockIdx.x)
                            ? (P.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
                            : 0;
-  Ctl ctl{P.spin_limit, abort_flag, P.status};
+  const Ctl ctl{P.spin_limit, abort_flag, P.status};
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < DSTAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&bfull[b], 1);
-      mbar_init(&bempty[b], NUM_EPI_WARPS);
-      mbar_init(&cfull[b], 1);
-      mbar_init(&cempty[b], NUM_EPI_WARPS);
-    }
+    mbar_init(bfull, 1);
+    mbar_init(bempty, 8);
+    mbar_init(cfull, 1);
+    mbar_init(cempty, 8);
     mbar_init(done, 1);
-    mbar_init(redw, 32 * NUM_EPI_WARPS);
-    mbar_init(redm, 32 * NUM_EPI_WARPS);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -264,240 +584,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-
-  if (warp == 0) {
-    // ------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
-      uint32_t issued_mask = 0u, issued_phase = 0u;  // per stage: issued at least once / its parity
-      bool ok = true;
-      for (int slot = 0; slot <= my_tiles && ok; ++slot) {
-        const int nbv = (slot < my_tiles) ? P.nb : 0;
-        const int ncv = (slot >= 1) ? P.ncs : 0;
-        int mt = 0, vt = 0, pmt = 0, pvt = 0;
-        if (slot < my_tiles) tile_of(P, slot, &mt, &vt);
-        if (slot >= 1) tile_of(P, slot - 1, &pmt, &pvt);
-        int c = 0;
-        for (int j = 0; j < nbv + ncv && ok; ++j) {
-          // decide the next item: base stage or branch stage
-          bool is_base;
-          int jb = j - c;  // base stages emitted so far
-          if (jb >= nbv) is_base = false;
-          else if (c < ncv && jb == ins_point(c, nbv, ncv) && nbv > 0) is_base = false;
-          else is_base = true;
-          if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) { ok = false; break; }
-          unsigned char* sa = stage_base + stage * STAGE_BYTES;
-          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          if (is_base) {
-            tma_load_2d(sa, &tm_a, &full[stage], jb * BK, mt * BM);
-            tma_load_2d(sa + STAGE_A, &tm_b, &full[stage], jb * BK, vt * BN);
-          } else {
-            tma_load_2d(sa, &tm_ca, &full[stage], c * BK, pmt * BM);
-            tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, pvt * BN);
-            ++c;
-          }
-          issued_mask |= 1u << stage;
-          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
-        }
-      }
-      // copies still in flight after an abort: wait (bounded) before leaving
-      for (int s = 0; s < STAGES; ++s)
-        if (issued_mask & (1u << s)) {
-          const uint64_t t0 = globaltimer();
-          while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
-                 (globaltimer() - t0) < 2000000000ull) {
-          }
-        }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t id_base = idesc_f16(true);
-      const uint32_t id_corr = idesc_f16(false);
-      int stage = 0;
-      uint32_t phase = 0;
-      uint32_t cuse0 = 0u, cuse1 = 0u;  // uses of the two branch accumulators
-      bool ok = true;
-      for (int slot = 0; slot <= my_tiles && ok; ++slot) {
-        const int nbv = (slot < my_tiles) ? P.nb : 0;
-        const int ncv = (slot >= 1) ? P.ncs : 0;
-        const int bb = slot & 1;
-        const uint32_t bcol = tmem + (uint32_t)(bb * BN);
-        int c = 0;
-        for (int j = 0; j < nbv + ncv && ok; ++j) {
-          bool is_base;
-          const int jb = j - c;
-          if (jb >= nbv) is_base = false;
-          else if (c < ncv && jb == ins_point(c, nbv, ncv) && nbv > 0) is_base = false;
-          else is_base = true;
-          if (is_base && jb == 0) {
-            if (!mbar_wait(&bempty[bb], (((uint32_t)slot >> 1) & 1u) ^ 1u, ctl, 2)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-          }
-          if (!mbar_wait(&full[stage], phase, ctl, 3)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t sa = smem_u32(stage_base + stage * STAGE_BYTES);
-          const uint32_t sb = sa + STAGE_A;
-          if (is_base) {
-#pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-              umma(bcol, sdesc(sa + k * 32), sdesc(sb + k * 32), id_base,
-                   (jb > 0 || k > 0) ? 1u : 0u);
-            umma_commit(&empty[stage]);
-            if (jb == nbv - 1) umma_commit(&bfull[bb]);
-          } else {
-            // branch stage c of the previous tile: components z0 .. z0+zps-1
-            const int z0 = c * P.zps;
-            for (int zz = 0; zz < P.zps && z0 + zz < P.K && ok; ++zz) {
-              const int z = z0 + zz;
-              const int cs = z & 1;
-              const uint32_t use = cs ? cuse1 : cuse0;
-              if (!mbar_wait(&cempty[cs], (use & 1u) ^ 1u, ctl, 4)) { ok = false; break; }
-              tc_fence_after();
-              const uint32_t ccol = tmem + 2u * BN + (uint32_t)(cs * BN);
-              const int o = zz * 2 * P.rp;  // element offset of this component in the stage
-              int first = 1;
-              for (int kk = 0; kk < P.rp; kk += 16) {
-                const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
-                umma(ccol, sdesc(sa + hi), sdesc(sb + hi), id_corr, first ? 0u : 1u);
-                umma(ccol, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
-                umma(ccol, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
-                first = 0;
-              }
-              umma_commit(&cfull[cs]);
-              if (cs) ++cuse1; else ++cuse0;
-            }
-            umma_commit(&empty[stage]);
-            ++c;
-          }
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
-        }
-      }
-      // wait (bounded) for every MMA this thread issued before TMEM is freed
-      umma_commit(done);
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
-      }
-    }
+  if (warp >= 4) {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
+    draft_epilogue(P, tmem, warp, lane, az, bfull, bempty, cfull, cempty, ctl, my_tiles);
   } else {
-    // ------------------------------------------------------ epilogue warps
-    const int ew = warp - 2;
-    const int q = warp & 3;          // TMEM lane quarter of this warp
-    const int half = ew >> 2;        // which 64 columns of the tile
-    const int row = q * 32 + lane;   // row of the tile
-    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    uint32_t cuse0 = 0u, cuse1 = 0u;
-    for (int slot = 0; slot < my_tiles; ++slot) {
-      int mt, vt;
-      tile_of(P, slot, &mt, &vt);
-      const int bb = slot & 1;
-      if (!mbar_wait(&bfull[bb], ((uint32_t)slot >> 1) & 1u, ctl, 5)) break;
-      tc_fence_after();
-      const int m = mt * BM + row;
-      const int v0 = vt * BN + half * 64;
-      float bk[64];
-      {
-        float t[32];
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-          tmem_ld32(tmem + lane_off + (uint32_t)(bb * BN + half * 64 + cc * 32), t);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) bk[cc * 32 + j] = t[j];
-        }
-      }
-      // base accumulator is in registers: hand the TMEM buffer back
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bempty[bb]);
-
-      if (P.mode == MODE_PREP) {
-        // WU[v][row] for rows < prep_rows
-        if (m < P.prep_rows) {
-#pragma unroll
-          for (int j = 0; j < 64; ++j) {
-            const int v = v0 + j;
-            if (v < P.V) P.wu[(size_t)v * P.prep_rows + m] = bk[j];
-          }
-        }
-        continue;
-      }
-
-      // draft: b_v, stash, scale by log2(e)/T
-      const bool full_vec = (v0 + 64 <= P.V) && ((P.V & 3) == 0);
-#pragma unroll
-      for (int j = 0; j < 64; ++j) {
-        const int v = v0 + j;
-        if (P.vbias && v < P.V) bk[j] += __ldg(P.vbias + v);
-      }
-      if (m < P.M) {
-        float* srow = P.stash + (size_t)m * P.V + v0;
-        if (full_vec) {
-#pragma unroll
-          for (int j = 0; j < 64; j += 4)
-            *reinterpret_cast<float4*>(srow + j) = make_float4(bk[j], bk[j + 1], bk[j + 2], bk[j + 3]);
-        } else {
-          for (int j = 0; j < 64; ++j)
-            if (v0 + j < P.V) srow[j] = bk[j];
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < 64; ++j) bk[j] = (v0 + j < P.V) ? bk[j] * P.k2 : -INFINITY;
-
-      // the previous tile's records must be merged before they are overwritten
-      if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 7)) break;
-      bool ok = true;
-      for (int z = 0; z < P.K; ++z) {
-        const int cs = z & 1;
-        const uint32_t use = cs ? cuse1 : cuse0;
-        if (!mbar_wait(&cfull[cs], use & 1u, ctl, 6)) { ok = false; break; }
-        if (cs) ++cuse1; else ++cuse0;
-        tc_fence_after();
-        const float a = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
-        float M2 = -INFINITY, S = 0.f;
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-          float cr[32];
-          tmem_ld32(tmem + lane_off + (uint32_t)(2 * BN + cs * BN + half * 64 + cc * 32), cr);
-          float mx = -INFINITY;
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            cr[j] = fmaf(cr[j], a, bk[cc * 32 + j]);
-            mx = fmaxf(mx, cr[j]);
-          }
-          const float Mn = fmaxf(M2, mx);
-          if (Mn != -INFINITY) {
-            float acc = 0.f;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) acc += exp2f(cr[j] - Mn);
-            S = S * exp2f(M2 - Mn) + acc;
-            M2 = Mn;
-          }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&cempty[cs]);
-        red[((size_t)z * 2 + half) * BM + row] = make_float2(M2, S);
-      }
-      if (!ok) break;
-      // merge the two column halves of every (row, z) and write the records
-      mbar_arrive(redw);
-      if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 8)) break;
-      for (int z = half; z < P.K; z += 2) {
-        const float2 p0 = red[((size_t)z * 2) * BM + row];
-        const float2 p1 = red[((size_t)z * 2 + 1) * BM + row];
-        const float mz = fmaxf(p0.x, p1.x);
-        float2 out = make_float2(-INFINITY, 0.f);
-        if (mz != -INFINITY)
-          out = make_float2(mz, p0.y * exp2f(p0.x - mz) + p1.y * exp2f(p1.x - mz));
-        P.partd[((size_t)vt * P.K + z) * P.Mpad + m] = out;
-      }
-      mbar_arrive(redm);
-    }
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
+    if (warp == 0 && lane == 0)
+      draft_producer(P, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
+    else if (warp == 1 && lane == 0)
+      draft_mma(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl, my_tiles);
   }
 
   tc_fence_before();
@@ -519,11 +614,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 struct VParams {
   int n_mt, n_vt, n_tiles, ncs, K, rp, zps, M, V, Mpad, B, Bt;
   float k2;
-  const float* cscale;   // [Mpad, K]
-  const float* sw;       // [K]
-  const double* lse2;    // [M, K]
-  const double* w2;      // [M, K]
-  const double* lse2t;   // [N (B+1)]
+  const float2* vcz;     // [M, K]: (k2 / (sc_{m,z} sw_z), log2 w_{m,z} - L_{m,z} + B0_m)
+  const float* vb0;      // [M]: B0_m
+  const float2* lt2;     // [N (B+1)]: target log2-sum-exp as a float pair
   const float* stash;    // [M, V]
   const __nv_bfloat16* target;  // [N, Bt, V]
   float2* partv;         // [nt, Mpad]
@@ -619,7 +712,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t id_corr = idesc_f16(false);
+      const uint32_t id_corr = idesc_f16(false, BN);
       int stage = 0;
       uint32_t phase = 0, guse0 = 0u, guse1 = 0u;
       bool ok = true;
@@ -680,21 +773,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int v0 = vt * BN + half * 64;
       // per-row constants
       float a[KMAX], cz[KMAX];
-      double B0 = 0.0;
-      if (mok) {
-        double mx = -INFINITY;
-        for (int z = 0; z < P.K; ++z) mx = fmax(mx, P.lse2[(size_t)m * P.K + z]);
-        B0 = floor(mx);
-      }
+      const float B0f = mok ? P.vb0[m] : 0.f;
 #pragma unroll
       for (int z = 0; z < KMAX; ++z) {
         a[z] = 0.f;
         cz[z] = -INFINITY;
         if (z < P.K && mok) {
-          a[z] = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
-          const double wz = P.w2[(size_t)m * P.K + z];
-          cz[z] = (wz == -INFINITY) ? -INFINITY
-                                    : (float)(wz - P.lse2[(size_t)m * P.K + z] + B0);
+          const float2 c = P.vcz[(size_t)m * P.K + z];
+          a[z] = c.x;
+          cz[z] = c.y;
         }
       }
       float acc[64];
@@ -733,8 +820,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float As = 0.f, Rs = 0.f;
       if (mok) {
         const int n = m / P.B, i = m - n * P.B;
-        const float Lt = (float)P.lse2t[(size_t)n * (P.B + 1) + i];
-        const float B0f = (float)B0;
+        const float2 Lt = P.lt2[(size_t)n * (P.B + 1) + i];
         const float* srow = P.stash + (size_t)m * P.V + v0;
         const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
         const bool vec = (v0 + 64 <= P.V) && ((P.V & 7) == 0);
@@ -767,7 +853,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const int j = cc * 8 + u;
             if (v0 + j < P.V) {
               const float qv = exp2f(fmaf(sv[u], P.k2, -B0f)) * acc[j];
-              const float pv = exp2f(fmaf(tv[u], P.k2, -Lt));
+              const float pv = exp2f(fmaf(tv[u], P.k2, -Lt.x) - Lt.y);
               const float mn = fminf(pv, qv);
               As += mn;
               Rs += pv - mn;
@@ -818,13 +904,14 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D K-major tile map: rows x cols elements of 2 bytes, box 128 rows x 64
-static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, bool bf16) {
+// 2-D K-major tile map: rows x cols elements of 2 bytes, box box_rows x 64
+static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, bool bf16,
+                     uint32_t box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t box[2] = {BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
                   const_cast<void*>(base), dims, strides, box, estr,
@@ -844,20 +931,33 @@ static int num_sms() {
   return n;
 }
 
-static size_t smem_bytes() { return STAGES * STAGE_BYTES + RED_BYTES + 256 + 1024; }
+// The register split of k_tc_pass (setmaxnreg) assumes the kernel was built
+// with exactly DREG registers per thread: with fewer, the epilogue's increase
+// could never be granted.  Such a build is refused instead of launched.
+static cudaError_t pass_kernel_ready() {
+  static int state = -1;
+  if (state < 0) {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs != DREG) {
+      state = 0;
+    } else {
+      e = cudaFuncSetAttribute(k_tc_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)DSMEM);
+      if (e != cudaSuccess) return e;
+      state = 1;
+    }
+  }
+  return state == 1 ? cudaSuccess : cudaErrorInvalidKernelImage;
+}
 
 static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
                           const CUtensorMap& cb, const Params& P, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_tc_pass, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem_bytes());
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  cudaError_t e = pass_kernel_ready();
+  if (e != cudaSuccess) return e;
   const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
   if (grid <= 0) return cudaSuccess;
-  k_tc_pass<<<grid, NUM_THREADS, smem_bytes(), s>>>(a, b, ca, cb, P);
+  k_tc_pass<<<grid, D_THREADS, DSMEM, s>>>(a, b, ca, cb, P);
   debug_kernel("k_tc_pass", s);
   count_launches(1);
   count_tc_launch();
@@ -873,7 +973,8 @@ bool tc_supported(const dblast_head* h) {
   return tc::encode_fn() != nullptr;
 }
 
-// transposed expander [U_z | e_z]^T as bf16 [rows_pad, H] for the prep GEMM
+// transposed expander factor [F_z | e_z]^T as bf16 [rows_pad, H] (zero rows
+// past K rr, and a zero row r of every block when e is null)
 __global__ void k_prep_transpose(const __nv_bfloat16* __restrict__ U,
                                  const __nv_bfloat16* __restrict__ e, int H, int K, int r, int rr,
                                  int rows_pad, __nv_bfloat16* __restrict__ ut) {
@@ -892,27 +993,34 @@ __global__ void k_prep_transpose(const __nv_bfloat16* __restrict__ U,
   }
 }
 
-cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStream_t s) {
-  unsigned char* prep = static_cast<unsigned char*>(h->prep);
-  void* ut = prep + pl.off_ut;
-  const int rows = h->K * pl.rr;
-  const int rows_pad = ceil_div(rows, tc::BM) * tc::BM;
-  auto* utp = static_cast<__nv_bfloat16*>(ut);
-  k_prep_transpose<<<1024, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(h->U),
-                                        static_cast<const __nv_bfloat16*>(h->e), h->H, h->K, h->r,
-                                        pl.rr, rows_pad, utp);
+static void transpose_expander(const void* F, const void* e, const dblast_head* h,
+                               const PrepLayout& pl, __nv_bfloat16* out, cudaStream_t s) {
+  const int rows_pad = ceil_div(h->K * pl.rr, tc::BM) * tc::BM;
+  k_prep_transpose<<<1024, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(F),
+                                        static_cast<const __nv_bfloat16*>(e), h->H, h->K, h->r,
+                                        pl.rr, rows_pad, out);
   debug_kernel("k_prep_transpose", s);
   count_launches(1);
+}
+
+cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStream_t s) {
+  unsigned char* prep = static_cast<unsigned char*>(h->prep);
+  const int rows = h->K * pl.rr;
+  const int rows_pad = ceil_div(rows, tc::BM) * tc::BM;
+  auto* utp = reinterpret_cast<__nv_bfloat16*>(prep + pl.off_ut);
+  transpose_expander(h->U, h->e, h, pl, utp, s);
+  // V_z^T (with a zero row for the constant code of e) for the per-call codes GEMM
+  transpose_expander(h->Vf, nullptr, h, pl, reinterpret_cast<__nv_bfloat16*>(prep + pl.off_vt), s);
   CUtensorMap ma, mb;
-  if (!tc::make_map(&ma, utp, h->H, rows_pad, true) || !tc::make_map(&mb, h->W, h->H, h->V, true))
+  if (!tc::make_map(&ma, utp, h->H, rows_pad, true, tc::BM) ||
+      !tc::make_map(&mb, h->W, h->H, h->V, true, tc::DBN))
     return cudaErrorInvalidValue;
   tc::Params P{};
   P.mode = tc::MODE_PREP;
   P.n_mt = rows_pad / tc::BM;
-  P.n_vt = ceil_div(h->V, tc::BN);
+  P.n_vt = ceil_div(h->V, tc::DBN);
   P.n_tiles = P.n_mt * P.n_vt;
   P.nb = h->H / tc::BK;
-  P.ncs = 0;
   P.K = h->K;
   P.rp = pl.rp;
   P.zps = 1;
@@ -921,9 +1029,47 @@ cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStrea
   P.Mpad = rows_pad;
   P.wu = reinterpret_cast<float*>(prep + pl.off_wu);
   P.prep_rows = rows;
+  P.split_stride = 0;
   P.status = reinterpret_cast<DevStatus*>(prep + pl.off_status);
   P.spin_limit = wait_limit();
   return tc::launch(ma, mb, ma, mb, P, s);
+}
+
+// codes c_{m,z} = V_z^T h_m for every position: the prep machinery with
+// A = V^T [K rr, H], B = hidden [M, H], split-K partials [ksplit][M][K rr]
+cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit) {
+  const dblast_head* h = c.head;
+  const WsLayout& w = c.wl;
+  const int rows = h->K * w.rr;
+  const int rows_pad = ceil_div(rows, tc::BM) * tc::BM;
+  CUtensorMap ma, mb;
+  if (!tc::make_map(&ma, c.prep + c.pl.off_vt, h->H, rows_pad, true, tc::BM) ||
+      !tc::make_map(&mb, c.args->hidden, h->H, w.M, true, tc::DBN))
+    return cudaErrorInvalidValue;
+  const int nb64 = h->H / tc::BK;
+  const int base_tiles = (rows_pad / tc::BM) * ceil_div(w.M, tc::DBN);
+  int ks = 1;
+  for (int d = 1; d <= 16 && d <= nb64; ++d)
+    if (nb64 % d == 0 && base_tiles * d <= tc::num_sms()) ks = d;
+  tc::Params P{};
+  P.mode = tc::MODE_PREP;
+  P.n_mt = rows_pad / tc::BM;
+  P.n_vt = ceil_div(w.M, tc::DBN);
+  P.n_tiles = P.n_mt * P.n_vt * ks;
+  P.nb = nb64 / ks;
+  P.K = h->K;
+  P.rp = w.rp;
+  P.zps = 1;
+  P.M = rows;
+  P.V = w.M;
+  P.Mpad = rows_pad;
+  P.wu = part;
+  P.prep_rows = rows;
+  P.split_stride = (size_t)w.M * rows;
+  P.status = wsp<DevStatus>(c, w.off_status);
+  P.spin_limit = wait_limit();
+  *nsplit = ks;
+  return tc::launch(ma, mb, ma, mb, P, c.stream);
 }
 
 cudaError_t launch_draft_pass_tc(const StepCtx& c) {
@@ -931,18 +1077,17 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   const WsLayout& w = c.wl;
   CUtensorMap ma, mb, mca, mcb;
   const unsigned char* prep = c.prep;
-  if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true) ||
-      !tc::make_map(&mb, h->W, h->H, h->V, true) ||
-      !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false) ||
-      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false))
+  if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true, tc::BM) ||
+      !tc::make_map(&mb, h->W, h->H, h->V, true, tc::DBN) ||
+      !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM) ||
+      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, tc::DBN))
     return cudaErrorInvalidValue;
   tc::Params P{};
   P.mode = tc::MODE_DRAFT;
   P.n_mt = w.Mpad / tc::BM;
-  P.n_vt = ceil_div(h->V, tc::BN);
+  P.n_vt = ceil_div(h->V, tc::DBN);
   P.n_tiles = P.n_mt * P.n_vt;
   P.nb = h->H / tc::BK;
-  P.ncs = ceil_div(w.KC, tc::BK);
   P.K = h->K;
   P.rp = w.rp;
   P.zps = tc::BK / (2 * w.rp);
@@ -964,8 +1109,8 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   const dblast_head* h = c.head;
   const WsLayout& w = c.wl;
   CUtensorMap mca, mcb;
-  if (!tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false) ||
-      !tc::make_map(&mcb, c.prep + c.pl.off_wuop, w.KC, h->V, false))
+  if (!tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM) ||
+      !tc::make_map(&mcb, c.prep + c.pl.off_wuop, w.KC, h->V, false, tc::BN))
     return cudaErrorInvalidValue;
   tc::VParams P{};
   P.n_mt = w.Mpad / tc::BM;
@@ -981,11 +1126,9 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   P.B = w.B;
   P.Bt = c.Bt;
   P.k2 = c.k2;
-  P.cscale = wsp<float>(c, w.off_cscale);
-  P.sw = prp<float>(c, c.pl.off_sw);
-  P.lse2 = wsp<double>(c, w.off_lse2);
-  P.w2 = wsp<double>(c, w.off_w2);
-  P.lse2t = wsp<double>(c, w.off_lse2t);
+  P.vcz = wsp<float2>(c, w.off_vcz);
+  P.vb0 = wsp<float>(c, w.off_vb0);
+  P.lt2 = wsp<float2>(c, w.off_lt2);
   P.stash = wsp<float>(c, w.off_stash);
   P.target = static_cast<const __nv_bfloat16*>(c.target);
   P.partv = wsp<float2>(c, w.off_partv);
