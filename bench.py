@@ -190,11 +190,13 @@ def main():
     ap.add_argument("--kernels", default="auto", choices=["auto", "simt", "tcgen05"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--n-seqs", type=int, default=None,
+                    help="override the number of sequences N (smaller cases for profiler captures)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
     import synth
-    cfg = synth.config(args.config)
+    cfg = synth.config(args.config, **({"N": args.n_seqs} if args.n_seqs else {}))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))

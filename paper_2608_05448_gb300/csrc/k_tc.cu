@@ -35,7 +35,6 @@ constexpr int KMAX = 16;           // components supported by the tensor-core pa
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int NUM_THREADS = 32 * (2 + NUM_EPI_WARPS);
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int RED_BYTES = KMAX * 2 * BM * 8;   // [z][half][row] (max, sum)
 
 enum Mode { MODE_PREP = 0, MODE_DRAFT = 1 };
 
@@ -190,7 +189,8 @@ constexpr int DREG = 168, DREG_LO = 56, DREG_HI = 224;
 static_assert(4 * DREG_LO + 8 * DREG_HI == 12 * DREG, "register split must equal the launch pool");
 constexpr int D_EPI = 256;                   // epilogue threads
 constexpr int DAZ_BYTES = KMAX * D_EPI * 4;  // per-thread branch scales
-constexpr size_t DSMEM = (size_t)DSTAGES * DSTAGE + DAZ_BYTES + 256 + 1024;
+constexpr int DVB_BYTES = 2 * DBN * 4;       // vocabulary bias of two tiles
+constexpr size_t DSMEM = (size_t)DSTAGES * DSTAGE + DAZ_BYTES + DVB_BYTES + 256 + 1024;
 
 struct Params {
   int mode;
@@ -368,14 +368,11 @@ __device__ __forceinline__ void tmem_ld16_raw(uint32_t taddr, uint32_t (&r)[16])
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
-// Volatile on purpose: the math on one TMEM chunk must stay ahead of the
-// next chunk's tcgen05.ld, or the compiler keeps every chunk live at once.
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ void pin(float& x) { asm volatile("" : "+f"(x)); }
 
 // Epilogue: per tile, the base accumulator plus b_v becomes the stash; then
 // for every component z the record (ref, sum 2^{t_v}) of this thread's 128
@@ -383,7 +380,8 @@ __device__ __forceinline__ void pin(float& x) { asm volatile("" : "+f"(x)); }
 // (base_v + b_v) taken once per tile.  A sum outside [2^-100, 2^100] (a branch
 // offset far from the base logits) is redone against the exact maximum.
 __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, int warp, int lane,
-                                            float* az, uint64_t* bfull, uint64_t* bempty,
+                                            float* az, float* vbs, uint64_t* vbar,
+                                            uint64_t* bfull, uint64_t* bempty,
                                             uint64_t* cfull, uint64_t* cempty, const Ctl& ctl,
                                             int my_tiles) {
   const int ew = warp - 4;
@@ -399,23 +397,17 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     const int m = mt * BM + row;
     const int v0 = vt * DBN + half * DCOLS;
     float bk[DCOLS];
+    // this tile's vocabulary bias, staged in shared memory (double-buffered by
+    // slot parity: every thread arrives on vbar of slot s+1 only after its
+    // reads of slot s, so the writes of slot s+2 cannot overtake them), and the
+    // branch scales, while the main loop still runs
+    const float* vb = vbs + (slot & 1) * DBN + half * DCOLS;
     if (P.mode == MODE_DRAFT) {
-      // branch scales and vocabulary bias while the main loop still runs
       for (int z = 0; z < P.K; ++z) az[z * D_EPI + et] = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
-      if (P.vbias && v0 + DCOLS <= P.V) {
-        const float4* vb = reinterpret_cast<const float4*>(P.vbias + v0);
-#pragma unroll
-        for (int j = 0; j < DCOLS / 4; ++j) {
-          const float4 t = __ldg(vb + j);
-          bk[4 * j] = t.x;
-          bk[4 * j + 1] = t.y;
-          bk[4 * j + 2] = t.z;
-          bk[4 * j + 3] = t.w;
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < DCOLS; ++j) bk[j] = (P.vbias && v0 + j < P.V) ? __ldg(P.vbias + v0 + j) : 0.f;
-      }
+      const int vc = vt * DBN + et;
+      vbs[(slot & 1) * DBN + et] = (P.vbias && vc < P.V) ? __ldg(P.vbias + vc) : 0.f;
+      mbar_arrive(vbar);
+      if (!mbar_wait(vbar, (uint32_t)slot & 1u, ctl, 7)) break;
     }
     if (!mbar_wait(bfull, (uint32_t)slot & 1u, ctl, 5)) break;
     tc_fence_after();
@@ -425,11 +417,9 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       tmem_ld16_raw(tmem + lane_off + (uint32_t)(half * DCOLS + cc * 16), r);
       tmem_wait_ld();
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        bk[cc * 16 + j] = (P.mode == MODE_DRAFT) ? bk[cc * 16 + j] + __uint_as_float(r[j])
+      for (int j = 0; j < 16; ++j)
+        bk[cc * 16 + j] = (P.mode == MODE_DRAFT) ? __uint_as_float(r[j]) + vb[cc * 16 + j]
                                                  : __uint_as_float(r[j]);
-        pin(bk[cc * 16 + j]);
-      }
     }
     // the base accumulator is in registers: hand TMEM back to the MMA thread
     tc_fence_before();
@@ -507,7 +497,6 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
           tmem_wait_ld();
 #pragma unroll
           for (int j = 0; j < 16; ++j) mx = fmaxf(mx, fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]));
-          pin(mx);
         }
         float s = 0.f;
 #pragma unroll
@@ -542,7 +531,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stages = smem;
   float* az = reinterpret_cast<float*>(smem + DSTAGES * DSTAGE);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DSTAGES * DSTAGE + DAZ_BYTES);
+  float* vbs = reinterpret_cast<float*>(smem + DSTAGES * DSTAGE + DAZ_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DSTAGES * DSTAGE + DAZ_BYTES + DVB_BYTES);
   uint64_t* full = bars;                 // [DSTAGES]
   uint64_t* empty = bars + DSTAGES;      // [DSTAGES]
   uint64_t* bfull = bars + 2 * DSTAGES;  // base accumulator ready
@@ -550,7 +540,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   uint64_t* cfull = bfull + 2;           // branch accumulator ready
   uint64_t* cempty = bfull + 3;          // branch accumulator taken (8 epilogue warps)
   uint64_t* done = bfull + 4;            // every MMA of this CTA finished
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 5);
+  uint64_t* vbar = bfull + 5;            // a tile's vocabulary bias staged (256 epilogue threads)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 6);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -569,6 +560,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
     mbar_init(cfull, 1);
     mbar_init(cempty, 8);
     mbar_init(done, 1);
+    mbar_init(vbar, D_EPI);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -586,7 +578,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
 
   if (warp >= 4) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
-    draft_epilogue(P, tmem, warp, lane, az, bfull, bempty, cfull, cempty, ctl, my_tiles);
+    draft_epilogue(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl, my_tiles);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
     if (warp == 0 && lane == 0)
