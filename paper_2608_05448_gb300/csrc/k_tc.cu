@@ -16,6 +16,9 @@
 // WU = [U_z | e_z]^T . W^T and stores it as fp32 [V, K, rr].
 #include <cuda.h>
 
+#include <algorithm>
+#include <cstdlib>
+
 #include "dblast_internal.cuh"
 
 namespace dblast {
@@ -107,6 +110,38 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// the same copy written to the same shared-memory offset of every CTA in
+// cta_mask (this GPU's own memory only); each destination's mbarrier at the
+// same offset receives the complete_tx bytes
+__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                               int x, int y, uint16_t cta_mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster "
+      "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(cta_mask)
+      : "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_count_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -147,6 +182,15 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
+      : "memory");
+}
+
+// arrive on the mbarrier at this offset in every CTA of cta_mask once the
+// MMAs issued so far have completed
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+      "[%0], %1;" ::"r"(smem_u32(bar)), "h"(cta_mask)
       : "memory");
 }
 
@@ -194,7 +238,8 @@ constexpr size_t DSMEM = (size_t)DSTAGES * DSTAGE + DAZ_BYTES + DVB_BYTES + 256 
 
 struct Params {
   int mode;
-  int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles, tiles (x ksplit in prep mode)
+  int cs;                    // CTAs per cluster: M tiles sharing one vocabulary tile (1, 2 or 4)
+  int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles, cluster tiles (x ksplit in prep mode)
   int nb;                    // base stages per tile
   int K, rp, zps;            // components, padded rank, components per 64-wide block
   int M, V, Mpad;            // valid rows, vocabulary (B-operand rows), padded rows
@@ -211,31 +256,57 @@ struct Params {
   uint32_t spin_limit;
 };
 
-// tile `slot` of this CTA: split (prep mode), M tile, vocabulary tile; the
-// order is vocabulary-major so concurrent CTAs share the B tile through L2
-__device__ __forceinline__ void tile_of(const Params& P, int slot, int* sp, int* mt, int* vt) {
-  const int t = (int)blockIdx.x + slot * (int)gridDim.x;
-  const int per = P.n_mt * P.n_vt;
+// Tile `slot` of this CTA.  The CTAs of one cluster (cs of them) share a
+// vocabulary tile and take consecutive M tiles; cluster tiles are numbered
+// split-major (prep mode), then vocabulary-major, so concurrently running
+// clusters also share B tiles through L2.
+struct Sched {
+  int cid, ncl, rank;  // cluster index, cluster count, rank in the cluster
+};
+__device__ __forceinline__ Sched sched_of(const Params& P) {
+  if (P.cs == 1) return Sched{(int)blockIdx.x, (int)gridDim.x, 0};
+  return Sched{(int)cluster_id_x(), (int)cluster_count_x(), (int)cluster_ctarank()};
+}
+__device__ __forceinline__ void tile_of(const Params& P, const Sched& S, int slot, int* sp,
+                                        int* mt, int* vt) {
+  const int t = S.cid + slot * S.ncl;
+  const int ng = P.n_mt / P.cs;
+  const int per = ng * P.n_vt;
   *sp = t / per;
   const int r = t - *sp * per;
-  *vt = r / P.n_mt;
-  *mt = r - *vt * P.n_mt;
+  *vt = r / ng;
+  *mt = (r - *vt * ng) * P.cs + S.rank;
 }
 
 // The item sequence of slot s (consumed by the MMA thread, produced by the TMA
 // thread): the base stages of tile s, with the branch items (one per
 // component) of tile s-1 inserted before base stage ins_point(z).  The last
-// slot (s == my_tiles) holds only the branch items of the last tile.
-__device__ __forceinline__ int ins_point(int z, int nb, int nz) { return ((z + 1) * nb) / (nz + 2); }
-__device__ __forceinline__ bool is_branch(int jb, int zd, int nbv, int nzv) {
-  return zd < nzv && (jb >= nbv || jb == ins_point(zd, nbv, nzv));
+// slot (s == my_tiles) holds only the branch items of the last tile.  The
+// first branch item waits until 3/8 of the base stages have been issued (the
+// epilogue is still taking the base accumulator and writing the stash), the
+// others follow evenly up to two stages before the end, about one
+// component's epilogue apart.
+__device__ __forceinline__ int ins_point(int z, int nb, int nz) {
+  const int first = (3 * nb) / 8;
+  const int last = nb - 2 > first ? nb - 2 : first;
+  return nz > 1 ? first + (z * (last - first)) / (nz - 1) : first;
 }
 
-__device__ __noinline__ void draft_producer(const Params& P, const CUtensorMap* tm_a,
-                                            const CUtensorMap* tm_b, const CUtensorMap* tm_ca,
-                                            const CUtensorMap* tm_cb, unsigned char* stages,
-                                            uint64_t* full, uint64_t* empty, const Ctl& ctl,
-                                            int my_tiles) {
+// The producer and the MMA issuer are single threads whose instruction chain
+// sits on the critical path of every stage (a stage is 512 tensor cycles), so
+// their loops avoid divisions and descriptor rebuilds: insertion points are
+// advanced once per branch item, coordinates and descriptors by constants.
+__device__ __noinline__ void draft_producer(const Params& P, const Sched& S,
+                                            const CUtensorMap* tm_a, const CUtensorMap* tm_b,
+                                            const CUtensorMap* tm_ca, const CUtensorMap* tm_cb,
+                                            unsigned char* stages, uint64_t* full, uint64_t* empty,
+                                            const Ctl& ctl, int my_tiles) {
+  // with cs > 1 every CTA loads its own A tile and a 1/cs slice of the shared
+  // B tile, multicast to the whole cluster (the B maps then have DBN/cs rows)
+  const int bq = DBN / P.cs;
+  const bool mc = P.cs > 1;
+  const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
+  const uint32_t boff = (uint32_t)(S.rank * bq * BK * 2);
   int stage = 0;
   uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
   bool ok = true;
@@ -244,27 +315,35 @@ __device__ __noinline__ void draft_producer(const Params& P, const CUtensorMap* 
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
     int sp = 0, mt = 0, vt = 0, psp = 0, pmt = 0, pvt = 0;
-    if (slot < my_tiles) tile_of(P, slot, &sp, &mt, &vt);
-    if (slot >= 1) tile_of(P, slot - 1, &psp, &pmt, &pvt);
-    int zd = 0;
-    for (int j = 0; j < nbv + nzv; ++j) {
-      const int jb = j - zd;
-      const bool br = is_branch(jb, zd, nbv, nzv);
+    if (slot < my_tiles) tile_of(P, S, slot, &sp, &mt, &vt);
+    if (slot >= 1) tile_of(P, S, slot - 1, &psp, &pmt, &pvt);
+    const int ya = mt * BM, yb = vt * DBN + S.rank * bq;
+    const int yca = pmt * BM, ycb = pvt * DBN + S.rank * bq;
+    int kx = sp * P.nb * BK;
+    int jb = 0, zd = 0;
+    int ins = nzv > 0 ? ins_point(0, nbv, nzv) : 0x7fffffff;
+    while (jb < nbv || zd < nzv) {
+      const bool br = zd < nzv && (jb >= nbv || jb == ins);
       if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) {
         ok = false;
         break;
       }
       unsigned char* sa = stages + stage * DSTAGE;
-      mbar_arrive_expect_tx(&full[stage], DSTAGE);
+      uint64_t* fb = &full[stage];
+      mbar_arrive_expect_tx(fb, DSTAGE);
       if (!br) {
-        const int kx = (sp * P.nb + jb) * BK;
-        tma_load_2d(sa, tm_a, &full[stage], kx, mt * BM);
-        tma_load_2d(sa + DSTAGE_A, tm_b, &full[stage], kx, vt * DBN);
+        tma_load_2d(sa, tm_a, fb, kx, ya);
+        if (!mc) tma_load_2d(sa + DSTAGE_A, tm_b, fb, kx, yb);
+        else tma_load_2d_mc(sa + DSTAGE_A + boff, tm_b, fb, kx, yb, mask);
+        kx += BK;
+        ++jb;
       } else {
-        const int kx = (zd / P.zps) * BK;
-        tma_load_2d(sa, tm_ca, &full[stage], kx, pmt * BM);
-        tma_load_2d(sa + DSTAGE_A, tm_cb, &full[stage], kx, pvt * DBN);
+        const int kc = (P.zps == 2 ? (zd >> 1) : zd) * BK;
+        tma_load_2d(sa, tm_ca, fb, kc, yca);
+        if (!mc) tma_load_2d(sa + DSTAGE_A, tm_cb, fb, kc, ycb);
+        else tma_load_2d_mc(sa + DSTAGE_A + boff, tm_cb, fb, kc, ycb, mask);
         ++zd;
+        ins = zd < nzv ? ins_point(zd, nbv, nzv) : 0x7fffffff;
       }
       issued_mask |= 1u << stage;
       issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -290,6 +369,12 @@ __device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned 
                                        uint64_t* done, const Ctl& ctl, int my_tiles) {
   const uint32_t id_base = idesc_f16(true, DBN);
   const uint32_t id_corr = idesc_f16(false, DBN);
+  const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
+  const bool mc = P.cs > 1;
+  // shared-memory descriptors: the start-address field holds addr >> 4, so a
+  // byte offset off inside the 1024-aligned stages moves it by off >> 4
+  const uint64_t d0 = sdesc(smem_u32(stages));
+  const uint32_t dcol = tmem + (uint32_t)DBN;
   int stage = 0;
   uint32_t phase = 0, cuse = 0;
   bool ok = true;
@@ -297,10 +382,10 @@ __device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned 
   for (int slot = 0; slot <= my_tiles && ok; ++slot) {
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
-    int zd = 0;
-    for (int j = 0; j < nbv + nzv; ++j) {
-      const int jb = j - zd;
-      const bool br = is_branch(jb, zd, nbv, nzv);
+    int jb = 0, zd = 0;
+    int ins = nzv > 0 ? ins_point(0, nbv, nzv) : 0x7fffffff;
+    while (jb < nbv || zd < nzv) {
+      const bool br = zd < nzv && (jb >= nbv || jb == ins);
       if (!br && jb == 0) {  // the epilogue has taken the previous base accumulator
         if (!mbar_wait(bempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 2)) {
           ok = false;
@@ -320,28 +405,33 @@ __device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned 
         break;
       }
       tc_fence_after();
-      const uint32_t sa = smem_u32(stages + stage * DSTAGE);
-      const uint32_t sb = sa + DSTAGE_A;
+      const uint64_t da = d0 + (uint64_t)(stage * (DSTAGE >> 4));
+      const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
       if (!br) {
-#pragma unroll
-        for (int k = 0; k < BK / 16; ++k)
-          umma(tmem, sdesc(sa + k * 32), sdesc(sb + k * 32), id_base, (jb > 0 || k > 0) ? 1u : 0u);
-        umma_commit(&empty[stage]);
+        umma(tmem, da, db, id_base, jb > 0 ? 1u : 0u);
+        umma(tmem, da + 2, db + 2, id_base, 1u);
+        umma(tmem, da + 4, db + 4, id_base, 1u);
+        umma(tmem, da + 6, db + 6, id_base, 1u);
+        if (!mc) umma_commit(&empty[stage]);
+        else umma_commit_mc(&empty[stage], mask);
         if (jb == nbv - 1) umma_commit(bfull);
+        ++jb;
       } else {
-        // component zd of the previous tile: hi.hi + hi.lo + lo.hi
-        const uint32_t dcol = tmem + (uint32_t)DBN;
-        const int o = (zd % P.zps) * 2 * P.rp;
+        // component zd of the previous tile: hi.hi + hi.lo + lo.hi; element
+        // offsets o (hi) and o + rp (lo) are multiples of 16 (32 bytes)
+        const int o = (P.zps == 2 ? (zd & 1) : 0) * 2 * P.rp;
         for (int kk = 0; kk < P.rp; kk += 16) {
-          const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
-          umma(dcol, sdesc(sa + hi), sdesc(sb + hi), id_corr, kk > 0 ? 1u : 0u);
-          umma(dcol, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
-          umma(dcol, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
+          const uint64_t hi = (uint64_t)((o + kk) >> 3), lo = (uint64_t)((o + P.rp + kk) >> 3);
+          umma(dcol, da + hi, db + hi, id_corr, kk > 0 ? 1u : 0u);
+          umma(dcol, da + hi, db + lo, id_corr, 1u);
+          umma(dcol, da + lo, db + hi, id_corr, 1u);
         }
         umma_commit(cfull);
-        umma_commit(&empty[stage]);
+        if (!mc) umma_commit(&empty[stage]);
+        else umma_commit_mc(&empty[stage], mask);
         ++cuse;
         ++zd;
+        ins = zd < nzv ? ins_point(zd, nbv, nzv) : 0x7fffffff;
       }
       if (++stage == DSTAGES) {
         stage = 0;
@@ -391,9 +481,10 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
   const int et = ew * 32 + lane;
   const uint32_t lane_off = (uint32_t)(q * 32) << 16;
   uint32_t cuse = 0;
+  const Sched S = sched_of(P);
   for (int slot = 0; slot < my_tiles; ++slot) {
     int sp, mt, vt;
-    tile_of(P, slot, &sp, &mt, &vt);
+    tile_of(P, S, slot, &sp, &mt, &vt);
     const int m = mt * BM + row;
     const int v0 = vt * DBN + half * DCOLS;
     float bk[DCOLS];
@@ -438,10 +529,17 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       continue;
     }
 
-    // stash W h + b
+    // stash W h + b (32-byte stores: each fills one sector of this thread's row)
     if (m < P.M) {
       float* srow = P.stash + (size_t)m * P.V + v0;
-      if (v0 + DCOLS <= P.V && (P.V & 3) == 0) {
+      if (v0 + DCOLS <= P.V && (P.V & 7) == 0) {
+#pragma unroll
+        for (int j = 0; j < DCOLS; j += 8)
+          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(srow + j),
+                       "f"(bk[j]), "f"(bk[j + 1]), "f"(bk[j + 2]), "f"(bk[j + 3]), "f"(bk[j + 4]),
+                       "f"(bk[j + 5]), "f"(bk[j + 6]), "f"(bk[j + 7])
+                       : "memory");
+      } else if (v0 + DCOLS <= P.V && (P.V & 3) == 0) {
 #pragma unroll
         for (int j = 0; j < DCOLS; j += 4)
           *reinterpret_cast<float4*>(srow + j) = make_float4(bk[j], bk[j + 1], bk[j + 2], bk[j + 3]);
@@ -545,15 +643,14 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int my_tiles = (P.n_tiles > (int)blockIdx.x)
-                           ? (P.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
-                           : 0;
+  const Sched S = sched_of(P);
+  const int my_tiles = (P.n_tiles > S.cid) ? (P.n_tiles - 1 - S.cid) / S.ncl + 1 : 0;
   const Ctl ctl{P.spin_limit, abort_flag, P.status};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < DSTAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], P.cs);  // one MMA commit from every CTA of the cluster
     }
     mbar_init(bfull, 1);
     mbar_init(bempty, 8);
@@ -574,6 +671,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // every CTA's barriers exist before any multicast copy or commit reaches them
+  if (P.cs > 1) cluster_sync_all();
   const uint32_t tmem = *tmem_slot;
 
   if (warp >= 4) {
@@ -582,7 +681,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
     if (warp == 0 && lane == 0)
-      draft_producer(P, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
+      draft_producer(P, S, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
     else if (warp == 1 && lane == 0)
       draft_mma(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl, my_tiles);
   }
@@ -594,6 +693,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(TMEM_COLS));
   }
+  // no CTA leaves while a peer may still multicast into it or arrive on it
+  if (P.cs > 1) cluster_sync_all();
 }
 
 // ------------------------------------------------------------ verify pass
@@ -943,17 +1044,71 @@ static cudaError_t pass_kernel_ready() {
   return state == 1 ? cudaSuccess : cudaErrorInvalidKernelImage;
 }
 
+// clusters of cs CTAs that can be resident at once (cached per size)
+static int max_clusters(int cs) {
+  static int cache[5] = {0, 0, 0, 0, 0};
+  if (cs < 1 || cs > 4) return 0;
+  if (!cache[cs]) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cs * num_sms());
+    cfg.blockDim = dim3(D_THREADS);
+    cfg.dynamicSmemBytes = DSMEM;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = cs;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass, &cfg) != cudaSuccess || n < 1) n = 1;
+    cache[cs] = n;
+  }
+  return cache[cs];
+}
+
 static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
                           const CUtensorMap& cb, const Params& P, cudaStream_t s) {
   cudaError_t e = pass_kernel_ready();
   if (e != cudaSuccess) return e;
-  const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
-  if (grid <= 0) return cudaSuccess;
-  k_tc_pass<<<grid, D_THREADS, DSMEM, s>>>(a, b, ca, cb, P);
+  if (P.n_tiles <= 0) return cudaSuccess;
+  if (P.cs == 1) {
+    const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
+    k_tc_pass<<<grid, D_THREADS, DSMEM, s>>>(a, b, ca, cb, P);
+  } else {
+    const int ncl = std::min(P.n_tiles, max_clusters(P.cs));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(ncl * P.cs);
+    cfg.blockDim = dim3(D_THREADS);
+    cfg.dynamicSmemBytes = DSMEM;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = P.cs;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, k_tc_pass, a, b, ca, cb, P);
+    if (e != cudaSuccess) return e;
+  }
   debug_kernel("k_tc_pass", s);
   count_launches(1);
   count_tc_launch();
   return cudaGetLastError();
+}
+
+// CTAs per cluster of the draft pass: the M tiles that share a vocabulary
+// tile.  One by default: multicasting the shared B tile halves L2 reads but
+// not the shared-memory traffic per SM, and the lockstep it imposes measured
+// slower on this GPU.  DBLAST_DRAFT_CLUSTER=2|4 selects the multicast
+// schedule (tests cover every size).
+static int draft_cluster_size(int n_mt) {
+  int cs = 1;
+  const char* env = getenv("DBLAST_DRAFT_CLUSTER");
+  if (env && (env[0] == '1' || env[0] == '2' || env[0] == '4') && env[1] == 0) cs = env[0] - '0';
+  while (cs > 1 && (n_mt % cs) != 0) cs >>= 1;
+  return cs;
 }
 
 }  // namespace tc
@@ -1009,6 +1164,7 @@ cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStrea
     return cudaErrorInvalidValue;
   tc::Params P{};
   P.mode = tc::MODE_PREP;
+  P.cs = 1;
   P.n_mt = rows_pad / tc::BM;
   P.n_vt = ceil_div(h->V, tc::DBN);
   P.n_tiles = P.n_mt * P.n_vt;
@@ -1045,6 +1201,7 @@ cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit) {
     if (nb64 % d == 0 && base_tiles * d <= tc::num_sms()) ks = d;
   tc::Params P{};
   P.mode = tc::MODE_PREP;
+  P.cs = 1;
   P.n_mt = rows_pad / tc::BM;
   P.n_vt = ceil_div(w.M, tc::DBN);
   P.n_tiles = P.n_mt * P.n_vt * ks;
@@ -1067,18 +1224,22 @@ cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit) {
 cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   const dblast_head* h = c.head;
   const WsLayout& w = c.wl;
+  const int n_mt = w.Mpad / tc::BM;
+  const int cs = tc::draft_cluster_size(n_mt);
+  const uint32_t bq = tc::DBN / cs;  // B rows each CTA of a cluster loads
   CUtensorMap ma, mb, mca, mcb;
   const unsigned char* prep = c.prep;
   if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true, tc::BM) ||
-      !tc::make_map(&mb, h->W, h->H, h->V, true, tc::DBN) ||
+      !tc::make_map(&mb, h->W, h->H, h->V, true, bq) ||
       !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM) ||
-      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, tc::DBN))
+      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, bq))
     return cudaErrorInvalidValue;
   tc::Params P{};
   P.mode = tc::MODE_DRAFT;
-  P.n_mt = w.Mpad / tc::BM;
+  P.cs = cs;
+  P.n_mt = n_mt;
   P.n_vt = ceil_div(h->V, tc::DBN);
-  P.n_tiles = P.n_mt * P.n_vt;
+  P.n_tiles = (P.n_mt / cs) * P.n_vt;
   P.nb = h->H / tc::BK;
   P.K = h->K;
   P.rp = w.rp;
