@@ -15,6 +15,7 @@ sequences are independent units; there is no data-path collective) and rank
 bounded sample (one sequence per step) on the host cores.
 """
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -309,12 +310,16 @@ def main():
         achieved = wm["flop_draft_pass"] / (draft_ms * 1e-3) / 1e12
         t_roof = max(wm["flop"] / (peaks["bf16"] * 1e12), wm["bytes"] / (peaks["hbm"] * 1e9))
         traffic = None
-        tr_path = os.path.join(ROOT, "profiles", "draft_pass_traffic.json")
-        if os.path.exists(tr_path):
+        # DRAM bytes per draft-pass launch from the committed ncu summary, used
+        # only while the kernel source is the one that was profiled
+        tr_path = os.path.join(ROOT, "profiles", "draft_pass_%s_traffic.json" % cfg["name"])
+        if os.path.exists(tr_path) and st["tc_launches"] > 0 and not args.n_seqs:
             d = json.load(open(tr_path))
-            if d.get("kernel_impl") == ("tcgen05" if st["tc_launches"] > 0 else "simt") and \
-                    d.get("workload") == cfg["name"]:
-                traffic = d.get("bytes_per_launch")
+            src = os.path.join(ROOT, d.get("source", ""))
+            if os.path.exists(src):
+                hsh = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+                if hsh == d.get("source_sha256_16"):
+                    traffic = d.get("bytes_per_launch")
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": K_steps, "warmup": args.warmup, "ms_per_step": ms_step,
