@@ -110,6 +110,15 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
 // the same copy written to the same shared-memory offset of every CTA in
 // cta_mask (this GPU's own memory only); each destination's mbarrier at the
 // same offset receives the complete_tx bytes
@@ -704,8 +713,16 @@ __global__ void __launch_bounds__(D_THREADS, 1)
 //   p(v)      = 2^{t_v log2(e)/T - Lt_m},
 // and the tile records (sum min(p, q), sum [p - q]_+).  bk = stash log2(e)/T;
 // B0 = floor(max_z L_{m,z}) keeps both factors inside the fp32 range.
+// The stash and target tiles of a verify tile go through shared memory when
+// use_x (V % 8 == 0 and 128 % B == 0): the producer loads them by TMA while
+// the epilogue is still busy with the tile's branch exponentials.
+constexpr int VSTAGES = 3;
+constexpr int XS_BYTES = BM * BN * 4;   // stash tile: 4 boxes [128 rows][32 fp32], SW128
+constexpr int XT_BYTES = BM * BN * 2;   // target tile: 2 boxes [128 rows][64 bf16], SW128
+constexpr size_t VSMEM = (size_t)VSTAGES * STAGE_BYTES + XS_BYTES + XT_BYTES + 2 * BM * 8 + 256 + 1024;
 struct VParams {
   int n_mt, n_vt, n_tiles, ncs, K, rp, zps, M, V, Mpad, B, Bt;
+  int use_x;
   float k2;
   const float2* vcz;     // [M, K]: (k2 / (sc_{m,z} sw_z), log2 w_{m,z} - L_{m,z} + B0_m)
   const float* vb0;      // [M]: B0_m
@@ -725,21 +742,26 @@ __device__ __forceinline__ void vtile_of(const VParams& P, int slot, int* mt, in
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     k_tc_verify(const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
+                const __grid_constant__ CUtensorMap tm_xs, const __grid_constant__ CUtensorMap tm_xt,
                 const VParams P) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stage_base = smem;
-  float2* red = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES);   // [2][BM]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + 2 * BM * 8);
+  unsigned char* xs = smem + VSTAGES * STAGE_BYTES;  // stash tile
+  unsigned char* xt = xs + XS_BYTES;                 // target tile
+  float2* red = reinterpret_cast<float2*>(xt + XT_BYTES);   // [2][BM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xt + XT_BYTES + 2 * BM * 8);
   uint64_t* full = bars;
-  uint64_t* empty = bars + STAGES;
-  uint64_t* sfull = bars + 2 * STAGES;   // [2] TMEM slot ready
+  uint64_t* empty = bars + VSTAGES;
+  uint64_t* sfull = bars + 2 * VSTAGES;  // [2] TMEM slot ready
   uint64_t* sempty = sfull + 2;          // [2] TMEM slot free
   uint64_t* done = sfull + 4;
   uint64_t* redw = sfull + 5;
   uint64_t* redm = sfull + 6;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 7);
+  uint64_t* xfull = sfull + 7;           // stash and target tile landed
+  uint64_t* xempty = sfull + 8;          // stash and target tile read (8 epilogue warps)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -750,7 +772,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   Ctl ctl{P.spin_limit, abort_flag, P.status};
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < VSTAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -761,6 +783,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(done, 1);
     mbar_init(redw, 32 * NUM_EPI_WARPS);
     mbar_init(redm, 32 * NUM_EPI_WARPS);
+    mbar_init(xfull, 1);
+    mbar_init(xempty, NUM_EPI_WARPS);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -781,6 +805,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
       bool ok = true;
+      bool x_issued = false;
+      uint32_t x_phase = 0;
       for (int slot = 0; slot < my_tiles && ok; ++slot) {
         int mt, vt;
         vtile_of(P, slot, &mt, &vt);
@@ -792,16 +818,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, vt * BN);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+          if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (ok && P.use_x) {
+          // this tile's stash rows and target rows, once the epilogue has read the previous ones
+          if (!mbar_wait(xempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) { ok = false; break; }
+          mbar_arrive_expect_tx(xfull, XS_BYTES + XT_BYTES);
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            tma_load_2d(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM);
+          const int n0 = (mt * BM) / P.B;
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            tma_load_3d(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0);
+          x_issued = true;
+          x_phase = (uint32_t)slot & 1u;
         }
       }
-      for (int s = 0; s < STAGES; ++s)
+      for (int s = 0; s < VSTAGES; ++s)
         if (issued_mask & (1u << s)) {
           const uint64_t t0 = globaltimer();
           while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
                  (globaltimer() - t0) < 2000000000ull) {
           }
         }
+      if (x_issued) {
+        const uint64_t t0 = globaltimer();
+        while (!mbar_try_wait(xfull, x_phase) && (globaltimer() - t0) < 2000000000ull) {
+        }
+      }
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -838,7 +883,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               }
             }
             umma_commit(&empty[stage]);
-            if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+            if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
             ++c;
           }
           if (!ok) break;
@@ -911,48 +956,55 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (!ok) break;
       float As = 0.f, Rs = 0.f;
-      if (mok) {
-        const int n = m / P.B, i = m - n * P.B;
-        const float2 Lt = P.lt2[(size_t)n * (P.B + 1) + i];
-        const float* srow = P.stash + (size_t)m * P.V + v0;
-        const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
-        const bool vec = (v0 + 64 <= P.V) && ((P.V & 7) == 0);
+      const int n = m / P.B, i = m - n * P.B;
+      const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
+      auto accumulate = [&](int j, float sv, float tv) {
+        const float qv = exp2f(fmaf(sv, P.k2, -B0f)) * acc[j];
+        const float pv = exp2f(fmaf(tv, P.k2, -Lt.x) - Lt.y);
+        const float mn = fminf(pv, qv);
+        As += mn;
+        Rs += pv - mn;
+      };
+      if (P.use_x) {
+        // stash and target rows from shared memory (128-byte swizzle: the
+        // 16-byte chunk c of row r sits at chunk c ^ (r & 7))
+        if (!mbar_wait(xfull, (uint32_t)slot & 1u, ctl, 18)) break;
+        if (mok) {
+          const unsigned char* sbase = xs + half * 2 * (XS_BYTES / 4) + row * 128;
+          const unsigned char* tbase = xt + half * (XT_BYTES / 2) + row * 128;
 #pragma unroll
-        for (int cc = 0; cc < 8; ++cc) {
-          float sv[8], tv[8];
-          if (vec) {
-            const float4 s0 = *reinterpret_cast<const float4*>(srow + cc * 8);
-            const float4 s1 = *reinterpret_cast<const float4*>(srow + cc * 8 + 4);
-            sv[0] = s0.x; sv[1] = s0.y; sv[2] = s0.z; sv[3] = s0.w;
-            sv[4] = s1.x; sv[5] = s1.y; sv[6] = s1.z; sv[7] = s1.w;
-            const uint4 t8 = *reinterpret_cast<const uint4*>(trow + cc * 8);
+          for (int cc = 0; cc < 8; ++cc) {
+            const int sb = cc >> 2;                  // stash box (32 columns)
+            const int c0 = ((cc & 3) * 2) ^ (row & 7), c1 = ((cc & 3) * 2 + 1) ^ (row & 7);
+            const float4 s0 = *reinterpret_cast<const float4*>(sbase + sb * (XS_BYTES / 4) + c0 * 16);
+            const float4 s1 = *reinterpret_cast<const float4*>(sbase + sb * (XS_BYTES / 4) + c1 * 16);
+            const uint4 t8 = *reinterpret_cast<const uint4*>(tbase + ((cc ^ (row & 7)) * 16));
             const __nv_bfloat162* tp = reinterpret_cast<const __nv_bfloat162*>(&t8);
+            const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+            float tv[8];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
               const float2 f = __bfloat1622float2(tp[u]);
               tv[2 * u] = f.x;
               tv[2 * u + 1] = f.y;
             }
-          } else {
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              const int v = v0 + cc * 8 + u;
-              sv[u] = (v < P.V) ? srow[cc * 8 + u] : 0.f;
-              tv[u] = (v < P.V) ? __bfloat162float(trow[cc * 8 + u]) : 0.f;
-            }
-          }
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const int j = cc * 8 + u;
-            if (v0 + j < P.V) {
-              const float qv = exp2f(fmaf(sv[u], P.k2, -B0f)) * acc[j];
-              const float pv = exp2f(fmaf(tv[u], P.k2, -Lt.x) - Lt.y);
-              const float mn = fminf(pv, qv);
-              As += mn;
-              Rs += pv - mn;
-            }
+            for (int u = 0; u < 8; ++u)
+              if (v0 + cc * 8 + u < P.V) accumulate(cc * 8 + u, sv[u], tv[u]);
           }
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(xempty);
+      } else if (mok) {
+        const float* srow = P.stash + (size_t)m * P.V + v0;
+        const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int v = v0 + cc * 8 + u;
+            if (v < P.V) accumulate(cc * 8 + u, srow[cc * 8 + u], __bfloat162float(trow[cc * 8 + u]));
+          }
       }
       // the other column half of this row, then one record per (tile, row)
       if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 15)) break;
@@ -1008,6 +1060,27 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t r
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
                   const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// general tiled map: rank 2 or 3, dims/strides in elements (strides in bytes
+// are derived), box in elements, 128-byte swizzle
+static bool make_map_nd(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int esize,
+                        int rank, const uint64_t* dims, const uint32_t* box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t d[3], st[2];
+  cuuint32_t bx[3], es[3] = {1, 1, 1};
+  uint64_t stride = (uint64_t)esize;
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    if (i > 0) st[i - 1] = stride;
+    stride *= dims[i];
+  }
+  CUresult r = fn(m, dt, (cuuint32_t)rank, const_cast<void*>(base), d, st, bx, es,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -1261,10 +1334,25 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
 cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   const dblast_head* h = c.head;
   const WsLayout& w = c.wl;
-  CUtensorMap mca, mcb;
+  CUtensorMap mca, mcb, mxs, mxt;
   if (!tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM) ||
       !tc::make_map(&mcb, c.prep + c.pl.off_wuop, w.KC, h->V, false, tc::BN))
     return cudaErrorInvalidValue;
+  // stash and target tiles through shared memory: 16-byte row strides and
+  // whole sequences per 128-row tile
+  const bool use_x = (h->V % 8) == 0 && (tc::BM % w.B) == 0 &&
+                     (reinterpret_cast<uintptr_t>(c.target) & 15u) == 0;
+  mxs = mca;
+  mxt = mca;
+  if (use_x) {
+    const uint64_t ds[2] = {(uint64_t)h->V, (uint64_t)w.M};
+    const uint32_t bs[2] = {32, (uint32_t)tc::BM};
+    const uint64_t dt[3] = {(uint64_t)h->V, (uint64_t)c.Bt, (uint64_t)w.N};
+    const uint32_t bt[3] = {64, (uint32_t)w.B, (uint32_t)(tc::BM / w.B)};
+    if (!tc::make_map_nd(&mxs, c.ws + w.off_stash, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 2, ds, bs) ||
+        !tc::make_map_nd(&mxt, c.target, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 3, dt, bt))
+      return cudaErrorInvalidValue;
+  }
   tc::VParams P{};
   P.n_mt = w.Mpad / tc::BM;
   P.n_vt = ceil_div(h->V, tc::BN);
@@ -1278,6 +1366,7 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   P.Mpad = w.Mpad;
   P.B = w.B;
   P.Bt = c.Bt;
+  P.use_x = use_x ? 1 : 0;
   P.k2 = c.k2;
   P.vcz = wsp<float2>(c, w.off_vcz);
   P.vb0 = wsp<float>(c, w.off_vb0);
@@ -1288,15 +1377,15 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
   static bool attr = false;
-  const size_t smem = tc::STAGES * tc::STAGE_BYTES + 2 * tc::BM * 8 + 256 + 1024;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(tc::k_tc_verify,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)tc::VSMEM);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   const int grid = P.n_tiles < tc::num_sms() ? P.n_tiles : tc::num_sms();
-  tc::k_tc_verify<<<grid, tc::NUM_THREADS, smem, c.stream>>>(mca, mcb, P);
+  tc::k_tc_verify<<<grid, tc::NUM_THREADS, tc::VSMEM, c.stream>>>(mca, mcb, mxs, mxt, P);
   debug_kernel("k_tc_verify", c.stream);
   count_launches(1);
   count_tc_launch();
