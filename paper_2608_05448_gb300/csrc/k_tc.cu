@@ -455,6 +455,19 @@ __device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned 
   }
 }
 
+__device__ __forceinline__ void tmem_ld32_raw(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_ld16_raw(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
@@ -909,19 +922,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int m = mt * BM + row;
       const bool mok = m < P.M;
       const int v0 = vt * BN + half * 64;
-      // per-row constants
-      float a[KMAX], cz[KMAX];
+      // per-row constants: B0 here, (k2 / scale, log2 w - L + B0) per component below
       const float B0f = mok ? P.vb0[m] : 0.f;
-#pragma unroll
-      for (int z = 0; z < KMAX; ++z) {
-        a[z] = 0.f;
-        cz[z] = -INFINITY;
-        if (z < P.K && mok) {
-          const float2 c = P.vcz[(size_t)m * P.K + z];
-          a[z] = c.x;
-          cz[z] = c.y;
-        }
-      }
+      const float2* vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
       float acc[64];
 #pragma unroll
       for (int j = 0; j < 64; ++j) acc[j] = 0.f;
@@ -932,22 +935,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!mbar_wait(&sfull[gs], use & 1u, ctl, 14)) { ok = false; break; }
         if (gs) ++guse1; else ++guse0;
         tc_fence_after();
-#pragma unroll
         for (int zz = 0; zz < 2; ++zz) {
           const int z = 2 * g + zz;
-          if (z < P.K) {
-            float az = 0.f, cc_z = -INFINITY;
+          if (z >= P.K) break;
+          const float2 cz = mok ? vrow[z] : make_float2(0.f, -INFINITY);
+          // both 32-column chunks of this component, one wait
+          uint32_t r0[32], r1[32];
+          const uint32_t col = tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + half * 64);
+          tmem_ld32_raw(col, r0);
+          tmem_ld32_raw(col + 32, r1);
+          tmem_wait_ld();
 #pragma unroll
-            for (int k = 0; k < KMAX; ++k)
-              if (k == z) { az = a[k]; cc_z = cz[k]; }
-#pragma unroll
-            for (int cc = 0; cc < 2; ++cc) {
-              float cr[32];
-              tmem_ld32(tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + half * 64 + cc * 32),
-                        cr);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) acc[cc * 32 + j] += exp2f(fmaf(cr[j], az, cc_z));
-            }
+          for (int j = 0; j < 32; ++j) {
+            acc[j] += ex2(fmaf(__uint_as_float(r0[j]), cz.x, cz.y));
+            acc[32 + j] += ex2(fmaf(__uint_as_float(r1[j]), cz.x, cz.y));
           }
         }
         tc_fence_before();
@@ -959,8 +960,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int n = m / P.B, i = m - n * P.B;
       const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
       auto accumulate = [&](int j, float sv, float tv) {
-        const float qv = exp2f(fmaf(sv, P.k2, -B0f)) * acc[j];
-        const float pv = exp2f(fmaf(tv, P.k2, -Lt.x) - Lt.y);
+        const float qv = ex2(fmaf(sv, P.k2, -B0f)) * acc[j];
+        const float pv = ex2(fmaf(tv, P.k2, -Lt.x) - Lt.y);
         const float mn = fminf(pv, qv);
         As += mn;
         Rs += pv - mn;
