@@ -240,7 +240,8 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   g_calls.fetch_add(1, std::memory_order_relaxed);
   cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t),
                                   c.stream);
-  if (e == cudaSuccess) e = dbg(launch_prior_codes(c), "prior_codes", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
     e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
@@ -251,18 +252,91 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   return cuda_status(e);
 }
 
+static cudaError_t verify_passes(const StepCtx& c, dblast_verify_out* out) {
+  pass_event_begin(1, c.stream);
+  cudaError_t e = c.tc ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
+  pass_event_end(1, c.stream);
+  e = dbg(e, "verify_pass", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_verify_finalize(c, out), "verify_finalize", c.stream);
+  return e;
+}
+
 static dblast_status verify_impl(StepCtx c, dblast_verify_out* out) {
   c.target = out->target;
   c.Bt = c.args->B + (out->has_bonus ? 1 : 0);
   g_calls.fetch_add(1, std::memory_order_relaxed);
   cudaError_t e = dbg(launch_target_stats(c, out), "target_stats", c.stream);
-  if (e == cudaSuccess) {
-    pass_event_begin(1, c.stream);
-    e = c.tc ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
-    pass_event_end(1, c.stream);
-    e = dbg(e, "verify_pass", c.stream);
+  if (e == cudaSuccess) e = verify_passes(c, out);
+  return cuda_status(e);
+}
+
+// One internal stream and four events per device for the fork/join of
+// kernels that do not depend on each other inside dblast_draft_and_verify
+// (no device memory; created by the first such call on the device and held
+// until the process exits).  The mutex keeps one call's fork/join pairs
+// together when several host threads call in.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+};
+static std::mutex g_side_mu;
+static SideStream g_side[64];
+
+static cudaError_t side_stream(SideStream** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  SideStream& ss = g_side[dev];
+  if (!ss.s) {
+    e = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking);
+    for (int i = 0; i < 4 && e == cudaSuccess; ++i)
+      e = cudaEventCreateWithFlags(&ss.ev[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) return e;
   }
-  if (e == cudaSuccess) e = dbg(launch_verify_finalize(c, out), "verify_finalize", c.stream);
+  *out = &ss;
+  return cudaSuccess;
+}
+
+// draft and verify of one block with two forks: the category prior runs
+// beside the codes GEMM, and the target statistics beside the draft
+// finalize kernels (both pairs are independent and latency-bound).
+static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_out* vout) {
+  if (debug_sync()) {  // serial order, so a failing launcher is named
+    dblast_status st = draft_impl(c, dout);
+    return st != DBLAST_OK ? st : verify_impl(c, vout);
+  }
+  c.target = vout->target;
+  c.Bt = c.args->B + (vout->has_bonus ? 1 : 0);
+  g_calls.fetch_add(2, std::memory_order_relaxed);
+  std::lock_guard<std::mutex> lk(g_side_mu);
+  SideStream* ss = nullptr;
+  cudaError_t e = side_stream(&ss);
+  StepCtx side = c;
+  if (e == cudaSuccess) side.stream = ss->s;
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t), c.stream);
+  // fork 1: prior | codes
+  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[0], c.stream);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[0], 0);
+  if (e == cudaSuccess) e = launch_prior(side);
+  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[1], side.stream);
+  if (e == cudaSuccess) e = launch_codes(c);
+  if (e == cudaSuccess) {
+    pass_event_begin(0, c.stream);
+    e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
+    pass_event_end(0, c.stream);
+  }
+  // join 1, fork 2: target statistics | draft finalize
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[1], 0);
+  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[2], c.stream);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[2], 0);
+  if (e == cudaSuccess) e = launch_target_stats(side, vout);
+  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
+  if (e == cudaSuccess) e = launch_draft_finalize(c, dout);
+  // join 2
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[3], 0);
+  if (e == cudaSuccess) e = verify_passes(c, vout);
   return cuda_status(e);
 }
 
@@ -301,9 +375,7 @@ dblast_status dblast_draft_and_verify(const dblast_head* h, const dblast_block_a
   StepCtx c;
   st = make_ctx(h, a, ws, ws_bytes, vout->has_bonus ? 1 : 0, stream, &c);
   if (st != DBLAST_OK) return st;
-  st = draft_impl(c, dout);
-  if (st != DBLAST_OK) return st;
-  return verify_impl(c, vout);
+  return step_impl(c, dout, vout);
 }
 
 dblast_status dblast_device_status(void* ws, dblast_stream_t stream) {

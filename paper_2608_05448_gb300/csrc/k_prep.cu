@@ -288,7 +288,7 @@ __global__ void k_codes_finish(const float* __restrict__ part, int nsplit, int M
   }
 }
 
-template <typename Tin> static cudaError_t prior_codes_typed(const StepCtx& c) {
+template <typename Tin> static cudaError_t prior_typed(const StepCtx& c) {
   const dblast_head* h = c.head;
   const dblast_block_args* a = c.args;
   const WsLayout& w = c.wl;
@@ -299,6 +299,15 @@ template <typename Tin> static cudaError_t prior_codes_typed(const StepCtx& c) {
       a->round, wsp<int32_t>(c, w.off_zhat), wsp<float>(c, w.off_log2pi),
       wsp<uint32_t>(c, w.off_ties));
   debug_kernel("k_prior", s);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
+  const dblast_head* h = c.head;
+  const dblast_block_args* a = c.args;
+  const WsLayout& w = c.wl;
+  cudaStream_t s = c.stream;
   // codes: split-K partials go to the stash region (not yet written by this call)
   const int Nb = h->K * w.rr;
   float* part = wsp<float>(c, w.off_stash);
@@ -323,13 +332,16 @@ template <typename Tin> static cudaError_t prior_codes_typed(const StepCtx& c) {
       part, nsplit, w.M, w.Mpad, h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes),
       wsp<float>(c, w.off_cscale), wsp<__half>(c, w.off_cop));
   debug_kernel("k_codes_finish", s);
-  count_launches(2);
+  count_launches(1);
   return cudaGetLastError();
 }
 
-cudaError_t launch_prior_codes(const StepCtx& c) {
-  return c.head->dtype == DBLAST_F32 ? prior_codes_typed<float>(c)
-                                     : prior_codes_typed<__nv_bfloat16>(c);
+cudaError_t launch_prior(const StepCtx& c) {
+  return c.head->dtype == DBLAST_F32 ? prior_typed<float>(c) : prior_typed<__nv_bfloat16>(c);
+}
+
+cudaError_t launch_codes(const StepCtx& c) {
+  return c.head->dtype == DBLAST_F32 ? codes_typed<float>(c) : codes_typed<__nv_bfloat16>(c);
 }
 
 }  // namespace dblast
