@@ -956,16 +956,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (lane == 0) mbar_arrive(&sempty[gs]);
       }
       if (!ok) break;
-      float As = 0.f, Rs = 0.f;
+      // four partial sums per quantity keep the add chains short
+      float As4[4] = {0.f, 0.f, 0.f, 0.f}, Rs4[4] = {0.f, 0.f, 0.f, 0.f};
       const int n = m / P.B, i = m - n * P.B;
       const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
+      const float nB0 = -B0f;
       auto accumulate = [&](int j, float sv, float tv) {
-        const float qv = ex2(fmaf(sv, P.k2, -B0f)) * acc[j];
+        const float qv = ex2(fmaf(sv, P.k2, nB0)) * acc[j];
         const float pv = ex2(fmaf(tv, P.k2, -Lt.x) - Lt.y);
         const float mn = fminf(pv, qv);
-        As += mn;
-        Rs += pv - mn;
+        As4[j & 3] += mn;
+        Rs4[j & 3] += pv - mn;
       };
+      const bool full_cols = v0 + 64 <= P.V;
       if (P.use_x) {
         // stash and target rows from shared memory (128-byte swizzle: the
         // 16-byte chunk c of row r sits at chunk c ^ (r & 7))
@@ -989,9 +992,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               tv[2 * u] = f.x;
               tv[2 * u + 1] = f.y;
             }
+            if (full_cols) {
 #pragma unroll
-            for (int u = 0; u < 8; ++u)
-              if (v0 + cc * 8 + u < P.V) accumulate(cc * 8 + u, sv[u], tv[u]);
+              for (int u = 0; u < 8; ++u) accumulate(cc * 8 + u, sv[u], tv[u]);
+            } else {
+#pragma unroll
+              for (int u = 0; u < 8; ++u)
+                if (v0 + cc * 8 + u < P.V) accumulate(cc * 8 + u, sv[u], tv[u]);
+            }
           }
         }
         __syncwarp();
@@ -1007,6 +1015,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (v < P.V) accumulate(cc * 8 + u, srow[cc * 8 + u], __bfloat162float(trow[cc * 8 + u]));
           }
       }
+      const float As = (As4[0] + As4[1]) + (As4[2] + As4[3]);
+      const float Rs = (Rs4[0] + Rs4[1]) + (Rs4[2] + Rs4[3]);
       // the other column half of this row, then one record per (tile, row)
       if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 15)) break;
       red[half * BM + row] = make_float2(As, Rs);
