@@ -180,6 +180,104 @@ def run_reference(args, cfg, rank):
     print(json.dumps(line), flush=True)
 
 
+def _timed_steps(step, steps, warmup):
+    """CUDA-event time (ms) of `steps` calls of step(k) after `warmup` calls."""
+    import torch
+    for k in range(warmup):
+        step(k)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for k in range(steps):
+        step(warmup + k)
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def run_sweep(args):
+    """Entropy sweep (K=16, r=32, N=64): per (T, sigma) cell the mean accepted
+    length and throughput, next to the K=1 independent-block baseline with the
+    same shapes.  One JSON line per cell."""
+    import torch
+    import synth
+    from paper_2608_05448_gb300 import (Head, Workspace, alloc_draft_out, alloc_verify_out,
+                                        dblast_draft_and_verify)
+    dev = torch.device("cuda", 0)
+    for K in (16, 1):
+        for sigma in (0.3, 1.0):
+            cfg = synth.config("sweep_k16", K=K, sigma=sigma)
+            head_t = synth.make_head(cfg, dev)
+            blk = synth.make_block(cfg, head_t, 0, dev)
+            head = Head.from_dict(head_t)
+            ws = Workspace(head, cfg["N"], cfg["B"], True)
+            dout = alloc_draft_out(cfg["N"], cfg["B"], K, dev)
+            vouts = [alloc_verify_out(cfg["N"], cfg["B"], True, dev)
+                     for _ in range(args.warmup + args.steps)]
+            for T in (0.7, 1.0, 1.5):
+                pos, rnd = synth.initial_state(cfg, dev)
+
+                def step(k):
+                    dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, T, 1.0, 77 + k,
+                                            blk["target"], True, dout=dout, vout=vouts[k])
+                ms = _timed_steps(step, args.steps, args.warmup)
+                mean_L = float(torch.stack([v["accepted"].float().mean()
+                                            for v in vouts[args.warmup:]]).mean())
+                print(json.dumps({"sweep": {"K": K, "r": cfg["r"], "N": cfg["N"], "B": cfg["B"],
+                                            "T": T, "sigma": sigma, "mean_accepted_length": mean_L,
+                                            "blocks_per_s": cfg["N"] * args.steps / (ms / 1e3),
+                                            "accepted_tokens_per_s":
+                                                mean_L * cfg["N"] * args.steps / (ms / 1e3),
+                                            "ms_per_step": ms / args.steps,
+                                            "data": "synthetic"}}), flush=True)
+            del head, ws, blk, head_t
+
+
+def run_serve(args):
+    """Serving steps (N=256, B=8 and 32): four rounds with fresh hidden states
+    and targets per round and per-sequence state (positions, round counters,
+    hence Philox counters) carried on the device.  One JSON line per round."""
+    import torch
+    import synth
+    from paper_2608_05448_gb300 import (Head, Workspace, alloc_draft_out, alloc_verify_out,
+                                        dblast_draft_and_verify)
+    dev = torch.device("cuda", 0)
+    for name in ("serve_b8", "serve_b32"):
+        cfg = synth.config(name)
+        head_t = synth.make_head(cfg, dev)
+        head = Head.from_dict(head_t)
+        ws = Workspace(head, cfg["N"], cfg["B"], True)
+        dout = alloc_draft_out(cfg["N"], cfg["B"], cfg["K"], dev)
+        vout = alloc_verify_out(cfg["N"], cfg["B"], True, dev)
+        pos, rnd = synth.initial_state(cfg, dev)
+        for rd in range(4):
+            blk = synth.make_block(cfg, head_t, rd, dev)
+            # the timed call is the round itself; warm-up calls run on copies of the state
+            p_w, r_w = pos.clone(), rnd.clone()
+            for _ in range(args.warmup):
+                dblast_draft_and_verify(head, ws, blk["hidden"], p_w, r_w, 1.0, 1.0, 5,
+                                        blk["target"], True, dout=dout, vout=vout)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, 1.0, 1.0, 5,
+                                    blk["target"], True, dout=dout, vout=vout)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            L = vout["accepted"].float()
+            print(json.dumps({"serve": {"workload": name, "round": rd, "N": cfg["N"],
+                                        "B": cfg["B"], "ms": ms,
+                                        "blocks_per_s": cfg["N"] / (ms / 1e3),
+                                        "mean_accepted_length": float(L.mean()),
+                                        "min_accepted": int(L.min()), "max_accepted": int(L.max()),
+                                        "emitted_tokens": int(vout["n_emitted"].sum()),
+                                        "mean_position": float(pos.double().mean()),
+                                        "data": "synthetic"}}), flush=True)
+            del blk
+        del head, ws, head_t
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -191,6 +289,10 @@ def main():
     ap.add_argument("--kernels", default="auto", choices=["auto", "simt", "tcgen05"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--sweep", action="store_true",
+                    help="entropy-sweep report (K=16 vs K=1 cells), one JSON line per cell")
+    ap.add_argument("--serve", action="store_true",
+                    help="serving report (N=256, B=8/32, four rounds), one JSON line per round")
     ap.add_argument("--n-seqs", type=int, default=None,
                     help="override the number of sequences N (smaller cases for profiler captures)")
     args = ap.parse_args()
@@ -204,6 +306,14 @@ def main():
 
     if args.impl == "reference":
         run_reference(args, cfg, rank)
+        return
+    if args.sweep or args.serve:
+        import torch
+        torch.cuda.set_device(0)
+        if args.sweep:
+            run_sweep(args)
+        if args.serve:
+            run_serve(args)
         return
 
     import torch

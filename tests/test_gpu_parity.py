@@ -139,3 +139,41 @@ def test_qwen3_8b_batched_sampled(impl, T):
     cfg = synth.config("qwen3_8b_b32")
     _skip_unsupported(cfg, impl)
     _case(cfg, T, 1.0, seed=0, impl=impl, seqs=[0, 31])
+
+
+@pytest.mark.parametrize("T,sigma", [(0.7, 0.3), (1.5, 1.0)])
+def test_entropy_sweep_k16_r32_sampled(T, sigma):
+    """Entropy-sweep shapes at full size (N=64, K=16, r=32, V=151936), two cells."""
+    cfg = synth.config("sweep_k16", sigma=sigma)
+    _case(cfg, T, 1.0, seed=4, impl="tcgen05", seqs=[0, 63])
+
+
+def test_entropy_sweep_k1_baseline_sampled():
+    """The K=1 independent-block baseline of the sweep (same shapes, one component)."""
+    cfg = synth.config("sweep_k16", K=1)
+    _case(cfg, 1.0, 1.0, seed=5, impl="tcgen05", seqs=[7])
+
+
+@pytest.mark.parametrize("B", [8, 32])
+def test_serving_batch_four_rounds_sampled(B):
+    """Serving step at full size (N=256, B=8 or 32): state carried over four
+    rounds, each round with fresh hidden states and targets; sampled sequences
+    checked against the oracle every round."""
+    from paper_2608_05448_gb300 import Head, Workspace
+    cfg = synth.config("serve_b8" if B == 8 else "serve_b32")
+    head_t = synth.make_head(cfg, "cuda")
+    head = Head.from_dict(head_t)
+    ws = Workspace(head, cfg["N"], cfg["B"], True)
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    seqs = [3, 255]
+    rounds = 4 if B == 8 else 2
+    for rd in range(rounds):
+        blk = synth.make_block(cfg, head_t, rd, "cuda")
+        pos0, rnd0 = pos.clone(), rnd.clone()
+        gpu = parity.run_gpu(head_t, blk, 1.0, 1.0, 21, pos, rnd, head=head, ws=ws)
+        orc = parity.run_oracle(head_t, blk, 1.0, 1.0, 21, pos0, rnd0, seqs)
+        parity.compare(gpu, orc, seqs)
+        assert torch.equal(pos.cpu(), pos0.cpu() + gpu["n_emitted"].long())
+        assert torch.equal(rnd.cpu(), rnd0.cpu() + 1)
+        del blk, gpu
+    assert int(rnd[0]) == rounds
