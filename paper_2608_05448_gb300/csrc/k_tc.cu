@@ -30,7 +30,6 @@ namespace tc {
 constexpr int BM = 128;            // rows per tile (TMEM lanes)
 constexpr int BN = 128;            // vocabulary tokens per tile (TMEM columns)
 constexpr int BK = 64;             // elements per stage row (128 bytes, SW128 atom)
-constexpr int STAGES = 5;
 constexpr int STAGE_A = BM * BK * 2;   // 16 KB
 constexpr int STAGE_B = BN * BK * 2;   // 16 KB
 constexpr int STAGE_BYTES = STAGE_A + STAGE_B;
@@ -172,10 +171,10 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
 }
 
 // instruction descriptor, kind::f16: fp32 accumulate, A/B both bf16 or both
-// fp16, both K-major, M = 128, N = n
-__host__ __device__ constexpr uint32_t idesc_f16(bool bf16, int n) {
+// fp16, both K-major, M = m (128, or 256 for a CTA pair), N = n
+__host__ __device__ constexpr uint32_t idesc_f16(bool bf16, int n, int m = BM) {
   return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) |
-         (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
+         (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(m >> 4) << 24);
 }
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -200,6 +199,74 @@ __device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t cta_mask)
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
       "[%0], %1;" ::"r"(smem_u32(bar)), "h"(cta_mask)
+      : "memory");
+}
+
+// ---- CTA pairs (cta_group::2): one MMA spans the tensor cores of two SMs.
+// The A operand and the accumulator are split by rows (128 per SM), the B
+// operand by N (half of the tile in each SM's shared memory, at the same
+// offset); the even CTA of the pair issues every MMA.
+
+// the shared::cluster address of the object at p's offset in CTA `rank`
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t caddr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr)
+               : "memory");
+}
+// a wait whose arrivals may come from the other CTA of the pair
+__device__ __forceinline__ bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity, const Ctl& c,
+                                             uint32_t where) {
+  if (mbar_try_wait_cl(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait_cl(bar, parity)) return true;
+    if (*c.abort) return false;
+    if ((c.spin_limit && i >= c.spin_limit) || (globaltimer() - t0) > 2000000000ull) {
+      record_timeout(c, where);
+      return false;
+    }
+  }
+}
+// a copy into this CTA's shared memory whose complete_tx goes to the mbarrier
+// at cluster address bar_cl (the even CTA's)
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cl, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cl), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// arrive on the mbarrier at bar's offset in both CTAs of the pair once the
+// pair MMAs issued so far have completed
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+      "[%0], %1;" ::"r"(smem_u32(bar)), "h"((uint16_t)3)
       : "memory");
 }
 
@@ -231,11 +298,16 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
 // 1 issues MMAs and owns TMEM, warps 4-11 are the epilogue (two per TMEM lane
 // quarter, 128 columns each).  Warpgroup 0 gives registers to the epilogue
 // warpgroups with setmaxnreg (56 + 2 x 224 = 3 x 168 per thread).
+//
+// The pair form (PAIR = true) runs the same roles on a cluster of two CTAs
+// with cta_group::2 MMAs of 256 x 256: each SM stages its own 128 rows of A
+// and 128 of the 256 B rows (32 KB a stage instead of 48), so six stages fit
+// and the L2 reads of the head per tile fall by a third.  Both CTAs' copies
+// complete on the even CTA's full barriers, its MMA commits arrive on both
+// CTAs' barriers, and both epilogues hand the accumulators back on the even
+// CTA's bempty / cempty.
 constexpr int DBN = 256;                     // vocabulary tokens per tile
-constexpr int DSTAGES = 4;
 constexpr int DSTAGE_A = BM * BK * 2;        // 16 KB
-constexpr int DSTAGE_B = DBN * BK * 2;       // 32 KB
-constexpr int DSTAGE = DSTAGE_A + DSTAGE_B;  // 48 KB
 constexpr int DCOLS = DBN / 2;               // columns per epilogue thread
 constexpr int D_THREADS = 384;
 constexpr int DREG = 168, DREG_LO = 56, DREG_HI = 224;
@@ -243,7 +315,16 @@ static_assert(4 * DREG_LO + 8 * DREG_HI == 12 * DREG, "register split must equal
 constexpr int D_EPI = 256;                   // epilogue threads
 constexpr int DAZ_BYTES = KMAX * D_EPI * 4;  // per-thread branch scales
 constexpr int DVB_BYTES = 2 * DBN * 4;       // vocabulary bias of two tiles
-constexpr size_t DSMEM = (size_t)DSTAGES * DSTAGE + DAZ_BYTES + DVB_BYTES + 256 + 1024;
+template <bool PAIR>
+struct DCfg {
+  static constexpr int STAGES = PAIR ? 6 : 4;
+  static constexpr int BROWS = PAIR ? DBN / 2 : DBN;       // B rows staged by one CTA
+  static constexpr int STAGE_B = BROWS * BK * 2;           // 16 or 32 KB
+  static constexpr int STAGE = DSTAGE_A + STAGE_B;         // 32 or 48 KB
+  static constexpr int TX = PAIR ? 2 * STAGE : STAGE;      // bytes completing one full barrier
+  static constexpr size_t SMEM = (size_t)STAGES * STAGE + DAZ_BYTES + DVB_BYTES + 256 + 1024;
+};
+static_assert(DCfg<true>::SMEM <= 227 * 1024 && DCfg<false>::SMEM <= 227 * 1024, "shared memory");
 
 struct Params {
   int mode;
@@ -291,35 +372,68 @@ __device__ __forceinline__ void tile_of(const Params& P, const Sched& S, int slo
 // thread): the base stages of tile s, with the branch items (one per
 // component) of tile s-1 inserted before base stage ins_point(z).  The last
 // slot (s == my_tiles) holds only the branch items of the last tile.  The
-// first branch item waits until 3/8 of the base stages have been issued (the
-// epilogue is still taking the base accumulator and writing the stash), the
-// others follow evenly up to two stages before the end, about one
-// component's epilogue apart.
+// first branch item comes after 1/8 of the base stages (the epilogue is
+// still taking the base accumulator and writing the stash), the others
+// follow evenly up to six stages before the end, so that the last
+// component's epilogue ends before the tile's base accumulator is complete
+// (measured best among first in {0, 1/8, 1/4, 3/8} x last in nb - {2..12}).
 __device__ __forceinline__ int ins_point(int z, int nb, int nz) {
-  const int first = (3 * nb) / 8;
-  const int last = nb - 2 > first ? nb - 2 : first;
+  const int first = nb / 8;
+  const int last = nb - 6 > first ? nb - 6 : first;
   return nz > 1 ? first + (z * (last - first)) / (nz - 1) : first;
 }
 
-// The producer and the MMA issuer are single threads whose instruction chain
-// sits on the critical path of every stage (a stage is 512 tensor cycles), so
-// their loops avoid divisions and descriptor rebuilds: insertion points are
-// advanced once per branch item, coordinates and descriptors by constants.
-__device__ __noinline__ void draft_producer(const Params& P, const Sched& S,
-                                            const CUtensorMap* tm_a, const CUtensorMap* tm_b,
-                                            const CUtensorMap* tm_ca, const CUtensorMap* tm_cb,
-                                            unsigned char* stages, uint64_t* full, uint64_t* empty,
-                                            const Ctl& ctl, int my_tiles) {
-  // with cs > 1 every CTA loads its own A tile and a 1/cs slice of the shared
-  // B tile, multicast to the whole cluster (the B maps then have DBN/cs rows)
+// The producer and the MMA issuer are single threads whose dependent
+// instruction chains sit on the critical path of every stage (a stage is 512
+// tensor cycles, a thread's chain runs at several cycles per instruction), so
+// both are inlined (parameters read from the constant bank, no local copies)
+// and run the base stages between two branch items in a loop that only
+// waits, issues and advances the stage; measured alone, such a loop keeps
+// the tensor pipe busy at 128 cycles per 128 x 256 x 16 MMA.
+template <bool PAIR>
+__device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
+                                               const CUtensorMap* tm_a, const CUtensorMap* tm_b,
+                                               const CUtensorMap* tm_ca, const CUtensorMap* tm_cb,
+                                               unsigned char* stages, uint64_t* full,
+                                               uint64_t* empty, const Ctl& ctl, int my_tiles) {
+  using C = DCfg<PAIR>;
+  // with cs > 1 (single form) every CTA loads its own A tile and a 1/cs slice
+  // of the shared B tile, multicast to the whole cluster (the B maps then
+  // have DBN/cs rows); a pair CTA loads its own A tile and its half of B
   const int bq = DBN / P.cs;
-  const bool mc = P.cs > 1;
+  const bool mc = !PAIR && P.cs > 1;
   const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
   const uint32_t boff = (uint32_t)(S.rank * bq * BK * 2);
+  const bool lead = !PAIR || S.rank == 0;
+  const uint32_t full_cl = PAIR ? cluster_addr(full, 0) : 0u;  // the even CTA's full barriers
   int stage = 0;
   uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
   bool ok = true;
   const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
+  // one stage: wait until the slot is free, arm its full barrier, copy the
+  // A and B boxes
+  auto load = [&](const CUtensorMap* ma, const CUtensorMap* mb, int xk, int y0, int y1) {
+    if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) return false;
+    unsigned char* sa = stages + stage * C::STAGE;
+    uint64_t* fb = &full[stage];
+    if (lead) mbar_arrive_expect_tx(fb, C::TX);
+    if constexpr (PAIR) {
+      const uint32_t fcl = full_cl + (uint32_t)(stage * 8);
+      tma_load_2d_pair(sa, ma, fcl, xk, y0);
+      tma_load_2d_pair(sa + DSTAGE_A, mb, fcl, xk, y1);
+    } else {
+      tma_load_2d(sa, ma, fb, xk, y0);
+      if (!mc) tma_load_2d(sa + DSTAGE_A, mb, fb, xk, y1);
+      else tma_load_2d_mc(sa + DSTAGE_A + boff, mb, fb, xk, y1, mask);
+    }
+    issued_mask |= 1u << stage;
+    issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+    if (++stage == C::STAGES) {
+      stage = 0;
+      phase ^= 1u;
+    }
+    return true;
+  };
   for (int slot = 0; slot <= my_tiles && ok; ++slot) {
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
@@ -329,127 +443,127 @@ __device__ __noinline__ void draft_producer(const Params& P, const Sched& S,
     const int ya = mt * BM, yb = vt * DBN + S.rank * bq;
     const int yca = pmt * BM, ycb = pvt * DBN + S.rank * bq;
     int kx = sp * P.nb * BK;
-    int jb = 0, zd = 0;
-    int ins = nzv > 0 ? ins_point(0, nbv, nzv) : 0x7fffffff;
-    while (jb < nbv || zd < nzv) {
-      const bool br = zd < nzv && (jb >= nbv || jb == ins);
-      if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) {
-        ok = false;
-        break;
-      }
-      unsigned char* sa = stages + stage * DSTAGE;
-      uint64_t* fb = &full[stage];
-      mbar_arrive_expect_tx(fb, DSTAGE);
-      if (!br) {
-        tma_load_2d(sa, tm_a, fb, kx, ya);
-        if (!mc) tma_load_2d(sa + DSTAGE_A, tm_b, fb, kx, yb);
-        else tma_load_2d_mc(sa + DSTAGE_A + boff, tm_b, fb, kx, yb, mask);
-        kx += BK;
-        ++jb;
-      } else {
-        const int kc = (P.zps == 2 ? (zd >> 1) : zd) * BK;
-        tma_load_2d(sa, tm_ca, fb, kc, yca);
-        if (!mc) tma_load_2d(sa + DSTAGE_A, tm_cb, fb, kc, ycb);
-        else tma_load_2d_mc(sa + DSTAGE_A + boff, tm_cb, fb, kc, ycb, mask);
-        ++zd;
-        ins = zd < nzv ? ins_point(zd, nbv, nzv) : 0x7fffffff;
-      }
-      issued_mask |= 1u << stage;
-      issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-      if (++stage == DSTAGES) {
-        stage = 0;
-        phase ^= 1u;
-      }
+    int jb = 0;
+    // base stages up to the next insertion point, then one branch item
+    for (int zd = 0; zd <= nzv && ok; ++zd) {
+      const int jend = zd < nzv ? ins_point(zd, nbv, nzv) : nbv;
+      for (; jb < jend; ++jb, kx += BK)
+        if (!(ok = load(tm_a, tm_b, kx, ya, yb))) break;
+      if (ok && zd < nzv) ok = load(tm_ca, tm_cb, (P.zps == 2 ? (zd >> 1) : zd) * BK, yca, ycb);
     }
   }
-  // copies still in flight after an abort: wait (bounded) before leaving
-  for (int s = 0; s < DSTAGES; ++s)
-    if (issued_mask & (1u << s)) {
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
-             (globaltimer() - t0) < 2000000000ull) {
+  // copies still in flight after an abort: wait (bounded) before leaving.  The
+  // odd CTA of a pair cannot wait on the even CTA's barriers; its copies land
+  // within microseconds, so it waits a fixed 100 us instead.
+  if (lead) {
+    for (int s = 0; s < C::STAGES; ++s)
+      if (issued_mask & (1u << s)) {
+        const uint64_t t0 = globaltimer();
+        while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
+               (globaltimer() - t0) < 2000000000ull) {
+        }
       }
+  } else if (!ok && issued_mask) {
+    const uint64_t t0 = globaltimer();
+    while ((globaltimer() - t0) < 100000ull) {
     }
+  }
 }
 
-__device__ __noinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned char* stages,
-                                       uint64_t* full, uint64_t* empty, uint64_t* bfull,
-                                       uint64_t* bempty, uint64_t* cfull, uint64_t* cempty,
-                                       uint64_t* done, const Ctl& ctl, int my_tiles) {
-  const uint32_t id_base = idesc_f16(true, DBN);
-  const uint32_t id_corr = idesc_f16(false, DBN);
+template <bool PAIR>
+__device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsigned char* stages,
+                                          uint64_t* full, uint64_t* empty, uint64_t* bfull,
+                                          uint64_t* bempty, uint64_t* cfull, uint64_t* cempty,
+                                          uint64_t* done, const Ctl& ctl, int my_tiles) {
+  using C = DCfg<PAIR>;
+  constexpr int MM = PAIR ? 2 * BM : BM;
+  const uint32_t id_base = idesc_f16(true, DBN, MM);
+  const uint32_t id_corr = idesc_f16(false, DBN, MM);
   const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
-  const bool mc = P.cs > 1;
+  const bool mc = !PAIR && P.cs > 1;
   // shared-memory descriptors: the start-address field holds addr >> 4, so a
   // byte offset off inside the 1024-aligned stages moves it by off >> 4
   const uint64_t d0 = sdesc(smem_u32(stages));
   const uint32_t dcol = tmem + (uint32_t)DBN;
+  auto mma = [&](uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc) {
+    if constexpr (PAIR) umma_pair(d, a, b, id, acc);
+    else umma(d, a, b, id, acc);
+  };
+  // release a stage / hand an accumulator over: in a pair the commit arrives
+  // on the barrier at the same offset in both CTAs
+  auto commit_all = [&](uint64_t* bar) {
+    if constexpr (PAIR) umma_commit_pair(bar);
+    else if (mc) umma_commit_mc(bar, mask);
+    else umma_commit(bar);
+  };
+  auto commit_acc = [&](uint64_t* bar) {
+    if constexpr (PAIR) umma_commit_pair(bar);
+    else umma_commit(bar);
+  };
+  auto wait_taken = [&](uint64_t* bar, uint32_t parity, uint32_t where) {
+    if constexpr (PAIR) return mbar_wait_cl(bar, parity, ctl, where);
+    else return mbar_wait(bar, parity, ctl, where);
+  };
   int stage = 0;
   uint32_t phase = 0, cuse = 0;
+  uint64_t da = d0;  // descriptor of the current stage's A box
+  auto next = [&]() {
+    if (++stage == C::STAGES) {
+      stage = 0;
+      phase ^= 1u;
+      da = d0;
+    } else {
+      da += (uint64_t)(C::STAGE >> 4);
+    }
+  };
   bool ok = true;
   const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
   for (int slot = 0; slot <= my_tiles && ok; ++slot) {
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
-    int jb = 0, zd = 0;
-    int ins = nzv > 0 ? ins_point(0, nbv, nzv) : 0x7fffffff;
-    while (jb < nbv || zd < nzv) {
-      const bool br = zd < nzv && (jb >= nbv || jb == ins);
-      if (!br && jb == 0) {  // the epilogue has taken the previous base accumulator
-        if (!mbar_wait(bempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 2)) {
-          ok = false;
-          break;
-        }
+    int jb = 0;
+    for (int zd = 0; zd <= nzv && ok; ++zd) {
+      const int jend = zd < nzv ? ins_point(zd, nbv, nzv) : nbv;
+      if (jb == 0 && jend > 0) {  // the epilogue has taken the previous base accumulator
+        if (!(ok = wait_taken(bempty, ((uint32_t)slot & 1u) ^ 1u, 2))) break;
         tc_fence_after();
       }
-      if (br) {  // the epilogue has taken the previous branch accumulator
-        if (!mbar_wait(cempty, (cuse & 1u) ^ 1u, ctl, 4)) {
-          ok = false;
-          break;
-        }
+      for (; jb < jend; ++jb) {
+        if (!(ok = mbar_wait(&full[stage], phase, ctl, 3))) break;
         tc_fence_after();
+        const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
+        mma(tmem, da, db, id_base, jb > 0 ? 1u : 0u);
+        mma(tmem, da + 2, db + 2, id_base, 1u);
+        mma(tmem, da + 4, db + 4, id_base, 1u);
+        mma(tmem, da + 6, db + 6, id_base, 1u);
+        commit_all(&empty[stage]);
+        if (jb == nbv - 1) commit_acc(bfull);
+        next();
       }
-      if (!mbar_wait(&full[stage], phase, ctl, 3)) {
-        ok = false;
-        break;
-      }
+      if (!ok || zd == nzv) break;
+      // branch item zd of the previous tile (the epilogue has taken the
+      // previous branch accumulator): hi.hi + hi.lo + lo.hi; element offsets
+      // o (hi) and o + rp (lo) are multiples of 16 (32 bytes)
+      if (!(ok = wait_taken(cempty, (cuse & 1u) ^ 1u, 4))) break;
       tc_fence_after();
-      const uint64_t da = d0 + (uint64_t)(stage * (DSTAGE >> 4));
+      if (!(ok = mbar_wait(&full[stage], phase, ctl, 3))) break;
+      tc_fence_after();
       const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
-      if (!br) {
-        umma(tmem, da, db, id_base, jb > 0 ? 1u : 0u);
-        umma(tmem, da + 2, db + 2, id_base, 1u);
-        umma(tmem, da + 4, db + 4, id_base, 1u);
-        umma(tmem, da + 6, db + 6, id_base, 1u);
-        if (!mc) umma_commit(&empty[stage]);
-        else umma_commit_mc(&empty[stage], mask);
-        if (jb == nbv - 1) umma_commit(bfull);
-        ++jb;
-      } else {
-        // component zd of the previous tile: hi.hi + hi.lo + lo.hi; element
-        // offsets o (hi) and o + rp (lo) are multiples of 16 (32 bytes)
-        const int o = (P.zps == 2 ? (zd & 1) : 0) * 2 * P.rp;
-        for (int kk = 0; kk < P.rp; kk += 16) {
-          const uint64_t hi = (uint64_t)((o + kk) >> 3), lo = (uint64_t)((o + P.rp + kk) >> 3);
-          umma(dcol, da + hi, db + hi, id_corr, kk > 0 ? 1u : 0u);
-          umma(dcol, da + hi, db + lo, id_corr, 1u);
-          umma(dcol, da + lo, db + hi, id_corr, 1u);
-        }
-        umma_commit(cfull);
-        if (!mc) umma_commit(&empty[stage]);
-        else umma_commit_mc(&empty[stage], mask);
-        ++cuse;
-        ++zd;
-        ins = zd < nzv ? ins_point(zd, nbv, nzv) : 0x7fffffff;
+      const int o = (P.zps == 2 ? (zd & 1) : 0) * 2 * P.rp;
+      for (int kk = 0; kk < P.rp; kk += 16) {
+        const uint64_t hi = (uint64_t)((o + kk) >> 3), lo = (uint64_t)((o + P.rp + kk) >> 3);
+        mma(dcol, da + hi, db + hi, id_corr, kk > 0 ? 1u : 0u);
+        mma(dcol, da + hi, db + lo, id_corr, 1u);
+        mma(dcol, da + lo, db + hi, id_corr, 1u);
       }
-      if (++stage == DSTAGES) {
-        stage = 0;
-        phase ^= 1u;
-      }
+      commit_acc(cfull);
+      commit_all(&empty[stage]);
+      ++cuse;
+      next();
     }
   }
   // wait (bounded) for every MMA this thread issued before TMEM is freed
-  umma_commit(done);
+  commit_acc(done);
   const uint64_t t0 = globaltimer();
   while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
   }
@@ -480,6 +594,19 @@ __device__ __forceinline__ void tmem_ld16_raw(uint32_t taddr, uint32_t (&r)[16])
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// the same wait, with r passed through it: the compiler then cannot move a
+// use of r (the destination of a load still in flight) above the wait
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
+                 "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
+                 "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
+                 "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -491,6 +618,7 @@ __device__ __forceinline__ float ex2(float x) {
 // columns, t_v = D_z a_z + (base_v + b_v) k2 - ref, with ref = k2 max_v
 // (base_v + b_v) taken once per tile.  A sum outside [2^-100, 2^100] (a branch
 // offset far from the base logits) is redone against the exact maximum.
+template <bool PAIR>
 __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, int warp, int lane,
                                             float* az, float* vbs, uint64_t* vbar,
                                             uint64_t* bfull, uint64_t* bempty,
@@ -524,20 +652,30 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     }
     if (!mbar_wait(bfull, (uint32_t)slot & 1u, ctl, 5)) break;
     tc_fence_after();
+    {
+      const uint32_t tb = tmem + lane_off + (uint32_t)(half * DCOLS);
+      uint32_t ra[32], rb[32];
+      tmem_ld32_raw(tb, ra);
+      tmem_wait_ld(ra);
 #pragma unroll
-    for (int cc = 0; cc < DCOLS / 16; ++cc) {
-      uint32_t r[16];
-      tmem_ld16_raw(tmem + lane_off + (uint32_t)(half * DCOLS + cc * 16), r);
-      tmem_wait_ld();
+      for (int cc = 0; cc < DCOLS / 32; ++cc) {
+        uint32_t(&cur)[32] = (cc & 1) ? rb : ra;
+        uint32_t(&nxt)[32] = (cc & 1) ? ra : rb;
+        if (cc + 1 < DCOLS / 32) tmem_ld32_raw(tb + (uint32_t)((cc + 1) * 32), nxt);
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        bk[cc * 16 + j] = (P.mode == MODE_DRAFT) ? __uint_as_float(r[j]) + vb[cc * 16 + j]
-                                                 : __uint_as_float(r[j]);
+        for (int j = 0; j < 32; ++j)
+          bk[cc * 32 + j] = (P.mode == MODE_DRAFT) ? __uint_as_float(cur[j]) + vb[cc * 32 + j]
+                                                   : __uint_as_float(cur[j]);
+        if (cc + 1 < DCOLS / 32) tmem_wait_ld(nxt);
+      }
     }
     // the base accumulator is in registers: hand TMEM back to the MMA thread
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(bempty);
+    if (lane == 0) {
+      if constexpr (PAIR) mbar_arrive_cluster(cluster_addr(bempty, 0));  // the even CTA's
+      else mbar_arrive(bempty);
+    }
 
     if (P.mode == MODE_PREP) {
       if (m < P.prep_rows) {
@@ -591,18 +729,24 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       tc_fence_after();
       const float a = az[z * D_EPI + et];
       float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      // 32-column chunks, the load of chunk c+1 in flight while chunk c is reduced
+      const uint32_t tb = tmem + lane_off + (uint32_t)(DBN + half * DCOLS);
+      uint32_t ra[32], rb[32];
+      tmem_ld32_raw(tb, ra);
+      tmem_wait_ld(ra);
 #pragma unroll
-      for (int cc = 0; cc < DCOLS / 16; ++cc) {
-        uint32_t r[16];
-        tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
-        tmem_wait_ld();
+      for (int cc = 0; cc < DCOLS / 32; ++cc) {
+        uint32_t(&cur)[32] = (cc & 1) ? rb : ra;
+        uint32_t(&nxt)[32] = (cc & 1) ? ra : rb;
+        if (cc + 1 < DCOLS / 32) tmem_ld32_raw(tb + (uint32_t)((cc + 1) * 32), nxt);
 #pragma unroll
-        for (int j = 0; j < 16; j += 4) {
-          s0 += ex2(fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]));
-          s1 += ex2(fmaf(__uint_as_float(r[j + 1]), a, bk[cc * 16 + j + 1]));
-          s2 += ex2(fmaf(__uint_as_float(r[j + 2]), a, bk[cc * 16 + j + 2]));
-          s3 += ex2(fmaf(__uint_as_float(r[j + 3]), a, bk[cc * 16 + j + 3]));
+        for (int j = 0; j < 32; j += 4) {
+          s0 += ex2(fmaf(__uint_as_float(cur[j]), a, bk[cc * 32 + j]));
+          s1 += ex2(fmaf(__uint_as_float(cur[j + 1]), a, bk[cc * 32 + j + 1]));
+          s2 += ex2(fmaf(__uint_as_float(cur[j + 2]), a, bk[cc * 32 + j + 2]));
+          s3 += ex2(fmaf(__uint_as_float(cur[j + 3]), a, bk[cc * 32 + j + 3]));
         }
+        if (cc + 1 < DCOLS / 32) tmem_wait_ld(nxt);
       }
       float sum = (s0 + s1) + (s2 + s3);
       float rz = ref;
@@ -635,32 +779,37 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       // the branch accumulator is read: hand it back
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(cempty);
+      if (lane == 0) {
+        if constexpr (PAIR) mbar_arrive_cluster(cluster_addr(cempty, 0));
+        else mbar_arrive(cempty);
+      }
       if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(rz, sum);
     }
     if (!ok) break;
   }
 }
 
+template <bool PAIR>
 __global__ void __launch_bounds__(D_THREADS, 1)
     k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
               const Params P) {
+  using C = DCfg<PAIR>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stages = smem;
-  float* az = reinterpret_cast<float*>(smem + DSTAGES * DSTAGE);
-  float* vbs = reinterpret_cast<float*>(smem + DSTAGES * DSTAGE + DAZ_BYTES);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DSTAGES * DSTAGE + DAZ_BYTES + DVB_BYTES);
-  uint64_t* full = bars;                 // [DSTAGES]
-  uint64_t* empty = bars + DSTAGES;      // [DSTAGES]
-  uint64_t* bfull = bars + 2 * DSTAGES;  // base accumulator ready
-  uint64_t* bempty = bfull + 1;          // base accumulator taken (8 epilogue warps)
-  uint64_t* cfull = bfull + 2;           // branch accumulator ready
-  uint64_t* cempty = bfull + 3;          // branch accumulator taken (8 epilogue warps)
-  uint64_t* done = bfull + 4;            // every MMA of this CTA finished
-  uint64_t* vbar = bfull + 5;            // a tile's vocabulary bias staged (256 epilogue threads)
+  float* az = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE);
+  float* vbs = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE + DAZ_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE + DAZ_BYTES + DVB_BYTES);
+  uint64_t* full = bars;                    // [STAGES]
+  uint64_t* empty = bars + C::STAGES;       // [STAGES]
+  uint64_t* bfull = bars + 2 * C::STAGES;   // base accumulator ready
+  uint64_t* bempty = bfull + 1;             // base accumulator taken (8 epilogue warps per CTA)
+  uint64_t* cfull = bfull + 2;              // branch accumulator ready
+  uint64_t* cempty = bfull + 3;             // branch accumulator taken (8 epilogue warps per CTA)
+  uint64_t* done = bfull + 4;               // every MMA of this CTA finished
+  uint64_t* vbar = bfull + 5;               // a tile's vocabulary bias staged (256 epilogue threads)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 6);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -670,14 +819,16 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   const Ctl ctl{P.spin_limit, abort_flag, P.status};
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < DSTAGES; ++s) {
+    for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], P.cs);  // one MMA commit from every CTA of the cluster
+      // one MMA commit from every CTA of a multicast cluster; a pair's MMAs
+      // are issued (and committed) by the even CTA alone
+      mbar_init(&empty[s], PAIR ? 1 : P.cs);
     }
     mbar_init(bfull, 1);
-    mbar_init(bempty, 8);
+    mbar_init(bempty, PAIR ? 16 : 8);
     mbar_init(cfull, 1);
-    mbar_init(cempty, 8);
+    mbar_init(cempty, PAIR ? 16 : 8);
     mbar_init(done, 1);
     mbar_init(vbar, D_EPI);
     *abort_flag = 0;
@@ -685,38 +836,55 @@ __global__ void __launch_bounds__(D_THREADS, 1)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS));
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    if constexpr (PAIR) {
+      // one warp of each CTA of the pair allocates the same columns in both SMs
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS));
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS));
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   // every CTA's barriers exist before any multicast copy or commit reaches them
-  if (P.cs > 1) cluster_sync_all();
+  if (PAIR || P.cs > 1) cluster_sync_all();
   const uint32_t tmem = *tmem_slot;
 
   if (warp >= 4) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
-    draft_epilogue(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl, my_tiles);
+    draft_epilogue<PAIR>(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl,
+                         my_tiles);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
     if (warp == 0 && lane == 0)
-      draft_producer(P, S, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
-    else if (warp == 1 && lane == 0)
-      draft_mma(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl, my_tiles);
+      draft_producer<PAIR>(P, S, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
+    else if (warp == 1 && lane == 0 && (!PAIR || S.rank == 0))
+      draft_mma<PAIR>(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl,
+                      my_tiles);
   }
 
   tc_fence_before();
   __syncthreads();
+  // a pair frees its columns only after the even CTA's MMAs (which write both
+  // SMs' TMEM) have completed
+  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(TMEM_COLS));
+    if constexpr (PAIR)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                   "r"(TMEM_COLS));
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                   "r"(TMEM_COLS));
   }
   // no CTA leaves while a peer may still multicast into it or arrive on it
-  if (P.cs > 1) cluster_sync_all();
+  if (PAIR || P.cs > 1) cluster_sync_all();
 }
 
 // ------------------------------------------------------------ verify pass
@@ -1111,16 +1279,18 @@ static int num_sms() {
 // The register split of k_tc_pass (setmaxnreg) assumes the kernel was built
 // with exactly DREG registers per thread: with fewer, the epilogue's increase
 // could never be granted.  Such a build is refused instead of launched.
+template <bool PAIR>
 static cudaError_t pass_kernel_ready() {
   static int state = -1;
   if (state < 0) {
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass);
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != DREG) {
       state = 0;
     } else {
-      e = cudaFuncSetAttribute(k_tc_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)DSMEM);
+      e = cudaFuncSetAttribute(k_tc_pass<PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)DCfg<PAIR>::SMEM);
       if (e != cudaSuccess) return e;
       state = 1;
     }
@@ -1128,52 +1298,51 @@ static cudaError_t pass_kernel_ready() {
   return state == 1 ? cudaSuccess : cudaErrorInvalidKernelImage;
 }
 
-// clusters of cs CTAs that can be resident at once (cached per size)
+static cudaLaunchConfig_t cluster_config(int grid, int cs, size_t smem, cudaStream_t s,
+                                         cudaLaunchAttribute* at) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(D_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = cs;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+// clusters of cs CTAs that can be resident at once (cached per form and size)
+template <bool PAIR>
 static int max_clusters(int cs) {
   static int cache[5] = {0, 0, 0, 0, 0};
   if (cs < 1 || cs > 4) return 0;
   if (!cache[cs]) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(cs * num_sms());
-    cfg.blockDim = dim3(D_THREADS);
-    cfg.dynamicSmemBytes = DSMEM;
     cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = cs;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
+    cudaLaunchConfig_t cfg = cluster_config(cs * num_sms(), cs, DCfg<PAIR>::SMEM, 0, at);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass, &cfg) != cudaSuccess || n < 1) n = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass<PAIR>, &cfg) != cudaSuccess || n < 1) n = 1;
     cache[cs] = n;
   }
   return cache[cs];
 }
 
+template <bool PAIR>
 static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
                           const CUtensorMap& cb, const Params& P, cudaStream_t s) {
-  cudaError_t e = pass_kernel_ready();
+  cudaError_t e = pass_kernel_ready<PAIR>();
   if (e != cudaSuccess) return e;
   if (P.n_tiles <= 0) return cudaSuccess;
-  if (P.cs == 1) {
+  if (!PAIR && P.cs == 1) {
     const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
-    k_tc_pass<<<grid, D_THREADS, DSMEM, s>>>(a, b, ca, cb, P);
+    k_tc_pass<false><<<grid, D_THREADS, DCfg<false>::SMEM, s>>>(a, b, ca, cb, P);
   } else {
-    const int ncl = std::min(P.n_tiles, max_clusters(P.cs));
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(ncl * P.cs);
-    cfg.blockDim = dim3(D_THREADS);
-    cfg.dynamicSmemBytes = DSMEM;
-    cfg.stream = s;
+    const int ncl = std::min(P.n_tiles, max_clusters<PAIR>(P.cs));
     cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = P.cs;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, k_tc_pass, a, b, ca, cb, P);
+    cudaLaunchConfig_t cfg = cluster_config(ncl * P.cs, P.cs, DCfg<PAIR>::SMEM, s, at);
+    e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR>, a, b, ca, cb, P);
     if (e != cudaSuccess) return e;
   }
   debug_kernel("k_tc_pass", s);
@@ -1182,17 +1351,25 @@ static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUte
   return cudaGetLastError();
 }
 
-// CTAs per cluster of the draft pass: the M tiles that share a vocabulary
-// tile.  One by default: multicasting the shared B tile halves L2 reads but
-// not the shared-memory traffic per SM, and the lockstep it imposes measured
-// slower on this GPU.  DBLAST_DRAFT_CLUSTER=2|4 selects the multicast
-// schedule (tests cover every size).
+// CTAs per cluster of the single-SM draft schedule: the M tiles that share a
+// vocabulary tile.  One by default: multicasting the shared B tile halves L2
+// reads but not the shared-memory traffic per SM, and the lockstep it imposes
+// measured slower on this GPU.  DBLAST_DRAFT_CLUSTER=2|4 selects the
+// multicast schedule (tests cover every size).
 static int draft_cluster_size(int n_mt) {
   int cs = 1;
   const char* env = getenv("DBLAST_DRAFT_CLUSTER");
   if (env && (env[0] == '1' || env[0] == '2' || env[0] == '4') && env[1] == 0) cs = env[0] - '0';
   while (cs > 1 && (n_mt % cs) != 0) cs >>= 1;
   return cs;
+}
+
+// The CTA-pair schedule (the default) needs an even number of M tiles: a
+// pair covers 256 rows.  DBLAST_DRAFT_PAIR=0 forces the single-SM schedule.
+static bool draft_pair(int n_mt) {
+  if (n_mt % 2 != 0) return false;
+  const char* env = getenv("DBLAST_DRAFT_PAIR");
+  return !(env && env[0] == '0' && env[1] == 0);
 }
 
 }  // namespace tc
@@ -1264,7 +1441,7 @@ cudaError_t launch_prep_tc(const dblast_head* h, const PrepLayout& pl, cudaStrea
   P.split_stride = 0;
   P.status = reinterpret_cast<DevStatus*>(prep + pl.off_status);
   P.spin_limit = wait_limit();
-  return tc::launch(ma, mb, ma, mb, P, s);
+  return tc::launch<false>(ma, mb, ma, mb, P, s);
 }
 
 // codes c_{m,z} = V_z^T h_m for every position: the prep machinery with
@@ -1302,14 +1479,15 @@ cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit) {
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
   *nsplit = ks;
-  return tc::launch(ma, mb, ma, mb, P, c.stream);
+  return tc::launch<false>(ma, mb, ma, mb, P, c.stream);
 }
 
 cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   const dblast_head* h = c.head;
   const WsLayout& w = c.wl;
   const int n_mt = w.Mpad / tc::BM;
-  const int cs = tc::draft_cluster_size(n_mt);
+  const bool pair = tc::draft_pair(n_mt);
+  const int cs = pair ? 2 : tc::draft_cluster_size(n_mt);
   const uint32_t bq = tc::DBN / cs;  // B rows each CTA of a cluster loads
   CUtensorMap ma, mb, mca, mcb;
   const unsigned char* prep = c.prep;
@@ -1339,7 +1517,8 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   P.partd = wsp<float2>(c, w.off_partd);
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
-  return tc::launch(ma, mb, mca, mcb, P, c.stream);
+  return pair ? tc::launch<true>(ma, mb, mca, mcb, P, c.stream)
+              : tc::launch<false>(ma, mb, mca, mcb, P, c.stream);
 }
 
 cudaError_t launch_verify_pass_tc(const StepCtx& c) {

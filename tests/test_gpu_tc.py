@@ -51,6 +51,7 @@ def test_draft_pass_cluster_multicast_matches_single_cta(cs, monkeypatch):
     head = synth.make_head(cfg, "cuda")
     blk = synth.make_block(cfg, head, 0, "cuda")
     runs = {}
+    monkeypatch.setenv("DBLAST_DRAFT_PAIR", "0")  # the multicast schedule is a one-SM form
     for c in ("1", cs):
         monkeypatch.setenv("DBLAST_DRAFT_CLUSTER", c)
         pos, rnd = synth.initial_state(cfg, "cuda")
@@ -61,3 +62,28 @@ def test_draft_pass_cluster_multicast_matches_single_cta(cs, monkeypatch):
     seqs = [0, 13, 31]
     orc = parity.run_oracle(head, blk, 0.8, 1.0, 7, pos0, rnd0, seqs)
     parity.compare(runs[cs], orc, seqs)
+
+
+@pytest.mark.parametrize("over", [dict(V=20000, H=512, K=8, r=16, B=16, N=32),   # 4 M tiles
+                                  dict(V=3001, H=256, K=3, r=4, B=5, N=40,        # 2 M tiles
+                                       expander_bias=True)])
+def test_draft_pass_cta_pair_matches_single_cta(over, monkeypatch):
+    """The CTA-pair draft pass (cta_group::2 MMAs of 256 rows, B split between
+    the two SMs) computes the same products in the same order as the one-SM
+    pass: the oracle checks sampled sequences, and every output must equal
+    the one-SM schedule's bit for bit."""
+    from tests import parity
+    cfg = synth.config("qwen3_8b_b32", **over)
+    head = synth.make_head(cfg, "cuda")
+    blk = synth.make_block(cfg, head, 0, "cuda")
+    runs = {}
+    for c in ("0", "1"):
+        monkeypatch.setenv("DBLAST_DRAFT_PAIR", c)
+        pos, rnd = synth.initial_state(cfg, "cuda")
+        runs[c] = parity.run_gpu(head, blk, 0.8, 1.0, 7, pos, rnd, impl="tcgen05")
+    pos0, rnd0 = synth.initial_state(cfg, "cuda")
+    seqs = [0, cfg["N"] // 2 - 1, cfg["N"] - 1]
+    orc = parity.run_oracle(head, blk, 0.8, 1.0, 7, pos0, rnd0, seqs)
+    parity.compare(runs["1"], orc, seqs)
+    for k, v in runs["0"].items():
+        assert torch.equal(v, runs["1"][k]), k
