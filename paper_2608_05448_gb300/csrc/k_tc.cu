@@ -213,8 +213,18 @@ __device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
   return r;
 }
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t caddr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr)
+// Hand-over of a TMEM accumulator the thread has finished reading
+// (tcgen05.wait::ld has returned, so the values are in registers): nothing
+// written before it needs to be visible to the waiter, so the arrive is
+// relaxed.  A release arrive would first wait for the thread's earlier global
+// stores (the stash rows, the records) to become visible, which at cluster
+// scope takes a large part of a component's epilogue.
+__device__ __forceinline__ void mbar_arrive_taken(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_taken_cluster(uint32_t caddr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr)
                : "memory");
 }
 // a wait whose arrivals may come from the other CTA of the pair
@@ -293,8 +303,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
 }
 
 // ------------------------------------------------------------ draft pass
-// 128 x 256 tiles: TMEM columns [0, 256) hold the base accumulator, [256, 512)
-// the branch accumulator of one component.  12 warps: warp 0 issues TMA, warp
+// 128 x 256 tiles in two TMEM regions of 256 columns: tile t accumulates its
+// base GEMM in region t & 1, and once the epilogue has taken that base, the
+// same region holds its branch components one at a time, while tile t+1's
+// base accumulates in the other region.  The MMA issuer therefore never waits
+// for a base accumulator to be read; it waits only until tile t-1's last
+// component has been taken before starting tile t+1.  12 warps: warp 0 issues TMA, warp
 // 1 issues MMAs and owns TMEM, warps 4-11 are the epilogue (two per TMEM lane
 // quarter, 128 columns each).  Warpgroup 0 gives registers to the epilogue
 // warpgroups with setmaxnreg (56 + 2 x 224 = 3 x 168 per thread).
@@ -484,7 +498,6 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
   // shared-memory descriptors: the start-address field holds addr >> 4, so a
   // byte offset off inside the 1024-aligned stages moves it by off >> 4
   const uint64_t d0 = sdesc(smem_u32(stages));
-  const uint32_t dcol = tmem + (uint32_t)DBN;
   auto mma = [&](uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc) {
     if constexpr (PAIR) umma_pair(d, a, b, id, acc);
     else umma(d, a, b, id, acc);
@@ -505,7 +518,8 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
     else return mbar_wait(bar, parity, ctl, where);
   };
   int stage = 0;
-  uint32_t phase = 0, cuse = 0;
+  uint32_t phase = 0;
+  uint32_t cuse0 = 0u, cuse1 = 0u;  // components issued into TMEM region 0 / 1
   uint64_t da = d0;  // descriptor of the current stage's A box
   auto next = [&]() {
     if (++stage == C::STAGES) {
@@ -521,30 +535,43 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
   for (int slot = 0; slot <= my_tiles && ok; ++slot) {
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
+    // tile `slot` accumulates in region r, the components of tile slot-1 in
+    // the other one (where that tile's base was)
+    const int r = slot & 1;
+    const uint32_t dbase = tmem + (uint32_t)(r * DBN), dcol = tmem + (uint32_t)((r ^ 1) * DBN);
     int jb = 0;
     for (int zd = 0; zd <= nzv && ok; ++zd) {
       const int jend = zd < nzv ? ins_point(zd, nbv, nzv) : nbv;
-      if (jb == 0 && jend > 0) {  // the epilogue has taken the previous base accumulator
-        if (!(ok = wait_taken(bempty, ((uint32_t)slot & 1u) ^ 1u, 2))) break;
+      if (jb == 0 && jend > 0) {
+        // region r is free once the epilogue has taken tile slot-2's base
+        // and every component computed there
+        if (!(ok = wait_taken(&bempty[r], ((uint32_t)(slot >> 1) & 1u) ^ 1u, 2))) break;
+        const uint32_t cu = r ? cuse1 : cuse0;
+        if (cu > 0 && !(ok = wait_taken(&cempty[r], (cu - 1u) & 1u, 4))) break;
         tc_fence_after();
       }
       for (; jb < jend; ++jb) {
         if (!(ok = mbar_wait(&full[stage], phase, ctl, 3))) break;
         tc_fence_after();
         const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
-        mma(tmem, da, db, id_base, jb > 0 ? 1u : 0u);
-        mma(tmem, da + 2, db + 2, id_base, 1u);
-        mma(tmem, da + 4, db + 4, id_base, 1u);
-        mma(tmem, da + 6, db + 6, id_base, 1u);
+        mma(dbase, da, db, id_base, jb > 0 ? 1u : 0u);
+        mma(dbase, da + 2, db + 2, id_base, 1u);
+        mma(dbase, da + 4, db + 4, id_base, 1u);
+        mma(dbase, da + 6, db + 6, id_base, 1u);
         commit_all(&empty[stage]);
-        if (jb == nbv - 1) commit_acc(bfull);
+        if (jb == nbv - 1) commit_acc(&bfull[r]);
         next();
       }
       if (!ok || zd == nzv) break;
-      // branch item zd of the previous tile (the epilogue has taken the
-      // previous branch accumulator): hi.hi + hi.lo + lo.hi; element offsets
-      // o (hi) and o + rp (lo) are multiples of 16 (32 bytes)
-      if (!(ok = wait_taken(cempty, (cuse & 1u) ^ 1u, 4))) break;
+      // branch item zd of the previous tile, in its region once the epilogue
+      // has taken that tile's base (zd = 0) or component zd-1:
+      // hi.hi + hi.lo + lo.hi; element offsets o (hi) and o + rp (lo) are
+      // multiples of 16 (32 bytes)
+      if (zd == 0) {
+        if (!(ok = wait_taken(&bempty[r ^ 1], (uint32_t)((slot - 1) >> 1) & 1u, 2))) break;
+      } else {
+        if (!(ok = wait_taken(&cempty[r ^ 1], ((r ? cuse0 : cuse1) - 1u) & 1u, 4))) break;
+      }
       tc_fence_after();
       if (!(ok = mbar_wait(&full[stage], phase, ctl, 3))) break;
       tc_fence_after();
@@ -556,9 +583,10 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
         mma(dcol, da + hi, db + lo, id_corr, 1u);
         mma(dcol, da + lo, db + hi, id_corr, 1u);
       }
-      commit_acc(cfull);
+      commit_acc(&cfull[r ^ 1]);
       commit_all(&empty[stage]);
-      ++cuse;
+      if (r) ++cuse0;
+      else ++cuse1;
       next();
     }
   }
@@ -630,7 +658,6 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
   const int row = q * 32 + lane;
   const int et = ew * 32 + lane;
   const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-  uint32_t cuse = 0;
   const Sched S = sched_of(P);
   for (int slot = 0; slot < my_tiles; ++slot) {
     int sp, mt, vt;
@@ -650,10 +677,11 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       mbar_arrive(vbar);
       if (!mbar_wait(vbar, (uint32_t)slot & 1u, ctl, 7)) break;
     }
-    if (!mbar_wait(bfull, (uint32_t)slot & 1u, ctl, 5)) break;
+    const int rg = slot & 1;  // the tile's TMEM region (base, then its components)
+    if (!mbar_wait(&bfull[rg], (uint32_t)(slot >> 1) & 1u, ctl, 5)) break;
     tc_fence_after();
     {
-      const uint32_t tb = tmem + lane_off + (uint32_t)(half * DCOLS);
+      const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
       uint32_t ra[32], rb[32];
       tmem_ld32_raw(tb, ra);
       tmem_wait_ld(ra);
@@ -673,8 +701,8 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     tc_fence_before();
     __syncwarp();
     if (lane == 0) {
-      if constexpr (PAIR) mbar_arrive_cluster(cluster_addr(bempty, 0));  // the even CTA's
-      else mbar_arrive(bempty);
+      if constexpr (PAIR) mbar_arrive_taken_cluster(cluster_addr(&bempty[rg], 0));  // the even CTA's
+      else mbar_arrive_taken(&bempty[rg]);
     }
 
     if (P.mode == MODE_PREP) {
@@ -721,16 +749,15 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     const int rec = vt * 2 + half;
     bool ok = true;
     for (int z = 0; z < P.K; ++z) {
-      if (!mbar_wait(cfull, cuse & 1u, ctl, 6)) {
+      if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6)) {
         ok = false;
         break;
       }
-      ++cuse;
       tc_fence_after();
       const float a = az[z * D_EPI + et];
       float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
       // 32-column chunks, the load of chunk c+1 in flight while chunk c is reduced
-      const uint32_t tb = tmem + lane_off + (uint32_t)(DBN + half * DCOLS);
+      const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
       uint32_t ra[32], rb[32];
       tmem_ld32_raw(tb, ra);
       tmem_wait_ld(ra);
@@ -757,7 +784,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
 #pragma unroll
         for (int cc = 0; cc < DCOLS / 16; ++cc) {
           uint32_t r[16];
-          tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
+          tmem_ld16_raw(tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS + cc * 16), r);
           tmem_wait_ld();
 #pragma unroll
           for (int j = 0; j < 16; ++j) mx = fmaxf(mx, fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]));
@@ -766,7 +793,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
 #pragma unroll
         for (int cc = 0; cc < DCOLS / 16; ++cc) {
           uint32_t r[16];
-          tmem_ld16_raw(tmem + lane_off + (uint32_t)(DBN + half * DCOLS + cc * 16), r);
+          tmem_ld16_raw(tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS + cc * 16), r);
           tmem_wait_ld();
 #pragma unroll
           for (int j = 0; j < 16; ++j) s += ex2(fmaf(__uint_as_float(r[j]), a, bk[cc * 16 + j]) - mx);
@@ -780,8 +807,8 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if constexpr (PAIR) mbar_arrive_cluster(cluster_addr(cempty, 0));
-        else mbar_arrive(cempty);
+        if constexpr (PAIR) mbar_arrive_taken_cluster(cluster_addr(&cempty[rg], 0));
+        else mbar_arrive_taken(&cempty[rg]);
       }
       if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(rz, sum);
     }
@@ -804,13 +831,15 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE + DAZ_BYTES + DVB_BYTES);
   uint64_t* full = bars;                    // [STAGES]
   uint64_t* empty = bars + C::STAGES;       // [STAGES]
-  uint64_t* bfull = bars + 2 * C::STAGES;   // base accumulator ready
-  uint64_t* bempty = bfull + 1;             // base accumulator taken (8 epilogue warps per CTA)
-  uint64_t* cfull = bfull + 2;              // branch accumulator ready
-  uint64_t* cempty = bfull + 3;             // branch accumulator taken (8 epilogue warps per CTA)
-  uint64_t* done = bfull + 4;               // every MMA of this CTA finished
-  uint64_t* vbar = bfull + 5;               // a tile's vocabulary bias staged (256 epilogue threads)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 6);
+  // per TMEM region: base accumulator ready / taken (8 epilogue warps per
+  // CTA), branch accumulator ready / taken
+  uint64_t* bfull = bars + 2 * C::STAGES;   // [2]
+  uint64_t* bempty = bfull + 2;             // [2]
+  uint64_t* cfull = bfull + 4;              // [2]
+  uint64_t* cempty = bfull + 6;             // [2]
+  uint64_t* done = bfull + 8;               // every MMA of this CTA finished
+  uint64_t* vbar = bfull + 9;               // a tile's vocabulary bias staged (256 epilogue threads)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 10);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -825,10 +854,12 @@ __global__ void __launch_bounds__(D_THREADS, 1)
       // are issued (and committed) by the even CTA alone
       mbar_init(&empty[s], PAIR ? 1 : P.cs);
     }
-    mbar_init(bfull, 1);
-    mbar_init(bempty, PAIR ? 16 : 8);
-    mbar_init(cfull, 1);
-    mbar_init(cempty, PAIR ? 16 : 8);
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(&bfull[g], 1);
+      mbar_init(&bempty[g], PAIR ? 16 : 8);
+      mbar_init(&cfull[g], 1);
+      mbar_init(&cempty[g], PAIR ? 16 : 8);
+    }
     mbar_init(done, 1);
     mbar_init(vbar, D_EPI);
     *abort_flag = 0;
@@ -1121,7 +1152,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sempty[gs]);
+        if (lane == 0) mbar_arrive_taken(&sempty[gs]);
       }
       if (!ok) break;
       // four partial sums per quantity keep the add chains short
