@@ -16,6 +16,8 @@
 // float-float pairs (FF); exponents subtract a normaliser held as a pair, so
 // the rounded part of every exponent is the small difference, not the large
 // logit.
+#include <type_traits>
+
 #include "dblast_internal.cuh"
 
 namespace dblast {
@@ -558,12 +560,145 @@ __global__ void __launch_bounds__(TS_NT)
   }
 }
 
+// bf16 rows with V % 8 == 0 and 16-byte alignment: one block of TS2_NW warps
+// per row.  A warp stages groups of 32 whole tiles (32 x 128 tokens, 8 KB) in
+// shared memory with cp.async (double-buffered: the next group lands while
+// this one is reduced), then every lane reduces one tile by itself, with no
+// shuffles: the tile record (max, sum 2^{(t - max) k2}) and the lane's running
+// (max, float-float sum) for the row's log-sum-exp.  Chunk j (16 bytes) of
+// tile t sits at chunk j ^ (t & 7) of the tile's 256 bytes, so both the
+// copies and the per-lane reads touch eight different bank groups per phase.
+constexpr int TS2_NW = 3;
+__device__ __forceinline__ float ex2a(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__global__ void __launch_bounds__(32 * TS2_NW)
+    k_target_stats_tiles(const __nv_bfloat16* __restrict__ target, int V, int nt, int B, int Bt,
+                         int Rt, float k2, float2* __restrict__ partt, float2* __restrict__ lt2,
+                         float* __restrict__ lse_out) {
+  __shared__ __align__(16) uint4 stg[TS2_NW][2][32 * 16];  // 48 KB
+  const int row = blockIdx.x;
+  const int n = row / Bt, i = row - n * Bt;
+  const int rl = n * (B + 1) + i;
+  const uint4* tr = reinterpret_cast<const uint4*>(target + (size_t)row * V);
+  const int nchunk = V >> 3;
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  const int groups = (nt + 31) >> 5;
+  // lane l copies chunk (l & 15) of tiles 2k + (l >> 4) of group g into
+  // buffer b; chunks past the row become bf16 -inf
+  auto stage = [&](int g, int b) {
+    uint4* ws = stg[w][b];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int tt = 2 * k + (l >> 4), j = l & 15;
+      const int c = ((g << 5) + tt) * 16 + j;
+      uint4* dst = ws + tt * 16 + (j ^ (tt & 7));
+      if (c < nchunk) {
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                         static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+                     "l"(tr + c)
+                     : "memory");
+      } else {
+        *dst = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+      }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  float rmax = -INFINITY;
+  FF rsum{0.f, 0.f};
+  int buf = 0;
+  if (w < groups) stage(w, 0);
+  for (int g = w; g < groups; g += TS2_NW, buf ^= 1) {
+    if (g + TS2_NW < groups) {
+      stage(g + TS2_NW, buf ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncwarp();
+    const uint4* ws = stg[w][buf];
+    const int t = (g << 5) + l;
+    // the tile's maximum on bf16 pairs, then the sum against it
+    __nv_bfloat162 m2 = __float2bfloat162_rn(-INFINITY);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const uint4 q = ws[l * 16 + (j ^ (l & 7))];
+      m2 = __hmax2(m2, __hmax2(__hmax2(*reinterpret_cast<const __nv_bfloat162*>(&q.x),
+                                       *reinterpret_cast<const __nv_bfloat162*>(&q.y)),
+                               __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&q.z),
+                                       *reinterpret_cast<const __nv_bfloat162*>(&q.w))));
+    }
+    const float mx = fmaxf(__low2float(m2), __high2float(m2));
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const uint4 q = ws[l * 16 + (j ^ (l & 7))];
+      const uint32_t u[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const float a = __uint_as_float(u[h] << 16), b = __uint_as_float(u[h] & 0xFFFF0000u);
+        s4[h] += ex2a((a - mx) * k2) + ex2a((b - mx) * k2);
+      }
+    }
+    __syncwarp();  // every lane has read this buffer before it is refilled
+    if (t < nt) {
+      const float s = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      partt[(size_t)t * Rt + rl] = make_float2(mx, s);
+      if (mx > rmax) {
+        rsum = ff_mulf(rsum, exp2f((rmax - mx) * k2));
+        rmax = mx;
+      }
+      rsum = ff_addf(rsum, s * exp2f((mx - rmax) * k2));
+    }
+  }
+  // lanes, then warps
+  float M1 = rmax;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M1 = fmaxf(M1, __shfl_xor_sync(FULLMASK, M1, o));
+  FF S1{0.f, 0.f};
+  if (M1 != -INFINITY && rmax != -INFINITY) S1 = ff_mulf(rsum, exp2f((rmax - M1) * k2));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) S1 = ff_add(S1, ff_shfl_xor(S1, o));
+  // each warp's partial goes into the first entry of its own (now idle) buffer
+  if (l == 0) stg[w][0][0] = make_uint4(__float_as_uint(M1), __float_as_uint(S1.hi),
+                                        __float_as_uint(S1.lo), 0u);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float M2 = -INFINITY;
+    for (int k = 0; k < TS2_NW; ++k) M2 = fmaxf(M2, __uint_as_float(stg[k][0][0].x));
+    FF S{0.f, 0.f};
+    if (M2 != -INFINITY)
+      for (int k = 0; k < TS2_NW; ++k) {
+        const uint4 e = stg[k][0][0];
+        const float mk = __uint_as_float(e.x);
+        if (mk != -INFINITY)
+          S = ff_add(S, ff_mulf(FF{__uint_as_float(e.y), __uint_as_float(e.z)}, exp2f((mk - M2) * k2)));
+      }
+    const FF L = (M2 == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
+                                                   : ff_add(ff_prod(M2, k2), ff_log2(S));
+    lt2[rl] = ff_st(L);
+    if (lse_out) lse_out[row] = ff_f(L) * LN2;
+  }
+}
+
 template <typename Tin>
 static cudaError_t target_typed(const StepCtx& c, const dblast_verify_out* o) {
   const WsLayout& w = c.wl;
   const int Bt = w.B + (o->has_bonus ? 1 : 0);
   const int rows = w.N * Bt;
   const bool vec = (w.V % 8) == 0 && (reinterpret_cast<uintptr_t>(o->target) & 15u) == 0;
+  if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+    if (vec) {
+      k_target_stats_tiles<<<rows, 32 * TS2_NW, 0, c.stream>>>(
+          static_cast<const __nv_bfloat16*>(o->target), w.V, w.nt, w.B, Bt, w.Rt, c.k2,
+          wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), o->lse_target);
+      debug_kernel("k_target_stats_tiles", c.stream);
+      count_launches(1);
+      return cudaGetLastError();
+    }
+  }
   k_target_stats<Tin><<<rows, TS_NT, 0, c.stream>>>(
       static_cast<const Tin*>(o->target), w.V, w.nt, w.B, Bt, w.Rt, c.k2, vec,
       wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), o->lse_target);
