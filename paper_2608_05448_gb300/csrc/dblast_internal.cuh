@@ -244,6 +244,30 @@ void count_launches(int n);
 void count_tc_launch();
 // with DBLAST_DEBUG_SYNC=1: synchronise and report the kernel just launched
 void debug_kernel(const char* name, cudaStream_t s);
+
+// Programmatic dependent launch: a kernel launched this way may be scheduled
+// while the previous kernel of the stream is still finishing (its blocks
+// fill the SMs that kernel's blocks leave), and must run griddep_wait()
+// before it touches memory that kernel writes.  In a kernel launched the
+// ordinary way griddep_wait() returns at once.
+__device__ __forceinline__ void griddep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dep(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, static_cast<KArgs>(args)...);
+}
 void pass_event_begin(int which, cudaStream_t s);  // which: 0 draft pass, 1 verify pass
 void pass_event_end(int which, cudaStream_t s);
 

@@ -282,6 +282,7 @@ constexpr int LSE_WARPS = 16;
 __global__ void __launch_bounds__(LSE_WARPS * 32)
     k_draft_lse(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
                 float4* __restrict__ lsep) {
+  griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ float smx[LSE_WARPS][32];
   __shared__ FF ssum[LSE_WARPS][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -338,6 +339,7 @@ __global__ void __launch_bounds__(DT_NT)
                   const int64_t* __restrict__ pos, const uint32_t* __restrict__ rnd,
                   float2* __restrict__ lse2, int32_t* __restrict__ tok, float2* __restrict__ lq2,
                   uint32_t* __restrict__ ties) {
+  griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<DT_NT> fs;
   __shared__ FF sL[32];
   const int m = blockIdx.x, tid = threadIdx.x;
@@ -387,6 +389,7 @@ __global__ void __launch_bounds__(1024)
                 const float* __restrict__ sw, float k2, int B, int K, float2* __restrict__ w2,
                 float* __restrict__ qtok, float2* __restrict__ vcz, float* __restrict__ vb0,
                 dblast_draft_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FF A[1024];
   __shared__ FF rowv[32];
   __shared__ float rowb[32];
@@ -457,10 +460,11 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
   const WsLayout& w = c.wl;
   const dblast_block_args* a = c.args;
   const int K = c.head->K;
-  k_draft_lse<<<dim3(ceil_div(w.M, 32), K, LSE_SPLIT), LSE_WARPS * 32, 0, c.stream>>>(
-      wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+  cudaError_t le =
+      launch_dep(k_draft_lse, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
+                 c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
   debug_kernel("k_draft_lse", c.stream);
-  k_draft_token<<<w.M, DT_NT, 0, c.stream>>>(
+  if (le == cudaSuccess) le = launch_dep(k_draft_token, dim3(w.M), dim3(DT_NT), 0, c.stream,
       wsp<float2>(c, w.off_partd), wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_stash),
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<int32_t>(c, w.off_zhat), w.nt,
       w.V, K, w.rr, w.B, w.M, w.Mpad, c.k2, a->seed, a->pos, a->round, wsp<float2>(c, w.off_lse2),
@@ -469,14 +473,14 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
   dblast_draft_out out{};
   if (outp) out = *outp;
   const int pt = ceil_div(w.B * K, 32) * 32;
-  k_posterior<<<w.N, pt, 0, c.stream>>>(
+  if (le == cudaSuccess) le = launch_dep(k_posterior, dim3(w.N), dim3(pt), 0, c.stream,
       wsp<float2>(c, w.off_lq2), wsp<float2>(c, w.off_lse2), wsp<float>(c, w.off_log2pi),
       wsp<int32_t>(c, w.off_zhat), wsp<int32_t>(c, w.off_tok), wsp<float>(c, w.off_cscale),
       prp<float>(c, c.pl.off_sw), c.k2, w.B, K, wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_vcz), wsp<float>(c, w.off_vb0), out);
   debug_kernel("k_posterior", c.stream);
   count_launches(3);
-  return cudaGetLastError();
+  return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- target side
@@ -719,6 +723,7 @@ constexpr int AVM_WARPS = 16;
 __global__ void __launch_bounds__(AVM_WARPS * 32)
     k_verify_merge(const float2* __restrict__ partv, int nt, int M, int Mpad,
                    float4* __restrict__ avp) {
+  griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FF sa[AVM_WARPS][32], sr[AVM_WARPS][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int m = blockIdx.x * 32 + lane, sp = blockIdx.y;
@@ -766,6 +771,7 @@ __global__ void __launch_bounds__(VF_NT)
                    int nt, int M, int Mpad, int Rt, float k2, uint64_t seed,
                    int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
                    dblast_verify_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<VF_NT> fs;
   __shared__ FF sC[32];
   __shared__ int sL;
@@ -903,10 +909,10 @@ template <typename Tin>
 static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out* o) {
   const int Bt = c.Bt;
   const WsLayout& w = c.wl;
-  k_verify_merge<<<dim3(ceil_div(w.M, 32), AV_SPLIT), AVM_WARPS * 32, 0, c.stream>>>(
-      wsp<float2>(c, w.off_partv), w.nt, w.M, w.Mpad, wsp<float4>(c, w.off_av));
+  cudaError_t le = launch_dep(k_verify_merge, dim3(ceil_div(w.M, 32), AV_SPLIT),
+                              dim3(AVM_WARPS * 32), 0, c.stream, wsp<float2>(c, w.off_partv), w.nt, w.M, w.Mpad, wsp<float4>(c, w.off_av));
   debug_kernel("k_verify_merge", c.stream);
-  k_verify_final<Tin><<<w.N, VF_NT, 0, c.stream>>>(
+  if (le == cudaSuccess) le = launch_dep(k_verify_final<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
       static_cast<const Tin*>(o->target), wsp<float>(c, w.off_stash), prp<float>(c, c.pl.off_wu),
       wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2), wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
@@ -915,7 +921,7 @@ static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out*
       c.args->seed, c.args->pos, c.args->round, *o);
   debug_kernel("k_verify_final", c.stream);
   count_launches(2);
-  return cudaGetLastError();
+  return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {

@@ -251,6 +251,7 @@ __global__ void __launch_bounds__(256)
 __global__ void k_codes_finish(const float* __restrict__ part, int nsplit, int M, int Mpad, int K,
                                int r, int rr, int rp, bool has_e, float* __restrict__ codes,
                                float* __restrict__ cscale, __half* __restrict__ cop) {
+  griddep_wait();  // launched as a dependent of the codes GEMM
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (gw >= Mpad * K) return;
   const int m = gw / K, z = gw - m * K;
@@ -328,12 +329,13 @@ template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
     nsplit = (int)grid.z;
   }
   const int warps = w.Mpad * h->K;
-  k_codes_finish<<<ceil_div(warps * 32, 256), 256, 0, s>>>(
-      part, nsplit, w.M, w.Mpad, h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes),
-      wsp<float>(c, w.off_cscale), wsp<__half>(c, w.off_cop));
+  cudaError_t le = launch_dep(
+      k_codes_finish, dim3(ceil_div(warps * 32, 256)), dim3(256), 0, s, part, nsplit, w.M, w.Mpad,
+      h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes), wsp<float>(c, w.off_cscale),
+      wsp<__half>(c, w.off_cop));
   debug_kernel("k_codes_finish", s);
   count_launches(1);
-  return cudaGetLastError();
+  return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 cudaError_t launch_prior(const StepCtx& c) {

@@ -886,6 +886,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   // every CTA's barriers exist before any multicast copy or commit reaches them
   if (PAIR || P.cs > 1) cluster_sync_all();
   const uint32_t tmem = *tmem_slot;
+  griddep_wait();  // the set-up above overlaps the end of the previous kernel
 
   if (warp >= 4) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
@@ -1011,6 +1012,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  griddep_wait();  // the set-up above overlaps the end of the previous kernel
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1368,14 +1370,18 @@ static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUte
   if (P.n_tiles <= 0) return cudaSuccess;
   if (!PAIR && P.cs == 1) {
     const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
-    k_tc_pass<false><<<grid, D_THREADS, DCfg<false>::SMEM, s>>>(a, b, ca, cb, P);
+    e = launch_dep(k_tc_pass<false>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a, b, ca,
+                   cb, P);
   } else {
     const int ncl = std::min(P.n_tiles, max_clusters<PAIR>(P.cs));
-    cudaLaunchAttribute at[1];
+    cudaLaunchAttribute at[2];
     cudaLaunchConfig_t cfg = cluster_config(ncl * P.cs, P.cs, DCfg<PAIR>::SMEM, s, at);
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
     e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR>, a, b, ca, cb, P);
-    if (e != cudaSuccess) return e;
   }
+  if (e != cudaSuccess) return e;
   debug_kernel("k_tc_pass", s);
   count_launches(1);
   count_tc_launch();
@@ -1606,7 +1612,9 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
     attr = true;
   }
   const int grid = P.n_tiles < tc::num_sms() ? P.n_tiles : tc::num_sms();
-  tc::k_tc_verify<<<grid, tc::NUM_THREADS, tc::VSMEM, c.stream>>>(mca, mcb, mxs, mxt, P);
+  cudaError_t le = launch_dep(tc::k_tc_verify, dim3(grid), dim3(tc::NUM_THREADS), tc::VSMEM,
+                              c.stream, mca, mcb, mxs, mxt, P);
+  if (le != cudaSuccess) return le;
   debug_kernel("k_tc_verify", c.stream);
   count_launches(1);
   count_tc_launch();
