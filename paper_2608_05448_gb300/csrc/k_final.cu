@@ -344,24 +344,28 @@ __global__ void __launch_bounds__(DT_NT)
   __shared__ FF sL[32];
   const int m = blockIdx.x, tid = threadIdx.x;
   const int n = m / B, i = m - n * B;
+  // the sampled branch and the draw's uniform do not depend on the merge below
+  const int z = zhat[n];
+  const float u = decision_uniform(seed, 1u, rnd[n], (uint32_t)n, (uint32_t)(pos[n] + i));
   if (tid < K) {
+    float4 q[LSE_SPLIT];
+#pragma unroll
+    for (int sp = 0; sp < LSE_SPLIT; ++sp) q[sp] = lsep[((size_t)sp * M + m) * K + tid];
     float mx = -INFINITY;
-    for (int sp = 0; sp < LSE_SPLIT; ++sp) mx = fmaxf(mx, lsep[((size_t)sp * M + m) * K + tid].x);
+#pragma unroll
+    for (int sp = 0; sp < LSE_SPLIT; ++sp) mx = fmaxf(mx, q[sp].x);
     FF S{0.f, 0.f};
     if (mx != -INFINITY)
-      for (int sp = 0; sp < LSE_SPLIT; ++sp) {
-        const float4 q = lsep[((size_t)sp * M + m) * K + tid];
-        S = ff_add(S, ff_mulf(FF{q.y, q.z}, exp2f(q.x - mx)));
-      }
+#pragma unroll
+      for (int sp = 0; sp < LSE_SPLIT; ++sp)
+        S = ff_add(S, ff_mulf(FF{q[sp].y, q[sp].z}, exp2f(q[sp].x - mx)));
     const FF L = (mx == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
                                                    : ff_add(FF{mx, 0.f}, ff_log2(S));
     sL[tid] = L;
     lse2[(size_t)m * K + tid] = ff_st(L);
   }
   __syncthreads();
-  const int z = zhat[n];
   const FF L = sL[z];
-  const float u = decision_uniform(seed, 1u, rnd[n], (uint32_t)n, (uint32_t)(pos[n] + i));
   const float* cm = codes + (size_t)m * K * rr;
   const float* srow = stash + (size_t)m * V;
   const DraftTileMass tm{partd + (size_t)z * Mpad + m, (size_t)K * Mpad, L};
