@@ -34,8 +34,13 @@ constexpr int STAGE_A = BM * BK * 2;   // 16 KB
 constexpr int STAGE_B = BN * BK * 2;   // 16 KB
 constexpr int STAGE_BYTES = STAGE_A + STAGE_B;
 constexpr int KMAX = 16;           // components supported by the tensor-core path
-constexpr int NUM_EPI_WARPS = 8;
-constexpr int NUM_THREADS = 32 * (2 + NUM_EPI_WARPS);
+// verify pass: warp 0 TMA, warp 1 MMA (warps 2-3 idle), warps 4-19 the
+// epilogue, four per SM sub-partition with 32 columns each; warpgroup 0 gives
+// registers to the epilogue warpgroups (56 + 4 x 104 <= 5 x 96 per thread)
+constexpr int NUM_EPI_WARPS = 16;
+constexpr int NUM_THREADS = 32 * (4 + NUM_EPI_WARPS);
+constexpr int VREG = 96, VREG_LO = 56, VREG_HI = 104;
+static_assert(4 * VREG_LO + 16 * VREG_HI <= 20 * VREG, "register split must fit the launch pool");
 constexpr uint32_t TMEM_COLS = 512;
 
 enum Mode { MODE_PREP = 0, MODE_DRAFT = 1 };
@@ -932,7 +937,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
 constexpr int VSTAGES = 3;
 constexpr int XS_BYTES = BM * BN * 4;   // stash tile: 4 boxes [128 rows][32 fp32], SW128
 constexpr int XT_BYTES = BM * BN * 2;   // target tile: 2 boxes [128 rows][64 bf16], SW128
-constexpr size_t VSMEM = (size_t)VSTAGES * STAGE_BYTES + XS_BYTES + XT_BYTES + 2 * BM * 8 + 256 + 1024;
+constexpr size_t VSMEM = (size_t)VSTAGES * STAGE_BYTES + XS_BYTES + XT_BYTES + 4 * BM * 8 + 256 + 1024;
 struct VParams {
   int n_mt, n_vt, n_tiles, ncs, K, rp, zps, M, V, Mpad, B, Bt;
   int use_x;
@@ -963,8 +968,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   unsigned char* stage_base = smem;
   unsigned char* xs = smem + VSTAGES * STAGE_BYTES;  // stash tile
   unsigned char* xt = xs + XS_BYTES;                 // target tile
-  float2* red = reinterpret_cast<float2*>(xt + XT_BYTES);   // [2][BM]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xt + XT_BYTES + 2 * BM * 8);
+  float2* red = reinterpret_cast<float2*>(xt + XT_BYTES);   // [4][BM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xt + XT_BYTES + 4 * BM * 8);
   uint64_t* full = bars;
   uint64_t* empty = bars + VSTAGES;
   uint64_t* sfull = bars + 2 * VSTAGES;  // [2] TMEM slot ready
@@ -973,7 +978,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint64_t* redw = sfull + 5;
   uint64_t* redm = sfull + 6;
   uint64_t* xfull = sfull + 7;           // stash and target tile landed
-  uint64_t* xempty = sfull + 8;          // stash and target tile read (8 epilogue warps)
+  uint64_t* xempty = sfull + 8;          // stash and target tile read (16 epilogue warps)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -1014,106 +1019,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem = *tmem_slot;
   griddep_wait();  // the set-up above overlaps the end of the previous kernel
 
-  if (warp == 0) {
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
-      bool ok = true;
-      bool x_issued = false;
-      uint32_t x_phase = 0;
-      for (int slot = 0; slot < my_tiles && ok; ++slot) {
-        int mt, vt;
-        vtile_of(P, slot, &mt, &vt);
-        for (int c = 0; c < P.ncs; ++c) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 11)) { ok = false; break; }
-          unsigned char* sa = stage_base + stage * STAGE_BYTES;
-          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sa, &tm_ca, &full[stage], c * BK, mt * BM);
-          tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, vt * BN);
-          issued_mask |= 1u << stage;
-          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
-        }
-        if (ok && P.use_x) {
-          // this tile's stash rows and target rows, once the epilogue has read the previous ones
-          if (!mbar_wait(xempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) { ok = false; break; }
-          mbar_arrive_expect_tx(xfull, XS_BYTES + XT_BYTES);
-#pragma unroll
-          for (int b = 0; b < 4; ++b)
-            tma_load_2d(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM);
-          const int n0 = (mt * BM) / P.B;
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-            tma_load_3d(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0);
-          x_issued = true;
-          x_phase = (uint32_t)slot & 1u;
-        }
-      }
-      for (int s = 0; s < VSTAGES; ++s)
-        if (issued_mask & (1u << s)) {
-          const uint64_t t0 = globaltimer();
-          while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
-                 (globaltimer() - t0) < 2000000000ull) {
-          }
-        }
-      if (x_issued) {
-        const uint64_t t0 = globaltimer();
-        while (!mbar_try_wait(xfull, x_phase) && (globaltimer() - t0) < 2000000000ull) {
-        }
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t id_corr = idesc_f16(false, BN);
-      int stage = 0;
-      uint32_t phase = 0, guse0 = 0u, guse1 = 0u;
-      bool ok = true;
-      for (int slot = 0; slot < my_tiles && ok; ++slot) {
-        int c = 0;  // next stage of this tile
-        for (int g = 0; g < ngroups && ok; ++g) {
-          const int gs = g & 1;
-          const uint32_t use = gs ? guse1 : guse0;
-          if (!mbar_wait(&sempty[gs], (use & 1u) ^ 1u, ctl, 12)) { ok = false; break; }
-          tc_fence_after();
-          const int z0 = 2 * g, z1 = min(P.K, z0 + 2);
-          // stages holding components z0 .. z1-1
-          while (ok && c < P.ncs && c * P.zps < z1) {
-            if (!mbar_wait(&full[stage], phase, ctl, 13)) { ok = false; break; }
-            tc_fence_after();
-            const uint32_t sa = smem_u32(stage_base + stage * STAGE_BYTES);
-            const uint32_t sb = sa + STAGE_A;
-            for (int zz = 0; zz < P.zps; ++zz) {
-              const int z = c * P.zps + zz;
-              if (z >= z1) break;
-              const uint32_t col = tmem + (uint32_t)(gs * 2 * BN + (z - z0) * BN);
-              const int o = zz * 2 * P.rp;
-              int first = 1;
-              for (int kk = 0; kk < P.rp; kk += 16) {
-                const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
-                umma(col, sdesc(sa + hi), sdesc(sb + hi), id_corr, first ? 0u : 1u);
-                umma(col, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
-                umma(col, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
-                first = 0;
-              }
-            }
-            umma_commit(&empty[stage]);
-            if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
-            ++c;
-          }
-          if (!ok) break;
-          umma_commit(&sfull[gs]);
-          if (gs) ++guse1; else ++guse0;
-        }
-      }
-      umma_commit(done);
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
-      }
-    }
-  } else {
-    const int ew = warp - 2;
+  if (warp >= 4) {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(VREG_HI));
+    const int ew = warp - 4;
     const int q = warp & 3;
-    const int half = ew >> 2;
+    const int cq = ew >> 2;  // column quarter of the tile
     const int row = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint32_t guse0 = 0u, guse1 = 0u;
@@ -1122,13 +1032,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       vtile_of(P, slot, &mt, &vt);
       const int m = mt * BM + row;
       const bool mok = m < P.M;
-      const int v0 = vt * BN + half * 64;
+      const int v0 = vt * BN + cq * 32;
       // per-row constants: B0 here, (k2 / scale, log2 w - L + B0) per component below
       const float B0f = mok ? P.vb0[m] : 0.f;
       const float2* vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
-      float acc[64];
+      float acc[32];
 #pragma unroll
-      for (int j = 0; j < 64; ++j) acc[j] = 0.f;
+      for (int j = 0; j < 32; ++j) acc[j] = 0.f;
       bool ok = true;
       for (int g = 0; g < ngroups; ++g) {
         const int gs = g & 1;
@@ -1136,25 +1046,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!mbar_wait(&sfull[gs], use & 1u, ctl, 14)) { ok = false; break; }
         if (gs) ++guse1; else ++guse0;
         tc_fence_after();
-        for (int zz = 0; zz < 2; ++zz) {
-          const int z = 2 * g + zz;
-          if (z >= P.K) break;
-          const float2 cz = mok ? vrow[z] : make_float2(0.f, -INFINITY);
-          // both 32-column chunks of this component, one wait
-          uint32_t r0[32], r1[32];
-          const uint32_t col = tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + half * 64);
-          tmem_ld32_raw(col, r0);
-          tmem_ld32_raw(col + 32, r1);
+        // this quarter's 32 columns of each component of the group; the slot
+        // is handed back once the last one is in registers
+        const int nz = min(2, P.K - 2 * g);
+        for (int zz = 0; zz < nz; ++zz) {
+          const float2 cz = mok ? vrow[2 * g + zz] : make_float2(0.f, -INFINITY);
+          uint32_t r0[32];
+          tmem_ld32_raw(tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + cq * 32), r0);
           tmem_wait_ld();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            acc[j] += ex2(fmaf(__uint_as_float(r0[j]), cz.x, cz.y));
-            acc[32 + j] += ex2(fmaf(__uint_as_float(r1[j]), cz.x, cz.y));
+          if (zz == nz - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_taken(&sempty[gs]);
           }
+#pragma unroll
+          for (int j = 0; j < 32; ++j) acc[j] += ex2(fmaf(__uint_as_float(r0[j]), cz.x, cz.y));
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_taken(&sempty[gs]);
       }
       if (!ok) break;
       // four partial sums per quantity keep the add chains short
@@ -1169,21 +1076,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         As4[j & 3] += mn;
         Rs4[j & 3] += pv - mn;
       };
-      const bool full_cols = v0 + 64 <= P.V;
+      const bool full_cols = v0 + 32 <= P.V;
       if (P.use_x) {
         // stash and target rows from shared memory (128-byte swizzle: the
-        // 16-byte chunk c of row r sits at chunk c ^ (r & 7))
+        // 16-byte chunk c of row r sits at chunk c ^ (r & 7)); this quarter
+        // is stash box cq and half (cq & 1) of target box cq >> 1
         if (!mbar_wait(xfull, (uint32_t)slot & 1u, ctl, 18)) break;
         if (mok) {
-          const unsigned char* sbase = xs + half * 2 * (XS_BYTES / 4) + row * 128;
-          const unsigned char* tbase = xt + half * (XT_BYTES / 2) + row * 128;
+          const unsigned char* sbase = xs + cq * (XS_BYTES / 4) + row * 128;
+          const unsigned char* tbase = xt + (cq >> 1) * (XT_BYTES / 2) + row * 128;
 #pragma unroll
-          for (int cc = 0; cc < 8; ++cc) {
-            const int sb = cc >> 2;                  // stash box (32 columns)
-            const int c0 = ((cc & 3) * 2) ^ (row & 7), c1 = ((cc & 3) * 2 + 1) ^ (row & 7);
-            const float4 s0 = *reinterpret_cast<const float4*>(sbase + sb * (XS_BYTES / 4) + c0 * 16);
-            const float4 s1 = *reinterpret_cast<const float4*>(sbase + sb * (XS_BYTES / 4) + c1 * 16);
-            const uint4 t8 = *reinterpret_cast<const uint4*>(tbase + ((cc ^ (row & 7)) * 16));
+          for (int k = 0; k < 4; ++k) {
+            const int c0 = (2 * k) ^ (row & 7), c1 = (2 * k + 1) ^ (row & 7);
+            const float4 s0 = *reinterpret_cast<const float4*>(sbase + c0 * 16);
+            const float4 s1 = *reinterpret_cast<const float4*>(sbase + c1 * 16);
+            const uint4 t8 =
+                *reinterpret_cast<const uint4*>(tbase + ((((cq & 1) * 4 + k) ^ (row & 7)) * 16));
             const __nv_bfloat162* tp = reinterpret_cast<const __nv_bfloat162*>(&t8);
             const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
             float tv[8];
@@ -1195,11 +1103,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (full_cols) {
 #pragma unroll
-              for (int u = 0; u < 8; ++u) accumulate(cc * 8 + u, sv[u], tv[u]);
+              for (int u = 0; u < 8; ++u) accumulate(k * 8 + u, sv[u], tv[u]);
             } else {
 #pragma unroll
               for (int u = 0; u < 8; ++u)
-                if (v0 + cc * 8 + u < P.V) accumulate(cc * 8 + u, sv[u], tv[u]);
+                if (v0 + k * 8 + u < P.V) accumulate(k * 8 + u, sv[u], tv[u]);
             }
           }
         }
@@ -1209,25 +1117,121 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const float* srow = P.stash + (size_t)m * P.V + v0;
         const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
 #pragma unroll
-        for (int cc = 0; cc < 8; ++cc)
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const int v = v0 + cc * 8 + u;
-            if (v < P.V) accumulate(cc * 8 + u, srow[cc * 8 + u], __bfloat162float(trow[cc * 8 + u]));
-          }
+        for (int u = 0; u < 32; ++u)
+          if (v0 + u < P.V) accumulate(u, srow[u], __bfloat162float(trow[u]));
       }
       const float As = (As4[0] + As4[1]) + (As4[2] + As4[3]);
       const float Rs = (Rs4[0] + Rs4[1]) + (Rs4[2] + Rs4[3]);
-      // the other column half of this row, then one record per (tile, row)
+      // the other column quarters of this row, then one record per (tile, row)
       if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 15)) break;
-      red[half * BM + row] = make_float2(As, Rs);
+      red[cq * BM + row] = make_float2(As, Rs);
       mbar_arrive(redw);
       if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 16)) break;
-      if (half == 0) {
-        const float2 o = red[BM + row];
-        P.partv[(size_t)vt * P.Mpad + m] = make_float2(As + o.x, Rs + o.y);
+      if (cq == 0) {
+        const float2 o1 = red[BM + row], o2 = red[2 * BM + row], o3 = red[3 * BM + row];
+        P.partv[(size_t)vt * P.Mpad + m] =
+            make_float2((As + o1.x) + (o2.x + o3.x), (Rs + o1.y) + (o2.y + o3.y));
       }
       mbar_arrive(redm);
+    }
+  } else {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(VREG_LO));
+    if (warp == 0) {
+      if (lane == 0) {
+        int stage = 0;
+        uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
+        bool ok = true;
+        bool x_issued = false;
+        uint32_t x_phase = 0;
+        for (int slot = 0; slot < my_tiles && ok; ++slot) {
+          int mt, vt;
+          vtile_of(P, slot, &mt, &vt);
+          for (int c = 0; c < P.ncs; ++c) {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 11)) { ok = false; break; }
+            unsigned char* sa = stage_base + stage * STAGE_BYTES;
+            mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+            tma_load_2d(sa, &tm_ca, &full[stage], c * BK, mt * BM);
+            tma_load_2d(sa + STAGE_A, &tm_cb, &full[stage], c * BK, vt * BN);
+            issued_mask |= 1u << stage;
+            issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+            if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
+          }
+          if (ok && P.use_x) {
+            // this tile's stash rows and target rows, once the epilogue has read the previous ones
+            if (!mbar_wait(xempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) { ok = false; break; }
+            mbar_arrive_expect_tx(xfull, XS_BYTES + XT_BYTES);
+  #pragma unroll
+            for (int b = 0; b < 4; ++b)
+              tma_load_2d(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM);
+            const int n0 = (mt * BM) / P.B;
+  #pragma unroll
+            for (int h = 0; h < 2; ++h)
+              tma_load_3d(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0);
+            x_issued = true;
+            x_phase = (uint32_t)slot & 1u;
+          }
+        }
+        for (int s = 0; s < VSTAGES; ++s)
+          if (issued_mask & (1u << s)) {
+            const uint64_t t0 = globaltimer();
+            while (!mbar_try_wait(&full[s], (issued_phase >> s) & 1u) &&
+                   (globaltimer() - t0) < 2000000000ull) {
+            }
+          }
+        if (x_issued) {
+          const uint64_t t0 = globaltimer();
+          while (!mbar_try_wait(xfull, x_phase) && (globaltimer() - t0) < 2000000000ull) {
+          }
+        }
+      }
+    } else if (warp == 1) {
+      if (lane == 0) {
+        const uint32_t id_corr = idesc_f16(false, BN);
+        int stage = 0;
+        uint32_t phase = 0, guse0 = 0u, guse1 = 0u;
+        bool ok = true;
+        for (int slot = 0; slot < my_tiles && ok; ++slot) {
+          int c = 0;  // next stage of this tile
+          for (int g = 0; g < ngroups && ok; ++g) {
+            const int gs = g & 1;
+            const uint32_t use = gs ? guse1 : guse0;
+            if (!mbar_wait(&sempty[gs], (use & 1u) ^ 1u, ctl, 12)) { ok = false; break; }
+            tc_fence_after();
+            const int z0 = 2 * g, z1 = min(P.K, z0 + 2);
+            // stages holding components z0 .. z1-1
+            while (ok && c < P.ncs && c * P.zps < z1) {
+              if (!mbar_wait(&full[stage], phase, ctl, 13)) { ok = false; break; }
+              tc_fence_after();
+              const uint32_t sa = smem_u32(stage_base + stage * STAGE_BYTES);
+              const uint32_t sb = sa + STAGE_A;
+              for (int zz = 0; zz < P.zps; ++zz) {
+                const int z = c * P.zps + zz;
+                if (z >= z1) break;
+                const uint32_t col = tmem + (uint32_t)(gs * 2 * BN + (z - z0) * BN);
+                const int o = zz * 2 * P.rp;
+                int first = 1;
+                for (int kk = 0; kk < P.rp; kk += 16) {
+                  const uint32_t hi = (uint32_t)(o + kk) * 2u, lo = (uint32_t)(o + P.rp + kk) * 2u;
+                  umma(col, sdesc(sa + hi), sdesc(sb + hi), id_corr, first ? 0u : 1u);
+                  umma(col, sdesc(sa + hi), sdesc(sb + lo), id_corr, 1u);
+                  umma(col, sdesc(sa + lo), sdesc(sb + hi), id_corr, 1u);
+                  first = 0;
+                }
+              }
+              umma_commit(&empty[stage]);
+              if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
+              ++c;
+            }
+            if (!ok) break;
+            umma_commit(&sfull[gs]);
+            if (gs) ++guse1; else ++guse0;
+          }
+        }
+        umma_commit(done);
+        const uint64_t t0 = globaltimer();
+        while (!mbar_try_wait(done, 0u) && (globaltimer() - t0) < 2000000000ull) {
+        }
+      }
     }
   }
 
@@ -1603,14 +1607,22 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   P.partv = wsp<float2>(c, w.off_partv);
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(tc::k_tc_verify,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)tc::VSMEM);
+  // the register split (setmaxnreg) assumes exactly VREG registers per thread
+  static int state = -1;
+  if (state < 0) {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, tc::k_tc_verify);
     if (e != cudaSuccess) return e;
-    attr = true;
+    if (fa.numRegs != tc::VREG) {
+      state = 0;
+    } else {
+      e = cudaFuncSetAttribute(tc::k_tc_verify, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)tc::VSMEM);
+      if (e != cudaSuccess) return e;
+      state = 1;
+    }
   }
+  if (state != 1) return cudaErrorInvalidKernelImage;
   const int grid = P.n_tiles < tc::num_sms() ? P.n_tiles : tc::num_sms();
   cudaError_t le = launch_dep(tc::k_tc_verify, dim3(grid), dim3(tc::NUM_THREADS), tc::VSMEM,
                               c.stream, mca, mcb, mxs, mxt, P);
