@@ -722,13 +722,15 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       continue;
     }
 
-    // stash W h + b (32-byte stores: each fills one sector of this thread's row)
+    // stash W h + b (32-byte stores: each fills one sector of this thread's
+    // row; streaming, since the verify pass reads it back only after the
+    // whole head has gone through L2)
     if (m < P.M) {
       float* srow = P.stash + (size_t)m * P.V + v0;
       if (v0 + DCOLS <= P.V && (P.V & 7) == 0) {
 #pragma unroll
         for (int j = 0; j < DCOLS; j += 8)
-          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(srow + j),
+          asm volatile("st.global.cs.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(srow + j),
                        "f"(bk[j]), "f"(bk[j + 1]), "f"(bk[j + 2]), "f"(bk[j + 3]), "f"(bk[j + 4]),
                        "f"(bk[j + 5]), "f"(bk[j + 6]), "f"(bk[j + 7])
                        : "memory");
