@@ -123,6 +123,29 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// copies of data read once (evict-first L2 policy)
+__device__ __forceinline__ uint64_t l2_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ void tma_load_2d_once(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                                 int x, int y, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_once(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                                 int x, int y, int z, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z), "l"(pol)
+      : "memory");
+}
+
 // the same copy written to the same shared-memory offset of every CTA in
 // cta_mask (this GPU's own memory only); each destination's mbarrier at the
 // same offset receives the complete_tx bytes
@@ -1162,13 +1185,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             // this tile's stash rows and target rows, once the epilogue has read the previous ones
             if (!mbar_wait(xempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) { ok = false; break; }
             mbar_arrive_expect_tx(xfull, XS_BYTES + XT_BYTES);
-  #pragma unroll
+            // the stash and target rows are read once: evict-first in L2
+            const uint64_t pol = l2_evict_first();
+#pragma unroll
             for (int b = 0; b < 4; ++b)
-              tma_load_2d(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM);
+              tma_load_2d_once(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM,
+                               pol);
             const int n0 = (mt * BM) / P.B;
-  #pragma unroll
+#pragma unroll
             for (int h = 0; h < 2; ++h)
-              tma_load_3d(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0);
+              tma_load_3d_once(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0,
+                               pol);
             x_issued = true;
             x_phase = (uint32_t)slot & 1u;
           }
