@@ -383,28 +383,47 @@ def main():
     value = N * world * K_steps / (ms / 1e3)
 
     # end to end through the public API with host buffers (pinned), per step:
-    # H2D of hidden + target, the call, D2H of the per-sequence results
+    # H2D of hidden + target, the call, D2H of the per-sequence results.  The
+    # inputs of step k+1 are copied on a second stream while step k runs
+    # (two device buffers); every copy and every call lie between e0 and e1.
     e2e_steps = args.e2e_steps or K_steps
     h_host = blk["hidden"].cpu().pin_memory()
     t_host = blk["target"].cpu().pin_memory()
     res_host = {k: torch.empty_like(vouts[0][k], device="cpu").pin_memory()
                 for k in ("accepted", "n_emitted", "emitted", "exp_len")}
-    h_dev, t_dev = torch.empty_like(blk["hidden"]), torch.empty_like(blk["target"])
+    h_dev = [torch.empty_like(blk["hidden"]) for _ in range(2)]
+    t_dev = [torch.empty_like(blk["target"]) for _ in range(2)]
     h2d = h_host.numel() * h_host.element_size() + t_host.numel() * t_host.element_size()
     d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    main = torch.cuda.current_stream()
+    cstream = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in range(2)]
+    freed = [torch.cuda.Event() for _ in range(2)]
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
+    e0.record(main)
+
+    def copy_in(b, after=None):
+        cstream.wait_event(after if after is not None else e0)
+        with torch.cuda.stream(cstream):
+            h_dev[b].copy_(h_host, non_blocking=True)
+            t_dev[b].copy_(t_host, non_blocking=True)
+            copied[b].record(cstream)
+
+    copy_in(0)
     for k in range(e2e_steps):
-        h_dev.copy_(h_host, non_blocking=True)
-        t_dev.copy_(t_host, non_blocking=True)
-        dblast_draft_and_verify(head, ws, h_dev, pos, rnd, args.T, cfg["Z_T"], seed, t_dev,
+        b = k & 1
+        if k + 1 < e2e_steps:
+            copy_in(b ^ 1, freed[b ^ 1] if k >= 1 else None)
+        main.wait_event(copied[b])
+        dblast_draft_and_verify(head, ws, h_dev[b], pos, rnd, args.T, cfg["Z_T"], seed, t_dev[b],
                                 blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0])
+        freed[b].record(main)
         for kk, v in res_host.items():
             v.copy_(vouts[0][kk], non_blocking=True)
-    e1.record()
+    e1.record(main)
     torch.cuda.synchronize()
     ems = e0.elapsed_time(e1)
     if world > 1:
@@ -458,7 +477,8 @@ def main():
             "prep_ms": prep_ms,
             "gpu_launches": int(st["kernel_launches"]),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "overlap": "inputs of step k+1 copied on a second stream during step k"},
             "clocks": clk,
         }
         if world == 1 and not args.no_cpu_baseline:
