@@ -33,8 +33,10 @@ def _case(cfg, T, Z_T, seed, impl, seqs=None, round_idx=0, device="cuda"):
 
 
 def _skip_unsupported(cfg, impl):
-    if impl == "tcgen05" and not (cfg["dtype"] == "bf16" and cfg["H"] % 64 == 0):
-        pytest.skip("tensor-core path needs bf16 and H % 64 == 0")
+    rr = cfg["r"] + (1 if cfg.get("expander_bias") else 0)
+    if impl == "tcgen05" and not (cfg["dtype"] == "bf16" and cfg["H"] % 64 == 0
+                                  and cfg["K"] <= 16 and rr <= 32):
+        pytest.skip("tensor-core path needs bf16, H % 64 == 0, K <= 16 and r (+1) <= 32")
 
 
 @pytest.mark.parametrize("T,Z_T", [(1.0, 1.0), (0.6, 1.0), (1.5, 0.0)])
@@ -56,9 +58,15 @@ SMALL = {
     "f32_b32": dict(base="tiny", V=777, H=32, K=2, r=2, B=32, N=2, bonus=False),
     # many components, rank 32
     "k16_r32": dict(base="sweep_k16", V=3000, H=128, B=4, N=4),
+    # the interface limits: B = 32 (one M tile, and two for the CTA pair) and
+    # K = 32 with r = 64 (CUDA-core path only)
+    "b32_bf16": dict(base="qwen3_8b_b32", V=2000, H=128, K=4, r=8, B=32, N=3),
+    "b32_pair": dict(base="qwen3_8b_b32", V=2000, H=128, K=4, r=8, B=32, N=8),
+    "k32_r64": dict(base="qwen3_8b_b32", V=1500, H=64, K=32, r=64, B=4, N=2),
 }
 SMALL_T = {"ragged_e": (0.8, 1.0), "zt0": (1.0, 0.0), "k1_b1": (1.5, 1.0),
-           "f32_b32": (1.0, 0.7), "k16_r32": (0.7, 1.0)}
+           "f32_b32": (1.0, 0.7), "k16_r32": (0.7, 1.0), "b32_bf16": (1.0, 1.0),
+           "b32_pair": (0.9, 1.0), "k32_r64": (1.2, 1.0)}
 
 
 @pytest.mark.parametrize("impl", IMPLS)
