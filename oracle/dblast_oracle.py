@@ -32,6 +32,11 @@ Definitions followed (section / equation of the paper):
   (Algorithm 1; Appendix A, "Distributional correctness").
 * Expected accepted length of the drafted block, sum_i prod_{j<=i} A_j
   (Eq. 3), and the overlap alpha_i = sum_v min(p_i(v), q(v|x_<i)).
+* Greedy-branch mode (Sec. 3.1, "Drafter sampling during inference"; App. A,
+  "Greedy-Branch Proposal", "Prefix-Marginalized Conditional" and its
+  verification algorithm): z-hat from the prior, the block is the greedy
+  branch x-hat_{.,z-hat}, and verification uses the sparse conditional
+  q_greedy over the consistent branches C_i.
 
 Readings where the paper is silent (the same list is kept in the design notes):
 the drafter's token distributions use the same temperature T as the target;
@@ -265,6 +270,167 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 lse_target=lse_t, ties=ties, first_tie=first_tie)
 
 
+# --------------------------------------------------------- greedy-branch mode
+# Decisions whose top-two logit gap is below this are "ties" of the greedy
+# argmax: the CUDA path forms the logits in fp32 (errors up to ~1e-5 at the
+# Qwen3 shapes), so only gaps below 1e-4 may resolve differently.
+GREEDY_TIE_TOL = 1e-4
+
+
+def greedy_branch_tokens(logits):
+    """x-hat_{i,z} = argmax_v q_i(v|y,z) for every position and branch.
+
+    Sec. 3.1 ("Drafter sampling during inference"), Eq. greedy-branch-proposal:
+    the greedy token of branch z at position i.  The argmax of q_i(.|y,z) =
+    softmax(l_{i,z}/T) is the argmax of the logits l_{i,z} for any T > 0; ties
+    go to the lowest index.  logits: [B, K, V].  Returns (xhat [B, K] int64,
+    gap [B, K]: the largest logit minus the second largest, +inf if V = 1).
+    """
+    xhat = np.argmax(logits, axis=-1)
+    if logits.shape[-1] < 2:
+        return xhat, np.full(xhat.shape, np.inf)
+    top2 = np.sort(logits, axis=-1)[..., -2:]
+    return xhat, top2[..., 1] - top2[..., 0]
+
+
+def consistent_branches(xhat, tokens):
+    """Membership of the consistent-branch sets C_i(x_<i).
+
+    App. A ("Prefix-Marginalized Conditional"): C_i = {z : x-hat_{j,z} = x_j
+    for every j < i}.  xhat: [B, K]; tokens: [B].  Returns bool [B, K] with
+    row i marking C_i (row 0 is every branch).
+    """
+    B, K = xhat.shape
+    C = np.ones((B, K), dtype=bool)
+    for i in range(1, B):
+        C[i] = C[i - 1] & (xhat[i - 1] == tokens[i - 1])
+    return C
+
+
+def greedy_conditional(pi, xhat, C, V):
+    """The sparse proposal conditional q_greedy(v|y,x_<i) at every position.
+
+    App. A: pi-tilde_{i,z} = pi_z 1{z in C_i} / sum_{z' in C_i} pi_{z'} and
+    q_greedy(v|y,x_<i) = sum_{z in C_i} pi-tilde_{i,z} 1{v = x-hat_{i,z}}
+    (Eq. appendix-greedy-conditional).  pi: [K]; xhat, C: [B, K].  Returns
+    (q [B, V] dense, with at most K non-zero entries per row; pit [B, K]).
+    A prefix that no branch drafts (zero proposal mass) gets all-zero rows.
+    """
+    B, K = xhat.shape
+    q = np.zeros((B, V), dtype=np.float64)
+    pit = np.zeros((B, K), dtype=np.float64)
+    for i in range(B):
+        wz = np.where(C[i], pi, 0.0)
+        tot = np.sum(wz)
+        if not tot > 0.0:
+            continue
+        pit[i] = wz / tot
+        for z in range(K):
+            if C[i, z]:
+                q[i, xhat[i, z]] += pit[i, z]
+    return q, pit
+
+
+def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
+                                     seed, n, pos, round_):
+    """One greedy-branch draft+verify step for sequence n (Algorithm 1 of App. A).
+
+    Same inputs and outputs as draft_and_verify_sequence.  The category is
+    drawn from the tempered prior as in the stochastic mode; the block is the
+    greedy branch x_i = x-hat_{i,z-hat}; verification uses q_greedy (App. A)
+    for the acceptance min(1, p/q) and the residual [p - q_greedy]_+, then the
+    usual bonus token.  Extra outputs: xhat [B, K] (all K greedy branches),
+    consistent [B, K] (C_i), gap [B, K] (top-two logit gaps).  "logw" holds
+    log pi-tilde (the category posterior given the greedy prefix, -inf
+    outside C_i).  A greedy argmax of a branch in C_i whose gap is below
+    GREEDY_TIE_TOL is recorded as a tie of kind "greedy".
+    """
+    B, H = h.shape
+    W = head["W"]
+    V = W.shape[0]
+    a = h[0] if anchor is None else anchor
+    ties = []
+
+    # prior and latent category, as in the stochastic mode
+    ell, pi = category_prior(head["Wp"], head["bp"], a, Z_T)
+    u0 = decision_uniform(seed, STREAM_PRIOR, round_, n, pos)
+    zhat, m0 = inverse_cdf(pi, u0)
+    if Z_T != 0 and m0 < TIE_TOL:
+        ties.append(("zhat", -1, m0))
+
+    # all K greedy branches and the selected block
+    hz = branch_hidden(h, head["U"], head["Vf"], head["e"])
+    logits = component_logits(W, hz, head["vbias"])          # [B, K, V]
+    xhat, gap = greedy_branch_tokens(logits)
+    tokens = xhat[:, zhat].astype(np.int64)
+    C = consistent_branches(xhat, tokens)
+    for i in range(B):
+        for z in range(xhat.shape[1]):
+            if C[i, z] and gap[i, z] < GREEDY_TIE_TOL:
+                ties.append(("greedy", i, float(gap[i, z])))
+
+    # the proposal conditional used by verification
+    q, pit = greedy_conditional(pi, xhat, C, V)
+    q_tok = q[np.arange(B), tokens]
+    with np.errstate(divide="ignore"):
+        logw = np.log(pit)
+
+    # target distributions p_i = softmax(t_i / T)
+    st = target / T
+    lse_t = logsumexp(st, axis=-1)
+    p = np.exp(st - lse_t[:, None])
+    p_tok = p[np.arange(B), tokens]
+    alpha = np.sum(np.minimum(p[:B], q), axis=-1)
+    ratio = p_tok / q_tok
+    accept_prob = np.minimum(1.0, ratio)
+
+    L = B
+    for i in range(B):
+        u2 = decision_uniform(seed, STREAM_ACCEPT, round_, n, pos + i)
+        m2 = abs(u2 * q_tok[i] - p_tok[i]) / q_tok[i]
+        if m2 < TIE_TOL:
+            ties.append(("accept", i, m2))
+        if not (u2 < ratio[i]):
+            L = i
+            break
+
+    emitted = list(int(x) for x in tokens[:L])
+    extra = -1
+    if L < B:
+        u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + L)
+        res = np.maximum(p[L] - q[L], 0.0)
+        mass = float(np.sum(res))
+        if mass > 0.0:
+            extra, m3 = inverse_cdf(res, u3)
+        else:
+            extra, m3 = inverse_cdf(p[L], u3)
+        if mass < TIE_TOL:
+            ties.append(("residual_mass", L, mass))
+        if m3 < TIE_TOL:
+            ties.append(("residual", L, m3))
+    elif has_bonus:
+        u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + B)
+        extra, m3 = inverse_cdf(p[B], u3)
+        if m3 < TIE_TOL:
+            ties.append(("bonus", B, m3))
+    if extra >= 0:
+        emitted.append(int(extra))
+
+    exp_len = float(np.sum(np.cumprod(accept_prob)))
+    alpha_len = float(np.sum(np.cumprod(alpha)))
+
+    first_tie = B + 1
+    for kind, i, _ in ties:
+        first_tie = min(first_tie, 0 if kind == "zhat" else i)
+
+    return dict(pi=pi, ell=ell, zhat=int(zhat), tokens=tokens, xhat=xhat,
+                consistent=C, gap=gap, logw=logw, q_tok=q_tok, p_tok=p_tok,
+                accept_prob=accept_prob, alpha=alpha, accepted=L,
+                emitted=emitted, n_emitted=len(emitted), exp_len=exp_len,
+                alpha_len=alpha_len, lse_target=lse_t, ties=ties,
+                first_tie=first_tie)
+
+
 def prepare_head(head):
     """fp64 copies of the small head tensors; W is left as given (chunked later)."""
     out = {k: f64(head.get(k)) for k in ("U", "Vf", "e", "Wp", "bp", "vbias")}
@@ -273,13 +439,17 @@ def prepare_head(head):
 
 
 def draft_and_verify(head, hidden, anchor, target, has_bonus, T, Z_T, seed,
-                     pos, round_, seqs=None):
+                     pos, round_, seqs=None, mode="soft"):
     """Run the step for the sequences in ``seqs`` (default: all).
 
     hidden: [N, B, H]; anchor: [N, H] or None; target: [N, B+has_bonus, V];
-    pos: [N] int; round_: [N] int.  Returns a list of per-sequence dicts
-    (see draft_and_verify_sequence) in the order of ``seqs``.
+    pos: [N] int; round_: [N] int; mode "soft" (tokens drawn from the branch
+    distributions) or "greedy" (greedy branches, App. A).  Returns a list of
+    per-sequence dicts (see draft_and_verify_sequence and
+    greedy_draft_and_verify_sequence) in the order of ``seqs``.
     """
+    step = {"soft": draft_and_verify_sequence,
+            "greedy": greedy_draft_and_verify_sequence}[mode]
     hd = prepare_head(head)
     N = hidden.shape[0]
     seqs = range(N) if seqs is None else seqs
@@ -288,7 +458,7 @@ def draft_and_verify(head, hidden, anchor, target, has_bonus, T, Z_T, seed,
         h = f64(hidden[n])
         a = None if anchor is None else f64(anchor[n])
         t = f64(target[n])
-        out.append(draft_and_verify_sequence(
+        out.append(step(
             hd, h, a, t, bool(has_bonus), float(T), float(Z_T), int(seed),
             int(n), int(pos[n]), int(round_[n])))
     return out
