@@ -104,7 +104,7 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
-def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0):
+def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft"):
     """Time the fp64 oracle, as it stands, on one sequence of the workload."""
     import torch
     from oracle import dblast_oracle as orc
@@ -117,15 +117,15 @@ def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0):
     while True:
         orc.draft_and_verify(head_cpu, blk_cpu["hidden"], None, blk_cpu["target"],
                              blk_cpu["has_bonus"], T, Z_T, 0, pos.numpy(), rnd.numpy(),
-                             seqs=[n_done % cfg["N"]])
+                             seqs=[n_done % cfg["N"]], mode=mode)
         n_done += 1
         el = time.perf_counter() - t0
         if el > budget_s / 3 or n_done >= 4:
             break
     return {"value": n_done / el, "unit": UNIT, "cores": _cpu_threads(),
             "kind": "oracle",
-            "sample": "%d sequence(s) of the %s workload (one block each), fp64 direct form"
-                      % (n_done, cfg["name"])}
+            "sample": "%d sequence(s) of the %s workload (one block each, %s mode), fp64 "
+                      "direct form" % (n_done, cfg["name"], mode)}
 
 
 def _cpu_threads():
@@ -154,7 +154,7 @@ def run_reference(args, cfg, rank):
     def step(i):
         o = orc.draft_and_verify(head, blk["hidden"], None, blk["target"], blk["has_bonus"],
                                  args.T, 1.0, i, pos.numpy(), rnd.numpy(),
-                                 seqs=[i % cfg["N"]])
+                                 seqs=[i % cfg["N"]], mode=args.mode)
         return o[0]["accepted"]
 
     for i in range(args.warmup):
@@ -170,7 +170,7 @@ def run_reference(args, cfg, rank):
             "dtype": "f64", "data": "synthetic",
             "config": {"workload": cfg["name"], "N": cfg["N"], "B": cfg["B"], "K": cfg["K"],
                        "r": cfg["r"], "H": cfg["H"], "V": cfg["V"], "T": args.T,
-                       "sample": "one sequence (block) per step"},
+                       "mode": args.mode, "sample": "one sequence (block) per step"},
             "accepted_tokens_per_s": L_total / el,
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": _cpu_threads(),
                              "kind": "oracle",
@@ -287,6 +287,9 @@ def main():
     ap.add_argument("--config", default="qwen3_8b_b32")
     ap.add_argument("--T", type=float, default=1.0)
     ap.add_argument("--kernels", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--mode", default="soft", choices=["soft", "greedy"],
+                    help="draft tokens sampled from the z-hat branch (soft) or the "
+                         "greedy-branch decoder")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--sweep", action="store_true",
@@ -339,14 +342,14 @@ def main():
     ws = Workspace(head, N, B, blk["has_bonus"])
     pos, rnd = synth.initial_state(cfg, dev)
     K_steps = args.steps
-    dout = alloc_draft_out(N, B, cfg["K"], dev)
+    dout = alloc_draft_out(N, B, cfg["K"], dev, args.mode)
     vouts = [alloc_verify_out(N, B, blk["has_bonus"], dev) for _ in range(K_steps)]
     seed = 1234 + 7919 * rank
 
     def step(vout):
         dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, args.T, cfg["Z_T"], seed,
                                 blk["target"], blk["has_bonus"], impl=args.kernels,
-                                dout=dout, vout=vout)
+                                dout=dout, vout=vout, mode=args.mode)
 
     for _ in range(args.warmup):
         step(vouts[0])
@@ -419,7 +422,8 @@ def main():
             copy_in(b ^ 1, freed[b ^ 1] if k >= 1 else None)
         main.wait_event(copied[b])
         dblast_draft_and_verify(head, ws, h_dev[b], pos, rnd, args.T, cfg["Z_T"], seed, t_dev[b],
-                                blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0])
+                                blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0],
+                                mode=args.mode)
         freed[b].record(main)
         for kk, v in res_host.items():
             v.copy_(vouts[0][kk], non_blocking=True)
@@ -442,6 +446,8 @@ def main():
         # DRAM bytes per draft-pass launch from the committed ncu summary, used
         # only while the kernel source is the one that was profiled
         tr_path = os.path.join(ROOT, "profiles", "draft_pass_%s_traffic.json" % cfg["name"])
+        if args.mode == "greedy":
+            tr_path = os.path.join(ROOT, "profiles", "draft_pass_greedy_%s_traffic.json" % cfg["name"])
         if os.path.exists(tr_path) and st["tc_launches"] > 0 and not args.n_seqs:
             d = json.load(open(tr_path))
             src = os.path.join(ROOT, d.get("source", ""))
@@ -456,7 +462,7 @@ def main():
             "dtype": "bf16" if cfg["dtype"] == "bf16" else "f32", "data": "synthetic",
             "config": {"workload": cfg["name"], "N": N, "B": B, "K": cfg["K"], "r": cfg["r"],
                        "H": cfg["H"], "V": cfg["V"], "T": args.T, "Z_T": cfg["Z_T"],
-                       "sigma": cfg["sigma"],
+                       "sigma": cfg["sigma"], "mode": args.mode,
                        "kernels": "tcgen05" if st["tc_launches"] > 0 else "simt",
                        "parallelism": "replicas" if world > 1 else "single",
                        "l2": "no flush: inputs larger than L2 (W %.2f GB, target %.0f MB)" % (
@@ -482,7 +488,8 @@ def main():
             "clocks": clk,
         }
         if world == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline(cfg, head_t, blk, args.T, cfg["Z_T"])
+            line["cpu_baseline"] = cpu_baseline(cfg, head_t, blk, args.T, cfg["Z_T"],
+                                                mode=args.mode)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

@@ -18,6 +18,17 @@
  *             alpha_i = sum_v min(p_i(v), q(v|x_<i)) and the expected accepted
  *             length of the drafted block sum_i prod_{j<=i} A_j (Eq. 3).
  *
+ * Greedy-branch mode (args->mode = DBLAST_MODE_GREEDY; Sec. 3.1, "Drafter
+ * sampling during inference"; Appendix A, "Greedy-Branch Proposal",
+ * "Prefix-Marginalized Conditional" and its verification algorithm): every
+ * branch is decoded greedily, x-hat_{i,z} = argmax_v l_{i,z,v} (lowest index
+ * on ties), the block is the z-hat branch, and verification uses the sparse
+ * conditional q_greedy(v|x_<i) = sum_{z in C_i} pi~_{i,z} 1{v = x-hat_{i,z}}
+ * over the consistent branches C_i = {z : x-hat_{j,z} = x_j for all j < i},
+ * pi~ = pi restricted to C_i and renormalised.  Acceptance, residual
+ * [p - q_greedy]_+, bonus, alpha and Eq. 3 are as above.  Stream 1 is not
+ * used in this mode.
+ *
  * The expander is rank r: h_{i,z} = h_i + U_z (V_z^T h_i) + e_z.
  * Temperatures: q_i(.|z) = softmax(l_{i,z}/T), p_i = softmax(t_i/T),
  * prior softmax(l/Z_T) (Z_T = 0 selects the highest-prior category).
@@ -69,6 +80,11 @@ typedef enum { DBLAST_BF16 = 0, DBLAST_F32 = 1 } dblast_dtype;
  * bf16 inputs with H % 64 == 0, else SIMT (plain CUDA cores, any shape). */
 typedef enum { DBLAST_IMPL_AUTO = 0, DBLAST_IMPL_SIMT = 1, DBLAST_IMPL_TCGEN05 = 2 } dblast_impl;
 
+/* Drafting mode.  SOFT: draft tokens sampled from the z-hat branch
+ * distribution, dense mixture conditional (Eq. dep-next-token).  GREEDY: the
+ * greedy-branch decoder of Appendix A (see the top of this file). */
+typedef enum { DBLAST_MODE_SOFT = 0, DBLAST_MODE_GREEDY = 1 } dblast_mode;
+
 /* Drafter head (Sec. 3.1, Architecture; Table 1 with a rank-r expander).
  * W is the reused vocabulary head, U/Vf the expander factors, e its optional
  * bias, Wp/bp the category-prior head, vbias an optional vocabulary bias.
@@ -101,6 +117,7 @@ typedef struct {
   int64_t* pos;          /* [N] in/out */
   uint32_t* round;       /* [N] in/out */
   dblast_impl impl;
+  dblast_mode mode;      /* SOFT (0) or GREEDY (1); draft and verify of one block use the same */
 } dblast_block_args;
 
 /* Draft outputs.  Every pointer may be NULL (not written). */
@@ -108,9 +125,13 @@ typedef struct {
   int32_t* z_hat;  /* [N]       latent category */
   float* pi;       /* [N, K]    tempered prior softmax(l/Z_T) */
   int32_t* tokens; /* [N, B]    draft block */
-  float* lse;      /* [N, B, K] natural log of sum_v exp(l_{i,z,v}/T) */
-  float* logw;     /* [N, B, K] natural log of the posterior q(z|y,x_<i) */
-  float* q_tok;    /* [N, B]    q(x_i|y,x_<i) */
+  float* lse;      /* [N, B, K] natural log of sum_v exp(l_{i,z,v}/T) (SOFT mode; not written
+                                in GREEDY mode) */
+  float* logw;     /* [N, B, K] natural log of the posterior q(z|y,x_<i); GREEDY: log pi~_{i,z},
+                                -inf for z outside C_i */
+  float* q_tok;    /* [N, B]    q(x_i|y,x_<i) (GREEDY: q_greedy) */
+  int32_t* branch_tokens; /* [N, B, K] GREEDY: x-hat_{i,z} of every branch (not written in SOFT
+                                mode) */
 } dblast_draft_out;
 
 /* Verify inputs/outputs.  target is required; every output may be NULL. */
@@ -127,7 +148,8 @@ typedef struct {
   float* exp_len;       /* [N]        sum_i prod_{j<=i} A_j (Eq. 3) */
   float* alpha_len;     /* [N]        sum_i prod_{j<=i} alpha_j */
   uint32_t* tie_flags;  /* [N]        bit0 z-hat, bit1 draft, bit2 accept, bit3 residual/bonus,
-                                       bit4 residual mass < 1e-6: a decision within 1e-6 of its threshold */
+                                       bit4 residual mass < 1e-6: a decision within 1e-6 of its threshold
+                                       (GREEDY mode leaves bit1 clear: argmax decisions are not flagged) */
 } dblast_verify_out;
 
 /* Bytes of the prep buffer for this head (depends on V, K, r, e != NULL). */

@@ -17,6 +17,7 @@ STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "unsupported",
                 3: "workspace", 4: "cuda", 5: "timeout", 6: "no device"}
 DTYPES = {torch.bfloat16: 0, torch.float32: 1}
 IMPLS = {"auto": 0, "simt": 1, "tcgen05": 2}
+MODES = {"soft": 0, "greedy": 1}
 
 TIE_ZHAT, TIE_DRAFT, TIE_ACCEPT, TIE_RESID, TIE_RMASS = 1, 2, 4, 8, 16
 
@@ -43,12 +44,13 @@ class CBlockArgs(ctypes.Structure):
                 ("temperature", ctypes.c_float), ("z_temperature", ctypes.c_float),
                 ("seed", ctypes.c_uint64), ("hidden", ctypes.c_void_p),
                 ("anchor", ctypes.c_void_p), ("pos", ctypes.c_void_p),
-                ("round", ctypes.c_void_p), ("impl", ctypes.c_int)]
+                ("round", ctypes.c_void_p), ("impl", ctypes.c_int),
+                ("mode", ctypes.c_int)]
 
 
 class CDraftOut(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
-                ("z_hat", "pi", "tokens", "lse", "logw", "q_tok")]
+                ("z_hat", "pi", "tokens", "lse", "logw", "q_tok", "branch_tokens")]
 
 
 class CStats(ctypes.Structure):
@@ -203,7 +205,7 @@ class Workspace:
         return ctypes.c_void_p(self.buf.data_ptr())
 
 
-def _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl):
+def _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode="soft"):
     N, B, H = hidden.shape
     if H != head.H:
         raise ValueError("hidden size mismatch")
@@ -214,17 +216,23 @@ def _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl):
         raise ValueError("round must be int32/uint32")
     _cuda_contig(round_, "round")
     return CBlockArgs(N, B, float(T), float(Z_T), int(seed) & ((1 << 64) - 1),
-                      _ptr(hidden), _ptr(anchor), _ptr(pos), _ptr(round_), IMPLS[impl])
+                      _ptr(hidden), _ptr(anchor), _ptr(pos), _ptr(round_), IMPLS[impl],
+                      MODES[mode])
 
 
-def alloc_draft_out(N, B, K, device):
+def alloc_draft_out(N, B, K, device, mode="soft"):
+    """Draft outputs; "lse" only in soft mode, "branch_tokens" only in greedy mode."""
     f, i = torch.float32, torch.int32
-    return dict(z_hat=torch.empty(N, dtype=i, device=device),
-                pi=torch.empty(N, K, dtype=f, device=device),
-                tokens=torch.empty(N, B, dtype=i, device=device),
-                lse=torch.empty(N, B, K, dtype=f, device=device),
-                logw=torch.empty(N, B, K, dtype=f, device=device),
-                q_tok=torch.empty(N, B, dtype=f, device=device))
+    out = dict(z_hat=torch.empty(N, dtype=i, device=device),
+               pi=torch.empty(N, K, dtype=f, device=device),
+               tokens=torch.empty(N, B, dtype=i, device=device),
+               logw=torch.empty(N, B, K, dtype=f, device=device),
+               q_tok=torch.empty(N, B, dtype=f, device=device))
+    if mode == "greedy":
+        out["branch_tokens"] = torch.empty(N, B, K, dtype=i, device=device)
+    else:
+        out["lse"] = torch.empty(N, B, K, dtype=f, device=device)
+    return out
 
 
 def alloc_verify_out(N, B, has_bonus, device):
@@ -255,10 +263,10 @@ def _verify_struct(target, has_bonus, v):
 
 
 def dblast_draft_block(head, ws, hidden, pos, round_, T, Z_T, seed, anchor=None,
-                       impl="auto", out=None):
-    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl)
+                       impl="auto", out=None, mode="soft"):
+    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode)
     N, B, _ = hidden.shape
-    out = out if out is not None else alloc_draft_out(N, B, head.K, hidden.device)
+    out = out if out is not None else alloc_draft_out(N, B, head.K, hidden.device, mode)
     d = _draft_struct(out)
     _check(lib().dblast_draft_block(ctypes.byref(head.c), ctypes.byref(args),
                                     ctypes.byref(d), ws.ptr, ws.nbytes, _stream()),
@@ -267,8 +275,8 @@ def dblast_draft_block(head, ws, hidden, pos, round_, T, Z_T, seed, anchor=None,
 
 
 def dblast_verify_block(head, ws, hidden, pos, round_, T, Z_T, seed, target, has_bonus,
-                        anchor=None, impl="auto", out=None):
-    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl)
+                        anchor=None, impl="auto", out=None, mode="soft"):
+    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode)
     N, B, _ = hidden.shape
     _cuda_contig(target, "target", head.dtype)
     if tuple(target.shape) != (N, B + int(has_bonus), head.V):
@@ -282,14 +290,16 @@ def dblast_verify_block(head, ws, hidden, pos, round_, T, Z_T, seed, target, has
 
 
 def dblast_draft_and_verify(head, ws, hidden, pos, round_, T, Z_T, seed, target,
-                            has_bonus, anchor=None, impl="auto", dout=None, vout=None):
-    """One fused draft+verify step; returns (draft_out, verify_out) dicts."""
-    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl)
+                            has_bonus, anchor=None, impl="auto", dout=None, vout=None,
+                            mode="soft"):
+    """One fused draft+verify step; returns (draft_out, verify_out) dicts.
+    mode: "soft" (sampled draft tokens) or "greedy" (greedy branches)."""
+    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode)
     N, B, _ = hidden.shape
     _cuda_contig(target, "target", head.dtype)
     if tuple(target.shape) != (N, B + int(has_bonus), head.V):
         raise ValueError("target must be [N, B + has_bonus, V]")
-    dout = dout if dout is not None else alloc_draft_out(N, B, head.K, hidden.device)
+    dout = dout if dout is not None else alloc_draft_out(N, B, head.K, hidden.device, mode)
     vout = vout if vout is not None else alloc_verify_out(N, B, has_bonus, hidden.device)
     d = _draft_struct(dout)
     v = _verify_struct(target, has_bonus, vout)

@@ -142,6 +142,8 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_partv = take((size_t)w.nt * w.Mpad * sizeof(float2));
   w.off_av = take((size_t)AV_SPLIT * w.M * sizeof(float4));
   w.off_ties = take((size_t)N * sizeof(uint32_t));
+  w.off_xhat = take((size_t)w.M * K * sizeof(int32_t));
+  w.off_cmask = take((size_t)w.M * sizeof(uint32_t));
   w.total = o;
   return w;
 }
@@ -181,6 +183,7 @@ static dblast_status check_args(const dblast_head* h, const dblast_block_args* a
   if (a->impl == DBLAST_IMPL_TCGEN05 && !tc_supported(h)) return DBLAST_ERR_UNSUPPORTED;
   if (a->impl != DBLAST_IMPL_AUTO && a->impl != DBLAST_IMPL_SIMT && a->impl != DBLAST_IMPL_TCGEN05)
     return DBLAST_ERR_INVALID_ARG;
+  if (a->mode != DBLAST_MODE_SOFT && a->mode != DBLAST_MODE_GREEDY) return DBLAST_ERR_INVALID_ARG;
   return DBLAST_OK;
 }
 
@@ -205,6 +208,7 @@ static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, 
   c->stream = reinterpret_cast<cudaStream_t>(stream);
   c->k2 = LOG2E / a->temperature;
   c->tc = use_tc(h, a);
+  c->greedy = a->mode == DBLAST_MODE_GREEDY;
   c->target = nullptr;
   c->Bt = a->B + (has_bonus ? 1 : 0);
   return DBLAST_OK;
@@ -248,11 +252,16 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
     pass_event_end(0, c.stream);
     e = dbg(e, "draft_pass", c.stream);
   }
-  if (e == cudaSuccess) e = dbg(launch_draft_finalize(c, out), "draft_finalize", c.stream);
+  if (e == cudaSuccess)
+    e = dbg(c.greedy ? launch_greedy_draft_finalize(c, out) : launch_draft_finalize(c, out),
+            "draft_finalize", c.stream);
   return cuda_status(e);
 }
 
 static cudaError_t verify_passes(const StepCtx& c, dblast_verify_out* out) {
+  // greedy-branch mode has no vocabulary-wide verify pass: q_greedy has at
+  // most K atoms, so one kernel reads p at them and draws the residual
+  if (c.greedy) return dbg(launch_greedy_verify_finalize(c, out), "verify_finalize", c.stream);
   pass_event_begin(1, c.stream);
   cudaError_t e = c.tc ? launch_verify_pass_tc(c) : launch_verify_pass_simt(c);
   pass_event_end(1, c.stream);
@@ -333,7 +342,8 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[2], 0);
   if (e == cudaSuccess) e = launch_target_stats(side, vout);
   if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
-  if (e == cudaSuccess) e = launch_draft_finalize(c, dout);
+  if (e == cudaSuccess)
+    e = c.greedy ? launch_greedy_draft_finalize(c, dout) : launch_draft_finalize(c, dout);
   // join 2
   if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[3], 0);
   if (e == cudaSuccess) e = verify_passes(c, vout);

@@ -46,13 +46,15 @@ struct PrepLayout {
 //   lsep float4 [LSE_SPLIT,M,K] | lse2, lq2, w2 ff [M,K] | qtok f32 [M] | tok i32 [M]
 //   vcz float2 [M,K] | vb0 f32 [M] | partt float2 [nt,Rt] | lt2 ff [Rt]
 //   partv float2 [nt,Mpad] | av float4 [AV_SPLIT,M] | ties u32 [N]
+//   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
+//   token and the consistent-branch set C_i as a bit mask over z)
 constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
 constexpr int AV_SPLIT = 8;   // partial sums of the verify records per row
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
       off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
-      off_partt, off_lt2, off_partv, off_av, off_ties, total;
+      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, total;
 };
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
@@ -230,6 +232,7 @@ struct StepCtx {
   float k2;  // log2(e) / T
   bool has_e;
   bool tc;   // tensor-core passes
+  bool greedy;  // greedy-branch mode (App. A) instead of sampled draft tokens
   const void* target;  // verify only: [N, Bt, V]
   int Bt;              // target rows per sequence (B + has_bonus)
 };
@@ -282,5 +285,7 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* out)
 cudaError_t launch_target_stats(const StepCtx& c, const dblast_verify_out* out);
 cudaError_t launch_verify_pass_simt(const StepCtx& c);
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
+cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* out);
+cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
 
 }  // namespace dblast

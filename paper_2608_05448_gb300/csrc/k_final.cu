@@ -108,10 +108,11 @@ struct FindOut {
 
 // Smallest token whose cumulative mass (in vocabulary order) exceeds `target`.
 // tmass(t): mass of tile t; emass(v): mass of token v (floats); `total` scales
-// the decision margin.
+// the decision margin.  With `frac`, target.hi is a fraction u of the summed
+// tile masses, and that sum scales the margin.
 template <int NT, typename TM, typename EM>
 __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF target,
-                              float total, FindShared<NT>& fs) {
+                              float total, FindShared<NT>& fs, bool frac = false) {
   static_assert(NT >= TILE_V, "one thread per token of a tile");
   const int tid = threadIdx.x, lane = tid & 31;
   const int chunk = ceil_div(nt, NT);
@@ -136,6 +137,10 @@ __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF 
     }
   }
   const BlockScan sc = block_scan_ff<NT>(loc, fs.d);
+  if (frac) {
+    target = ff_mulf(sc.total, target.hi);
+    total = ff_f(sc.total);
+  }
   const int first = block_min_i<NT>(ff_gt(sc.incl, target) ? tid : NT, fs.i);
   const int lastall = block_max_i<NT>(lastp, fs.i);
   if (first < NT) {
@@ -931,6 +936,385 @@ static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out*
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {
   return c.head->dtype == DBLAST_F32 ? verify_final_typed<float>(c, o)
                                      : verify_final_typed<__nv_bfloat16>(c, o);
+}
+
+// ---------------------------------------------------------------- greedy-branch mode
+// Sec. 3.1 ("Drafter sampling during inference") and App. A: the draft pass
+// leaves per-tile records partd[t][z][m] = (max logit, token) of every
+// branch; these kernels take x-hat_{i,z}, the block x_i = x-hat_{i,z-hat}, the
+// consistent-branch sets C_i and q_greedy (Eq. appendix-greedy-conditional),
+// and verify with it.  q_greedy has at most K atoms per position, so p is
+// needed only at those tokens, plus the target tile records for the residual
+// and bonus draws.
+__device__ __forceinline__ void arg_keep(float& mx, int& ix, float v, int i) {
+  if (v > mx || (v == mx && i < ix)) {
+    mx = v;
+    ix = i;
+  }
+}
+
+// Partial argmax of the draft records: block (row group of 32, z, split), lane
+// = row, warps and splits interleave over the tiles (as k_draft_lse).
+// lsep[sp][m][z] = (max, token bits, 0, 0).
+__global__ void __launch_bounds__(LSE_WARPS * 32)
+    k_greedy_argmax(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
+                    float4* __restrict__ lsep) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ float smx[LSE_WARPS][32];
+  __shared__ int six[LSE_WARPS][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int m = blockIdx.x * 32 + lane, z = blockIdx.y, sp = blockIdx.z;
+  const int step = LSE_WARPS * LSE_SPLIT;
+  float mx = -INFINITY;
+  int ix = 0x7fffffff;
+  if (m < M) {
+    const float2* p = partd + (size_t)z * Mpad + m;
+    const size_t st = (size_t)K * Mpad;
+    int t = sp * LSE_WARPS + warp;
+    for (; t + 3 * step < nt; t += 4 * step) {
+      const float2 q0 = p[(size_t)t * st], q1 = p[(size_t)(t + step) * st];
+      const float2 q2 = p[(size_t)(t + 2 * step) * st], q3 = p[(size_t)(t + 3 * step) * st];
+      arg_keep(mx, ix, q0.x, __float_as_int(q0.y));
+      arg_keep(mx, ix, q1.x, __float_as_int(q1.y));
+      arg_keep(mx, ix, q2.x, __float_as_int(q2.y));
+      arg_keep(mx, ix, q3.x, __float_as_int(q3.y));
+    }
+    for (; t < nt; t += step) {
+      const float2 q = p[(size_t)t * st];
+      arg_keep(mx, ix, q.x, __float_as_int(q.y));
+    }
+  }
+  smx[warp][lane] = mx;
+  six[warp][lane] = ix;
+  __syncthreads();
+  if (warp == 0 && m < M) {
+#pragma unroll
+    for (int w = 1; w < LSE_WARPS; ++w) arg_keep(mx, ix, smx[w][lane], six[w][lane]);
+    lsep[((size_t)sp * M + m) * K + z] = make_float4(mx, __int_as_float(ix), 0.f, 0.f);
+  }
+}
+
+// One block per sequence, thread t = (i, z) with i = t / K: x-hat_{i,z}, the
+// block, C_i (bit z of cmask[m]: branch z drafted x_j at every j < i),
+// pi~_{i,z} and q_greedy(x_i|x_<i), and the user-visible draft outputs.
+__global__ void __launch_bounds__(1024)
+    k_greedy_draft(const float4* __restrict__ lsep, const float* __restrict__ log2pi,
+                   const int32_t* __restrict__ zhat, int B, int K, int M, int V,
+                   int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
+                   float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
+                   dblast_draft_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ int X[1024];
+  __shared__ int tokS[32];
+  __shared__ uint32_t eqS[32], cmS[32];
+  __shared__ float piS[32], sumS[32];
+  const int n = blockIdx.x, t = threadIdx.x;
+  const int i = t / K, z = t - i * K;
+  const bool ok = i < B;
+  const size_t m = (size_t)n * B + (ok ? i : 0);
+  if (ok) {
+    float mx = -INFINITY;
+    int ix = 0x7fffffff;
+#pragma unroll
+    for (int sp = 0; sp < LSE_SPLIT; ++sp) {
+      const float4 q = lsep[((size_t)sp * M + m) * K + z];
+      arg_keep(mx, ix, q.x, __float_as_int(q.y));
+    }
+    ix = min(max(ix, 0), V - 1);  // every logit NaN: not a token, keep the index valid
+    X[t] = ix;
+    xhat_ws[m * K + z] = ix;
+    if (out.branch_tokens) out.branch_tokens[m * K + z] = ix;
+  }
+  if (t < K) piS[t] = exp2f(log2pi[n * K + t]);  // -inf (Z_T = 0) gives 0
+  if (t < 32) eqS[t] = 0u;
+  __syncthreads();
+  const int zh = zhat[n];
+  if (t < B) tokS[t] = X[t * K + zh];
+  __syncthreads();
+  if (ok && X[t] == tokS[i]) atomicOr(&eqS[i], 1u << z);
+  __syncthreads();
+  if (t < B) {  // C_t = branches that drafted x_j at every j < t
+    uint32_t c = (K >= 32) ? 0xffffffffu : ((1u << K) - 1u);
+    for (int j = 0; j < t; ++j) c &= eqS[j];
+    cmS[t] = c;
+    float S = 0.f, Q = 0.f;
+    for (int k = 0; k < K; ++k) {
+      if ((c >> k) & 1u) {
+        S += piS[k];
+        if ((eqS[t] >> k) & 1u) Q += piS[k];
+      }
+    }
+    sumS[t] = S;
+    const size_t mt = (size_t)n * B + t;
+    const float qt = S > 0.f ? Q / S : 0.f;
+    tok_ws[mt] = tokS[t];
+    qtok_ws[mt] = qt;
+    cmask_ws[mt] = c;
+    if (out.tokens) out.tokens[mt] = tokS[t];
+    if (out.q_tok) out.q_tok[mt] = qt;
+  }
+  __syncthreads();
+  if (ok && out.logw) {
+    const bool in = (cmS[i] >> z) & 1u;
+    const float w = (in && sumS[i] > 0.f) ? piS[z] / sumS[i] : 0.f;
+    out.logw[m * K + z] = w > 0.f ? logf(w) : -INFINITY;
+  }
+  if (t < K && out.pi) out.pi[n * K + t] = piS[t];
+  if (t == 0 && out.z_hat) out.z_hat[n] = zh;
+}
+
+cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* outp) {
+  const WsLayout& w = c.wl;
+  const int K = c.head->K;
+  cudaError_t le =
+      launch_dep(k_greedy_argmax, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
+                 c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+  debug_kernel("k_greedy_argmax", c.stream);
+  dblast_draft_out out{};
+  if (outp) out = *outp;
+  const int pt = ceil_div(w.B * K, 32) * 32;
+  if (le == cudaSuccess) le = launch_dep(k_greedy_draft, dim3(w.N), dim3(pt), 0, c.stream,
+      wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_log2pi), wsp<int32_t>(c, w.off_zhat), w.B,
+      K, w.M, w.V, wsp<int32_t>(c, w.off_xhat), wsp<int32_t>(c, w.off_tok),
+      wsp<float>(c, w.off_qtok), wsp<uint32_t>(c, w.off_cmask), out);
+  debug_kernel("k_greedy_draft", c.stream);
+  count_launches(2);
+  return le != cudaSuccess ? le : cudaGetLastError();
+}
+
+// Residual masses of the greedy conditional at the rejected row: the target
+// tile records, except for tiles holding an atom, whose masses are summed
+// token by token in shared memory (no cancellation of p_tile - q).
+struct GreedyResidTileMass {
+  TargetTileMass pt;
+  const int* atile;   // tile of atom k, -1 if an earlier atom has the same tile
+  const float* amass; // token-level residual mass of that tile
+  int na;
+  __device__ float operator()(int t) const {
+    for (int k = 0; k < na; ++k)
+      if (atile[k] == t) return amass[k];
+    return pt(t);
+  }
+};
+template <typename Tin> struct GreedyResidTokenMass {  // [p(v) - q_greedy(v)]_+
+  TargetTokenProb<Tin> p;
+  const int* atok;
+  const float* aq;
+  int na;
+  __device__ float operator()(int v) const {
+    float q = 0.f;
+    for (int k = 0; k < na; ++k)
+      if (atok[k] == v) q += aq[k];
+    return fmaxf(p(v) - q, 0.f);
+  }
+};
+
+// One block per sequence: p at the atoms of q_greedy, acceptance (stream 2),
+// alpha_i = sum over atoms of min(p, q), residual or bonus draw (stream 3),
+// expected lengths, emitted tokens, state update.
+template <typename Tin>
+__global__ void __launch_bounds__(VF_NT)
+    k_greedy_verify(const Tin* __restrict__ target, const float* __restrict__ log2pi,
+                    const int32_t* __restrict__ xhat, const uint32_t* __restrict__ cmask,
+                    const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
+                    const float2* __restrict__ partt, const int32_t* __restrict__ tok,
+                    const uint32_t* __restrict__ ties_draft, int V, int K, int B, int Bt, int nt,
+                    int Rt, float k2, uint64_t seed, int64_t* __restrict__ pos,
+                    uint32_t* __restrict__ rnd, dblast_verify_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ FindShared<VF_NT> fs;
+  __shared__ int X[1024];
+  __shared__ float piS[32];
+  __shared__ int atok[32], atile[32];
+  __shared__ float aq[32], amass[32];
+  __shared__ int sL, sna;
+  __shared__ uint32_t sties;
+  __shared__ float sR;
+  const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t p0 = pos[n];
+  const uint32_t rd = rnd[n];
+  for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[(size_t)n * B * K + j];
+  if (tid < K) piS[tid] = exp2f(log2pi[n * K + tid]);
+  __syncthreads();
+  if (tid < 32) {
+    uint32_t ties = ties_draft[n];
+    float A = 0.f, alpha = 0.f, ptok = 0.f, qtok = 1.f, u2 = 0.f;
+    bool acc_ok = false;
+    uint32_t c = 0u;
+    float S = 0.f;
+    FF Lt{0.f, 0.f};
+    const Tin* trow = target;
+    if (lane < B) {
+      const int m = n * B + lane;
+      const int x = min(max(tok[m], 0), V - 1);
+      Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
+      trow = target + ((size_t)n * Bt + lane) * V;
+      const float tx = ldf(trow + x);
+      ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
+      qtok = qtok_ws[m];
+      const float ratio = ptok / qtok;
+      A = fminf(1.f, ratio);
+      // alpha_i: one term min(p(a), q(a)) per distinct token a of the branches in C_i
+      c = cmask[m];
+      for (int k = 0; k < K; ++k)
+        if ((c >> k) & 1u) S += piS[k];
+      FF al{0.f, 0.f};
+      for (int k = 0; k < K; ++k) {
+        if (!((c >> k) & 1u)) continue;
+        const int a = X[lane * K + k];
+        bool first = true;
+        float qa = 0.f;
+        for (int k2i = 0; k2i < K; ++k2i) {
+          if (!((c >> k2i) & 1u) || X[lane * K + k2i] != a) continue;
+          if (k2i < k) first = false;
+          qa += piS[k2i];
+        }
+        if (!first) continue;
+        const float ta = ldf(trow + a);
+        const float pa = (ta == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(ta, k2), Lt));
+        al = ff_addf(al, fminf(pa, S > 0.f ? qa / S : 0.f));
+      }
+      alpha = ff_f(al);
+      u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
+      acc_ok = u2 < ratio;
+      if (out.p_tok) out.p_tok[m] = ptok;
+      if (out.accept_prob) out.accept_prob[m] = A;
+      if (out.alpha) out.alpha[m] = alpha;
+    }
+    const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
+    const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
+    const int L = rej ? (__ffs(rej) - 1) : B;
+    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float ta = __shfl_up_sync(FULLMASK, cA, o);
+      const float tl = __shfl_up_sync(FULLMASK, cAl, o);
+      if (lane >= o) {
+        cA *= ta;
+        cAl *= tl;
+      }
+    }
+    FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      el = ff_add(el, ff_shfl_xor(el, o));
+      ea = ff_add(ea, ff_shfl_xor(ea, o));
+    }
+    // the atoms of the rejected row: token, q_greedy, the tile (first atom of a tile only)
+    if (L < B && lane == L) {
+      int na = 0;
+      for (int k = 0; k < K; ++k) {
+        if (!((c >> k) & 1u)) continue;
+        const int a = X[L * K + k];
+        int j = 0;
+        while (j < na && atok[j] != a) ++j;
+        if (j == na) {
+          atok[na] = a;
+          aq[na] = 0.f;
+          ++na;
+        }
+        aq[j] += S > 0.f ? piS[k] / S : 0.f;
+      }
+      for (int j = 0; j < na; ++j) {
+        const int tj = atok[j] / TILE_V;
+        bool first = true;
+        for (int j2 = 0; j2 < j; ++j2) first = first && (atok[j2] / TILE_V != tj);
+        atile[j] = first ? tj : -1;
+      }
+      sna = na;
+      sR = 1.f - alpha;  // residual mass, for the tie flag
+    }
+    if (lane == 0) {
+      if (out.exp_len) out.exp_len[n] = ff_f(el);
+      if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
+      sL = L;
+      sties = ties;
+    }
+  }
+  __syncthreads();
+  const int L = sL;
+  int extra = -1;
+  bool tie = false;
+  uint32_t tbits = 0;
+  const int irow = (L < B) ? L : B;  // target row of the extra token
+  if ((L < B) || (Bt > B)) {
+    const float u3 = decision_uniform(seed, 3u, rd, (uint32_t)n, (uint32_t)(p0 + irow));
+    const int rl = n * (B + 1) + irow;
+    const FF Lt = ff_ld(lt2 + rl);
+    const TargetTokenProb<Tin> pv{target + ((size_t)n * Bt + irow) * V, k2, Lt};
+    const TargetTileMass ptm{partt + rl, (size_t)Rt, k2, Lt};
+    bool from_p = (L >= B);
+    if (L < B) {
+      const int na = sna;
+      const GreedyResidTokenMass<Tin> rm{pv, atok, aq, na};
+      // token-level residual mass of every tile that holds an atom, one warp per tile
+      for (int j = warp; j < na; j += VF_NT / 32) {
+        if (atile[j] < 0) continue;
+        FF sm{0.f, 0.f};
+        for (int o = lane; o < TILE_V; o += 32) {
+          const int v = atile[j] * TILE_V + o;
+          if (v < V) sm = ff_addf(sm, rm(v));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sm = ff_add(sm, ff_shfl_xor(sm, o));
+        if (lane == 0) amass[j] = ff_f(sm);
+      }
+      __syncthreads();
+      if (sR < TIE_TOL) tbits |= TIE_RMASS;
+      const FindOut f = block_find<VF_NT>(nt, V, GreedyResidTileMass{ptm, atile, amass, na}, rm,
+                                          FF{u3, 0.f}, 1.f, fs, true);
+      extra = f.x;
+      tie = f.tie;
+      if (extra < 0) {  // no positive residual mass left by rounding: draw from p
+        from_p = true;
+        tie = true;
+        tbits |= TIE_RMASS;
+      }
+    }
+    if (from_p) {
+      const FindOut f = block_find<VF_NT>(nt, V, ptm, pv, FF{u3, 0.f}, 1.f, fs);
+      extra = f.x >= 0 ? f.x : 0;
+      tie = tie || f.tie || f.x < 0;
+    }
+  }
+  if (tid == 0) {
+    const uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u);
+    const int ne = L + (extra >= 0 ? 1 : 0);
+    if (out.accepted) out.accepted[n] = L;
+    if (out.n_emitted) out.n_emitted[n] = ne;
+    if (out.tie_flags) out.tie_flags[n] = ties;
+    pos[n] = p0 + ne;
+    rnd[n] = rd + 1u;
+  }
+  if (out.emitted) {
+    for (int j = tid; j < B + 1; j += VF_NT) {
+      int val = -1;
+      if (j < L) val = tok[n * B + j];
+      else if (j == L && extra >= 0) val = extra;
+      out.emitted[(size_t)n * (B + 1) + j] = val;
+    }
+  }
+}
+
+template <typename Tin>
+static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out* o) {
+  const WsLayout& w = c.wl;
+  cudaError_t le = launch_dep(k_greedy_verify<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
+      static_cast<const Tin*>(o->target), wsp<float>(c, w.off_log2pi),
+      wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask), wsp<float>(c, w.off_qtok),
+      wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
+      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.B, c.Bt, w.nt, w.Rt, c.k2, c.args->seed,
+      c.args->pos, c.args->round, *o);
+  debug_kernel("k_greedy_verify", c.stream);
+  count_launches(1);
+  return le != cudaSuccess ? le : cudaGetLastError();
+}
+
+cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {
+  return c.head->dtype == DBLAST_F32 ? greedy_verify_typed<float>(c, o)
+                                     : greedy_verify_typed<__nv_bfloat16>(c, o);
 }
 
 }  // namespace dblast

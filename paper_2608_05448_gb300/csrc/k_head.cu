@@ -9,13 +9,19 @@ namespace dblast {
 constexpr int RB = 16;  // rows (positions) per CTA of the CUDA-core passes
 
 // ---------------------------------------------------------------------------
-// draft pass on CUDA cores: stash = W h + b; partd per (tile, z, row)
+// draft pass on CUDA cores: stash = W h + b; partd per (tile, z, row).
+// Greedy-branch mode: no stash, and the records hold (max logit, its token)
+// with ties to the lowest index (the token's bits stored in the float).
+__device__ __forceinline__ float2 arg_merge2(float2 a, float2 b) {
+  const int ia = __float_as_int(a.y), ib = __float_as_int(b.y);
+  return (b.x > a.x || (b.x == a.x && ib < ia)) ? b : a;
+}
 template <typename Tin>
 __global__ void __launch_bounds__(TILE_V)
     k_draft_simt(const Tin* __restrict__ W, const Tin* __restrict__ hid,
                  const float* __restrict__ vbias, const float* __restrict__ wu,
                  const float* __restrict__ codes, int V, int H, int K, int rr, int M, int Mpad,
-                 float k2, float* __restrict__ stash, float2* __restrict__ partd) {
+                 float k2, bool greedy, float* __restrict__ stash, float2* __restrict__ partd) {
   extern __shared__ float smem[];
   float* hs = smem;                    // [RB][64]
   float* cs = smem + RB * 64;          // [K*rr]
@@ -48,18 +54,28 @@ __global__ void __launch_bounds__(TILE_V)
     const int m = m0 + r;
     if (m >= M) break;  // uniform over the block
     const float base = acc[r] + b;
-    if (vok) stash[(size_t)m * V + v] = base;
+    if (vok && !greedy) stash[(size_t)m * V + v] = base;
     for (int idx = tid; idx < K * rr; idx += TILE_V) cs[idx] = codes[(size_t)m * K * rr + idx];
     __syncthreads();
     for (int z = 0; z < K; ++z) {
-      float2 p = make_float2(-INFINITY, 0.f);
+      float2 p = greedy ? make_float2(-INFINITY, __int_as_float(0x7fffffff))
+                        : make_float2(-INFINITY, 0.f);
       if (vok) {
         float corr = 0.f;
         const float* wr = wu + ((size_t)v * K + z) * rr;
         for (int k = 0; k < rr; ++k) corr = fmaf(wr[k], cs[z * rr + k], corr);
-        p = make_float2((base + corr) * k2, 1.f);
+        p = greedy ? make_float2(base + corr, __int_as_float(v)) : make_float2((base + corr) * k2, 1.f);
       }
-      p = warp_lse_merge(p);
+      if (greedy) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float2 q = make_float2(__shfl_xor_sync(0xffffffffu, p.x, o),
+                                       __shfl_xor_sync(0xffffffffu, p.y, o));
+          p = arg_merge2(p, q);
+        }
+      } else {
+        p = warp_lse_merge(p);
+      }
       if (lane == 0) red[(r * K + z) * 4 + warp] = p;
     }
     __syncthreads();
@@ -68,7 +84,7 @@ __global__ void __launch_bounds__(TILE_V)
     const int r = idx / K, z = idx - r * K, m = m0 + r;
     if (m >= M) continue;
     float2 p = red[idx * 4];
-    for (int j = 1; j < 4; ++j) p = lse_merge(p, red[idx * 4 + j]);
+    for (int j = 1; j < 4; ++j) p = greedy ? arg_merge2(p, red[idx * 4 + j]) : lse_merge(p, red[idx * 4 + j]);
     partd[((size_t)t * K + z) * Mpad + m] = p;
   }
 }
@@ -81,7 +97,7 @@ template <typename Tin> static cudaError_t draft_simt_typed(const StepCtx& c) {
   k_draft_simt<Tin><<<grid, TILE_V, smem, c.stream>>>(
       static_cast<const Tin*>(h->W), static_cast<const Tin*>(c.args->hidden), h->vbias,
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), h->V, h->H, h->K, w.rr, w.M,
-      w.Mpad, c.k2, wsp<float>(c, w.off_stash), wsp<float2>(c, w.off_partd));
+      w.Mpad, c.k2, c.greedy, wsp<float>(c, w.off_stash), wsp<float2>(c, w.off_partd));
   debug_kernel("k_draft_simt", c.stream);
   count_launches(1);
   return cudaGetLastError();

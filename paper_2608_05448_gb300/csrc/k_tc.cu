@@ -43,7 +43,7 @@ constexpr int VREG = 96, VREG_LO = 56, VREG_HI = 104;
 static_assert(4 * VREG_LO + 16 * VREG_HI <= 20 * VREG, "register split must fit the launch pool");
 constexpr uint32_t TMEM_COLS = 512;
 
-enum Mode { MODE_PREP = 0, MODE_DRAFT = 1 };
+enum Mode { MODE_PREP = 0, MODE_DRAFT = 1, MODE_GREEDY = 2 };
 
 // ------------------------------------------------------------------ PTX
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -451,7 +451,7 @@ __device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
   int stage = 0;
   uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
   bool ok = true;
-  const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
+  const int nzK = (P.mode != MODE_PREP) ? P.K : 0;
   // one stage: wait until the slot is free, arm its full barrier, copy the
   // A and B boxes
   auto load = [&](const CUtensorMap* ma, const CUtensorMap* mb, int xk, int y0, int y1) {
@@ -559,7 +559,7 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
     }
   };
   bool ok = true;
-  const int nzK = (P.mode == MODE_DRAFT) ? P.K : 0;
+  const int nzK = (P.mode != MODE_PREP) ? P.K : 0;
   for (int slot = 0; slot <= my_tiles && ok; ++slot) {
     const int nbv = (slot < my_tiles) ? P.nb : 0;
     const int nzv = (slot >= 1) ? nzK : 0;
@@ -669,12 +669,79 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Epilogue: per tile, the base accumulator plus b_v becomes the stash; then
+// Greedy-branch epilogue of one tile (Sec. 3.1, "Drafter sampling during
+// inference"): for every component z, the largest logit
+// l_v = base_v + b_v + D_z / (cscale sw) of this thread's 128 columns and its
+// token (lowest index on ties) become the record (max, index) of the half
+// tile; no stash and no exponentials.  Four interleaved chains keep the
+// compare-and-select sequences independent.
+__device__ __forceinline__ void arg_keep(float& mx, int& ix, float v, int i) {
+  if (v > mx || (v == mx && i < ix)) {
+    mx = v;
+    ix = i;
+  }
+}
+template <bool PAIR>
+__device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem, int lane,
+                                                  uint32_t lane_off, int rg, int half, int slot,
+                                                  int m, int v0, int et, const float* az,
+                                                  float (&bk)[DCOLS], uint64_t* cfull,
+                                                  uint64_t* cempty, const Ctl& ctl) {
+  const bool live = v0 < P.V;
+#pragma unroll
+  for (int j = 0; j < DCOLS; ++j)
+    if (v0 + j >= P.V) bk[j] = -INFINITY;
+  const int rec = (v0 / DCOLS);
+  for (int z = 0; z < P.K; ++z) {
+    if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6)) return false;
+    tc_fence_after();
+    const float a = az[z * D_EPI + et];
+    float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
+    int i0 = 0, i1 = 1, i2 = 2, i3 = 3;
+    const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
+    uint32_t ra[32], rb[32];
+    tmem_ld32_raw(tb, ra);
+    tmem_wait_ld(ra);
+#pragma unroll
+    for (int cc = 0; cc < DCOLS / 32; ++cc) {
+      uint32_t(&cur)[32] = (cc & 1) ? rb : ra;
+      uint32_t(&nxt)[32] = (cc & 1) ? ra : rb;
+      if (cc + 1 < DCOLS / 32) tmem_ld32_raw(tb + (uint32_t)((cc + 1) * 32), nxt);
+#pragma unroll
+      for (int j = 0; j < 32; j += 4) {
+        const int c = cc * 32 + j;
+        const float x0 = fmaf(__uint_as_float(cur[j]), a, bk[c]);
+        const float x1 = fmaf(__uint_as_float(cur[j + 1]), a, bk[c + 1]);
+        const float x2 = fmaf(__uint_as_float(cur[j + 2]), a, bk[c + 2]);
+        const float x3 = fmaf(__uint_as_float(cur[j + 3]), a, bk[c + 3]);
+        // each chain sees increasing columns, so a strict compare keeps the lowest
+        if (x0 > m0) { m0 = x0; i0 = c; }
+        if (x1 > m1) { m1 = x1; i1 = c + 1; }
+        if (x2 > m2) { m2 = x2; i2 = c + 2; }
+        if (x3 > m3) { m3 = x3; i3 = c + 3; }
+      }
+      if (cc + 1 < DCOLS / 32) tmem_wait_ld(nxt);
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) {
+      if constexpr (PAIR) mbar_arrive_taken_cluster(cluster_addr(&cempty[rg], 0));
+      else mbar_arrive_taken(&cempty[rg]);
+    }
+    arg_keep(m0, i0, m1, i1);
+    arg_keep(m2, i2, m3, i3);
+    arg_keep(m0, i0, m2, i2);
+    if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(m0, __int_as_float(v0 + i0));
+  }
+  return true;
+}
+
+// Epilogue: per tile, the base accumulator plus b_v becomes the stash; then// Epilogue: per tile, the base accumulator plus b_v becomes the stash; then
 // for every component z the record (ref, sum 2^{t_v}) of this thread's 128
 // columns, t_v = D_z a_z + (base_v + b_v) k2 - ref, with ref = k2 max_v
 // (base_v + b_v) taken once per tile.  A sum outside [2^-100, 2^100] (a branch
 // offset far from the base logits) is redone against the exact maximum.
-template <bool PAIR>
+template <bool PAIR, bool GREEDY>
 __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, int warp, int lane,
                                             float* az, float* vbs, uint64_t* vbar,
                                             uint64_t* bfull, uint64_t* bempty,
@@ -698,7 +765,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     // reads of slot s, so the writes of slot s+2 cannot overtake them), and the
     // branch scales, while the main loop still runs
     const float* vb = vbs + (slot & 1) * DBN + half * DCOLS;
-    if (P.mode == MODE_DRAFT) {
+    if (P.mode != MODE_PREP) {
       for (int z = 0; z < P.K; ++z) az[z * D_EPI + et] = P.k2 / (P.cscale[(size_t)m * P.K + z] * P.sw[z]);
       const int vc = vt * DBN + et;
       vbs[(slot & 1) * DBN + et] = (P.vbias && vc < P.V) ? __ldg(P.vbias + vc) : 0.f;
@@ -720,8 +787,8 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
         if (cc + 1 < DCOLS / 32) tmem_ld32_raw(tb + (uint32_t)((cc + 1) * 32), nxt);
 #pragma unroll
         for (int j = 0; j < 32; ++j)
-          bk[cc * 32 + j] = (P.mode == MODE_DRAFT) ? __uint_as_float(cur[j]) + vb[cc * 32 + j]
-                                                   : __uint_as_float(cur[j]);
+          bk[cc * 32 + j] = (P.mode != MODE_PREP) ? __uint_as_float(cur[j]) + vb[cc * 32 + j]
+                                                  : __uint_as_float(cur[j]);
         if (cc + 1 < DCOLS / 32) tmem_wait_ld(nxt);
       }
     }
@@ -742,6 +809,13 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
           if (v < P.V) out[(size_t)v * P.prep_rows + m] = bk[j];
         }
       }
+      continue;
+    }
+
+    if constexpr (GREEDY) {
+      if (!greedy_components<PAIR>(P, tmem, lane, lane_off, rg, half, slot, m, v0, et, az, bk, cfull,
+                             cempty, ctl))
+        break;
       continue;
     }
 
@@ -846,7 +920,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
   }
 }
 
-template <bool PAIR>
+template <bool PAIR, bool GREEDY = false>
 __global__ void __launch_bounds__(D_THREADS, 1)
     k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
@@ -920,7 +994,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
 
   if (warp >= 4) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
-    draft_epilogue<PAIR>(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl,
+    draft_epilogue<PAIR, GREEDY>(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl,
                          my_tiles);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
@@ -1345,17 +1419,17 @@ static int num_sms() {
 // The register split of k_tc_pass (setmaxnreg) assumes the kernel was built
 // with exactly DREG registers per thread: with fewer, the epilogue's increase
 // could never be granted.  Such a build is refused instead of launched.
-template <bool PAIR>
+template <bool PAIR, bool GREEDY>
 static cudaError_t pass_kernel_ready() {
   static int state = -1;
   if (state < 0) {
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR, GREEDY>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != DREG) {
       state = 0;
     } else {
-      e = cudaFuncSetAttribute(k_tc_pass<PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      e = cudaFuncSetAttribute(k_tc_pass<PAIR, GREEDY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)DCfg<PAIR>::SMEM);
       if (e != cudaSuccess) return e;
       state = 1;
@@ -1381,7 +1455,7 @@ static cudaLaunchConfig_t cluster_config(int grid, int cs, size_t smem, cudaStre
 }
 
 // clusters of cs CTAs that can be resident at once (cached per form and size)
-template <bool PAIR>
+template <bool PAIR, bool GREEDY>
 static int max_clusters(int cs) {
   static int cache[5] = {0, 0, 0, 0, 0};
   if (cs < 1 || cs > 4) return 0;
@@ -1389,30 +1463,31 @@ static int max_clusters(int cs) {
     cudaLaunchAttribute at[1];
     cudaLaunchConfig_t cfg = cluster_config(cs * num_sms(), cs, DCfg<PAIR>::SMEM, 0, at);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass<PAIR>, &cfg) != cudaSuccess || n < 1) n = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass<PAIR, GREEDY>, &cfg) != cudaSuccess || n < 1)
+      n = 1;
     cache[cs] = n;
   }
   return cache[cs];
 }
 
-template <bool PAIR>
+template <bool PAIR, bool GREEDY = false>
 static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
                           const CUtensorMap& cb, const Params& P, cudaStream_t s) {
-  cudaError_t e = pass_kernel_ready<PAIR>();
+  cudaError_t e = pass_kernel_ready<PAIR, GREEDY>();
   if (e != cudaSuccess) return e;
   if (P.n_tiles <= 0) return cudaSuccess;
   if (!PAIR && P.cs == 1) {
     const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
-    e = launch_dep(k_tc_pass<false>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a, b, ca,
-                   cb, P);
+    e = launch_dep(k_tc_pass<false, GREEDY>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a,
+                   b, ca, cb, P);
   } else {
-    const int ncl = std::min(P.n_tiles, max_clusters<PAIR>(P.cs));
+    const int ncl = std::min(P.n_tiles, max_clusters<PAIR, GREEDY>(P.cs));
     cudaLaunchAttribute at[2];
     cudaLaunchConfig_t cfg = cluster_config(ncl * P.cs, P.cs, DCfg<PAIR>::SMEM, s, at);
     at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.numAttrs = 2;
-    e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR>, a, b, ca, cb, P);
+    e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR, GREEDY>, a, b, ca, cb, P);
   }
   if (e != cudaSuccess) return e;
   debug_kernel("k_tc_pass", s);
@@ -1567,7 +1642,7 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
       !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, bq))
     return cudaErrorInvalidValue;
   tc::Params P{};
-  P.mode = tc::MODE_DRAFT;
+  P.mode = c.greedy ? tc::MODE_GREEDY : tc::MODE_DRAFT;
   P.cs = cs;
   P.n_mt = n_mt;
   P.n_vt = ceil_div(h->V, tc::DBN);
@@ -1579,7 +1654,7 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   P.M = w.M;
   P.V = h->V;
   P.Mpad = w.Mpad;
-  P.k2 = c.k2;
+  P.k2 = c.greedy ? 1.f : c.k2;  // greedy records hold logits, not log2-scaled ones
   P.vbias = h->vbias;
   P.cscale = wsp<float>(c, w.off_cscale);
   P.sw = prp<float>(c, c.pl.off_sw);
@@ -1587,6 +1662,9 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   P.partd = wsp<float2>(c, w.off_partd);
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
+  if (c.greedy)
+    return pair ? tc::launch<true, true>(ma, mb, mca, mcb, P, c.stream)
+                : tc::launch<false, true>(ma, mb, mca, mcb, P, c.stream);
   return pair ? tc::launch<true>(ma, mb, mca, mcb, P, c.stream)
               : tc::launch<false>(ma, mb, mca, mcb, P, c.stream);
 }

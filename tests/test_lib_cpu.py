@@ -65,6 +65,8 @@ def _args(N=2, B=3, T=1.0, zt=1.0):
     (lambda h, a: setattr(a, "z_temperature", -1.0), 1),
     (lambda h, a: setattr(a, "hidden", None), 1),
     (lambda h, a: setattr(h, "prep_bytes", 0), 3),
+    (lambda h, a: setattr(a, "mode", 2), 1),
+    (lambda h, a: setattr(a, "mode", -1), 1),
 ])
 def test_bad_arguments_are_rejected_before_launch(mutate, status):
     lib = bd.lib()
