@@ -32,6 +32,8 @@ Definitions followed (section / equation of the paper):
   (Algorithm 1; Appendix A, "Distributional correctness").
 * Expected accepted length of the drafted block, sum_i prod_{j<=i} A_j
   (Eq. 3), and the overlap alpha_i = sum_v min(p_i(v), q(v|x_<i)).
+* Target-block early determinism D_b and its M-sample estimator (App. B),
+  for target rows that do not depend on the sampled prefix.
 * Greedy-branch mode (Sec. 3.1, "Drafter sampling during inference"; App. A,
   "Greedy-Branch Proposal", "Prefix-Marginalized Conditional" and its
   verification algorithm): z-hat from the prior, the block is the greedy
@@ -49,7 +51,7 @@ positive residual mass the replacement is drawn from p and flagged.
 import numpy as np
 
 from .philox import (STREAM_ACCEPT, STREAM_DRAFT, STREAM_PRIOR,
-                     STREAM_RESIDUAL, decision_uniform)
+                     STREAM_RESIDUAL, STREAM_TARGET, decision_uniform)
 
 # decisions whose margin to the threshold is below this are "ties"
 TIE_TOL = 1e-6
@@ -429,6 +431,59 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 emitted=emitted, n_emitted=len(emitted), exp_len=exp_len,
                 alpha_len=alpha_len, lse_target=lse_t, ties=ties,
                 first_tie=first_tie)
+
+
+# ------------------------------------------------- target-block early determinism
+def target_probs(target_rows, T):
+    """p_i = softmax(t_i / T) of each target row, fp64.  target_rows: [R, V]."""
+    st = f64(target_rows) / T
+    return np.exp(st - logsumexp(st, axis=-1)[:, None])
+
+
+def collision_probability(p):
+    """sum_v p(v)^2 of each row: the probability that two independent draws
+    from p collide, i.e. E_{X ~ p}[p(X)] (App. B)."""
+    return np.sum(p * p, axis=-1)
+
+
+def early_determinism_exact(p_rows):
+    """Target-block early determinism D_b(y) (App. B, Eq.
+    appendix-early-determinism) for b = len(p_rows) target rows that do not
+    depend on the sampled prefix (the synthetic targets here).
+
+    D_b = E_{x ~ p}[(1/b) sum_j prod_{i<=j} p_i(x_i)].  With independent
+    positions the expectation of each product is the product of the
+    per-position collision probabilities, so
+    D_b = (1/b) sum_j prod_{i<=j} sum_v p_i(v)^2.  p_rows: [b, V].
+    """
+    c = collision_probability(p_rows)
+    return float(np.mean(np.cumprod(c)))
+
+
+def early_determinism_estimate(p_rows, M, seed, n):
+    """The M-sample estimator of App. B (Eq.
+    appendix-early-determinism-estimator):
+    D-hat_b = 1/(M b) sum_m sum_j prod_{i<=j} p_i(x_i^(m)),
+    with M blocks x^(m) drawn from the target.  For prefix-independent rows
+    x_i^(m) ~ p_i, each an inverse-CDF draw with the stream-4 uniform (round
+    field = m, sequence n, position i).  Returns (D-hat, samples [M, b],
+    ties: (m, i, margin) for draws within TIE_TOL of an edge).
+    """
+    b = p_rows.shape[0]
+    samples = np.empty((M, b), dtype=np.int64)
+    ties = []
+    tot = 0.0
+    for m in range(M):
+        prod = 1.0
+        for i in range(b):
+            u = decision_uniform(seed, STREAM_TARGET, m, n, i)
+            x, margin = inverse_cdf(p_rows[i], u)
+            if margin < TIE_TOL:
+                ties.append((m, i, margin))
+            samples[m, i] = x
+            prod *= p_rows[i, x]
+            tot += prod
+    return tot / (M * b), samples, ties
 
 
 def prepare_head(head):

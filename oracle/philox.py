@@ -41,6 +41,8 @@ STREAM_PRIOR = 0     # latent category z-hat, once per block
 STREAM_DRAFT = 1     # draft token x_i at position i
 STREAM_ACCEPT = 2    # accept / reject x_i
 STREAM_RESIDUAL = 3  # residual draw at the first rejection, or the bonus token
+STREAM_TARGET = 4    # target block samples of the early-determinism estimator
+                     # (round field = sample index m, pos_abs = position i)
 
 
 def philox4x32_10(ctr, key):
