@@ -223,14 +223,53 @@ def run_sweep(args):
                 ms = _timed_steps(step, args.steps, args.warmup)
                 mean_L = float(torch.stack([v["accepted"].float().mean()
                                             for v in vouts[args.warmup:]]).mean())
+                # target-block early determinism of the cell, in the bins of App. B
+                det = vouts[args.warmup]["determinism"].float().cpu()
+                bins = torch.histc(det, bins=5, min=0.0, max=1.0).int().tolist()
                 print(json.dumps({"sweep": {"K": K, "r": cfg["r"], "N": cfg["N"], "B": cfg["B"],
                                             "T": T, "sigma": sigma, "mean_accepted_length": mean_L,
+                                            "determinism_mean": float(det.mean()),
+                                            "determinism_bins_0.2": bins,
                                             "blocks_per_s": cfg["N"] * args.steps / (ms / 1e3),
                                             "accepted_tokens_per_s":
                                                 mean_L * cfg["N"] * args.steps / (ms / 1e3),
                                             "ms_per_step": ms / args.steps,
                                             "data": "synthetic"}}), flush=True)
             del head, ws, blk, head_t
+
+
+def run_determinism(args, cfg):
+    """Target-block early determinism (App. B) on the workload's target logits
+    [N, B+1, V]: the paper's estimator setting b = 15, M = 20.  One JSON line:
+    ms per call (target statistics, 9,600 inverse-CDF draws, reduction) and
+    the HBM rate of the one pass over the target."""
+    import torch
+    import synth
+    from paper_2608_05448_gb300 import dblast_target_determinism
+    dev = torch.device("cuda", 0)
+    head_t = synth.make_head(cfg, dev)
+    blk = synth.make_block(cfg, head_t, 0, dev)
+    del head_t
+    target = blk["target"]
+    N, rows, V = target.shape
+    b, M = min(15, rows), 20
+    from paper_2608_05448_gb300 import lib
+    nbytes = lib().dblast_determinism_workspace_bytes(N, rows, b, V, M)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    res = {}
+
+    def step(k):
+        res["out"] = dblast_target_determinism(target, b, args.T, M=M, seed=k, ws=ws)
+    ms = _timed_steps(step, args.steps, args.warmup) / args.steps
+    out = {k: v.cpu() for k, v in res["out"].items()}
+    tbytes = target.numel() * target.element_size()
+    print(json.dumps({"determinism": {
+        "workload": cfg["name"], "N": N, "rows": rows, "V": V, "b": b, "M": M, "T": args.T,
+        "ms_per_call": ms, "target_bytes": tbytes,
+        "target_pass_gbs": tbytes / (ms * 1e-3) / 1e9,
+        "d_exact_mean": float(out["d_exact"].mean()), "d_hat_mean": float(out["d_hat"].mean()),
+        "bins_0.2": torch.histc(out["d_exact"], bins=5, min=0.0, max=1.0).int().tolist(),
+        "data": "synthetic"}}), flush=True)
 
 
 def run_serve(args):
@@ -294,6 +333,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--sweep", action="store_true",
                     help="entropy-sweep report (K=16 vs K=1 cells), one JSON line per cell")
+    ap.add_argument("--determinism", action="store_true",
+                    help="target-block early determinism report (b = 15, M = 20), one JSON line")
     ap.add_argument("--serve", action="store_true",
                     help="serving report (N=256, B=8/32, four rounds), one JSON line per round")
     ap.add_argument("--n-seqs", type=int, default=None,
@@ -310,9 +351,11 @@ def main():
     if args.impl == "reference":
         run_reference(args, cfg, rank)
         return
-    if args.sweep or args.serve:
+    if args.sweep or args.serve or args.determinism:
         import torch
         torch.cuda.set_device(0)
+        if args.determinism:
+            run_determinism(args, cfg)
         if args.sweep:
             run_sweep(args)
         if args.serve:

@@ -150,6 +150,10 @@ typedef struct {
   uint32_t* tie_flags;  /* [N]        bit0 z-hat, bit1 draft, bit2 accept, bit3 residual/bonus,
                                        bit4 residual mass < 1e-6: a decision within 1e-6 of its threshold
                                        (GREEDY mode leaves bit1 clear: argmax decisions are not flagged) */
+  float* collision;     /* [N, B]     sum_v p_i(v)^2, the collision probability of target row i (App. B) */
+  float* determinism;   /* [N]        target-block early determinism D_B = (1/B) sum_j prod_{i<=j}
+                                       collision_i (App. B, Eq. appendix-early-determinism, for
+                                       target rows that do not depend on the drafted prefix) */
 } dblast_verify_out;
 
 /* Bytes of the prep buffer for this head (depends on V, K, r, e != NULL). */
@@ -227,6 +231,28 @@ dblast_status dblast_stats_get(dblast_stats* out);
 dblast_status dblast_target_lse_noalloc(const void* target, int rows, int V, dblast_dtype dtype,
                                         float temperature, float* lse_out,
                                         dblast_stream_t stream);
+
+/* Target-block early determinism of given target rows (App. B).
+ *   collision[n, i] = sum_v p_{n,i}(v)^2 for the first b rows of sequence n,
+ *   d_exact[n]      = (1/b) sum_j prod_{i<=j} collision[n, i]
+ *                     (Eq. appendix-early-determinism when the rows do not
+ *                     depend on the sampled prefix),
+ *   d_hat[n]        = 1/(M b) sum_m sum_j prod_{i<=j} p_{n,i}(x_i^(m)), the
+ *                     M-sample estimator (Eq. appendix-early-determinism-estimator)
+ *                     with x_i^(m) ~ p_{n,i} drawn by inverse CDF from the
+ *                     stream-4 uniform (round field = m, sequence n, pos_abs = i),
+ *   samples[n, m, i] = x_i^(m).
+ * target: [N, rows, V] device logits of `dtype`, p = softmax(t / temperature);
+ * 1 <= b <= min(rows, 32).  Every output is a device pointer or NULL; d_hat
+ * and samples need M >= 1.  Scratch: `workspace` of
+ * dblast_determinism_workspace_bytes(N, rows, b, V, M) bytes, 16-byte aligned.
+ * Asynchronous on `stream`; argument errors return before any launch. */
+size_t dblast_determinism_workspace_bytes(int N, int rows, int b, int V, int M);
+dblast_status dblast_target_determinism(const void* target, dblast_dtype dtype, int N, int rows,
+                                        int b, int V, float temperature, int M, uint64_t seed,
+                                        float* collision, float* d_exact, float* d_hat,
+                                        int32_t* samples, void* workspace,
+                                        size_t workspace_bytes, dblast_stream_t stream);
 
 const char* dblast_status_string(dblast_status s);
 const char* dblast_version(void);

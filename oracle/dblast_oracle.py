@@ -269,7 +269,9 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 logw=logw, q_tok=q_tok, p_tok=p_tok, accept_prob=accept_prob,
                 alpha=alpha, accepted=L, emitted=emitted,
                 n_emitted=len(emitted), exp_len=exp_len, alpha_len=alpha_len,
-                lse_target=lse_t, ties=ties, first_tie=first_tie)
+                lse_target=lse_t, ties=ties, first_tie=first_tie,
+                collision=collision_probability(p[:B]),
+                determinism=early_determinism_exact(p[:B]))
 
 
 # --------------------------------------------------------- greedy-branch mode
@@ -430,7 +432,8 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 accept_prob=accept_prob, alpha=alpha, accepted=L,
                 emitted=emitted, n_emitted=len(emitted), exp_len=exp_len,
                 alpha_len=alpha_len, lse_target=lse_t, ties=ties,
-                first_tie=first_tie)
+                first_tie=first_tie, collision=collision_probability(p[:B]),
+                determinism=early_determinism_exact(p[:B]))
 
 
 # ------------------------------------------------- target-block early determinism

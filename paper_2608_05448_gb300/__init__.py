@@ -8,6 +8,7 @@ from .binding import (DBLastError, Head, Workspace, alloc_draft_out,  # noqa: F4
                       alloc_verify_out, dblast_device_status,
                       dblast_draft_and_verify, dblast_draft_block,
                       dblast_set_wait_limit, dblast_stats_get,
-                      dblast_stats_reset, dblast_verify_block, lib)
+                      dblast_stats_reset, dblast_target_determinism,
+                      dblast_verify_block, lib)
 
 lib()

@@ -64,14 +64,14 @@ class CVerifyOut(ctypes.Structure):
     _fields_ = [("target", ctypes.c_void_p), ("has_bonus", ctypes.c_int)] + [
         (n, ctypes.c_void_p) for n in
         ("p_tok", "accept_prob", "alpha", "lse_target", "accepted", "emitted",
-         "n_emitted", "exp_len", "alpha_len", "tie_flags")]
+         "n_emitted", "exp_len", "alpha_len", "tie_flags", "collision", "determinism")]
 
 
 EXPORTS = ["dblast_prep_bytes", "dblast_workspace_bytes", "dblast_head_prepare",
            "dblast_draft_block", "dblast_verify_block", "dblast_draft_and_verify",
            "dblast_device_status", "dblast_set_wait_limit", "dblast_stats_reset",
            "dblast_stats_get", "dblast_target_lse_noalloc", "dblast_status_string",
-           "dblast_version"]
+           "dblast_version", "dblast_determinism_workspace_bytes", "dblast_target_determinism"]
 
 
 def load_library(path=None, build_if_missing=True):
@@ -112,6 +112,13 @@ def load_library(path=None, build_if_missing=True):
                                               ctypes.c_int, ctypes.c_float, ctypes.c_void_p,
                                               ctypes.c_void_p]
     lib.dblast_target_lse_noalloc.restype = ctypes.c_int
+    lib.dblast_determinism_workspace_bytes.argtypes = [ctypes.c_int] * 5
+    lib.dblast_determinism_workspace_bytes.restype = S
+    lib.dblast_target_determinism.argtypes = [
+        ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+        ctypes.c_float, ctypes.c_int, ctypes.c_uint64, ctypes.c_void_p, ctypes.c_void_p,
+        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, S, ctypes.c_void_p]
+    lib.dblast_target_determinism.restype = ctypes.c_int
     lib.dblast_status_string.argtypes = [ctypes.c_int]
     lib.dblast_status_string.restype = ctypes.c_char_p
     lib.dblast_version.argtypes = []
@@ -247,7 +254,9 @@ def alloc_verify_out(N, B, has_bonus, device):
                 n_emitted=torch.empty(N, dtype=i, device=device),
                 exp_len=torch.empty(N, dtype=f, device=device),
                 alpha_len=torch.empty(N, dtype=f, device=device),
-                tie_flags=torch.empty(N, dtype=i, device=device))
+                tie_flags=torch.empty(N, dtype=i, device=device),
+                collision=torch.empty(N, B, dtype=f, device=device),
+                determinism=torch.empty(N, dtype=f, device=device))
 
 
 def _draft_struct(d):
@@ -344,3 +353,30 @@ def dblast_target_lse_noalloc(target, temperature, lse_out):
         raise ValueError("lse_out must have one entry per row")
     return lib().dblast_target_lse_noalloc(_ptr(target), rows, V, DTYPES[target.dtype],
                                            float(temperature), _ptr(lse_out), _stream())
+
+
+def dblast_target_determinism(target, b, temperature, M=0, seed=0, samples=False, ws=None):
+    """Target-block early determinism of target logits [N, rows, V] (App. B):
+    returns a dict with collision [N, b], d_exact [N] and, for M >= 1, the
+    M-sample estimate d_hat [N] (and the drawn blocks [N, M, b] if samples)."""
+    _cuda_contig(target, "target")
+    if target.dtype not in DTYPES or target.dim() != 3:
+        raise ValueError("target must be a bf16/fp32 [N, rows, V] tensor")
+    N, rows, V = target.shape
+    dev = target.device
+    f = torch.float32
+    out = dict(collision=torch.empty(N, b, dtype=f, device=dev),
+               d_exact=torch.empty(N, dtype=f, device=dev))
+    if M >= 1:
+        out["d_hat"] = torch.empty(N, dtype=f, device=dev)
+        if samples:
+            out["samples"] = torch.empty(N, M, b, dtype=torch.int32, device=dev)
+    nbytes = lib().dblast_determinism_workspace_bytes(N, rows, b, V, int(M))
+    if ws is None or ws.numel() < nbytes:
+        ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=dev)
+    _check(lib().dblast_target_determinism(
+        _ptr(target), DTYPES[target.dtype], N, rows, int(b), V, float(temperature), int(M),
+        int(seed) & ((1 << 64) - 1), _ptr(out["collision"]), _ptr(out["d_exact"]),
+        _ptr(out.get("d_hat")), _ptr(out.get("samples")), _ptr(ws), nbytes, _stream()),
+        "dblast_target_determinism")
+    return out

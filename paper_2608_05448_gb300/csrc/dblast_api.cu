@@ -144,6 +144,7 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_ties = take((size_t)N * sizeof(uint32_t));
   w.off_xhat = take((size_t)w.M * K * sizeof(int32_t));
   w.off_cmask = take((size_t)w.M * sizeof(uint32_t));
+  w.off_coll = take((size_t)w.Rt * sizeof(float));
   w.total = o;
   return w;
 }
@@ -436,6 +437,80 @@ dblast_status dblast_stats_get(dblast_stats* out) {
   out->draft_pass_ms = ms[0];
   out->verify_pass_ms = ms[1];
   return DBLAST_OK;
+}
+
+// Workspace of dblast_target_determinism: the target statistics of the
+// N x rows target rows (tile records, log-sum-exp, collision probability) and
+// p_i(x_i^(m)) of every sample.
+struct DetLayout {
+  size_t off_partt, off_lt2, off_coll, off_pval, total;
+  int nt, Rt;
+};
+static DetLayout det_layout(int N, int rows, int b, int V, int M) {
+  DetLayout d{};
+  d.nt = ceil_div(V, TILE_V);
+  d.Rt = N * rows;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  d.off_partt = take((size_t)d.nt * d.Rt * sizeof(float2));
+  d.off_lt2 = take((size_t)d.Rt * sizeof(float2));
+  d.off_coll = take((size_t)d.Rt * sizeof(float));
+  d.off_pval = take((size_t)N * (M > 0 ? M : 1) * b * sizeof(float));
+  d.total = o;
+  return d;
+}
+
+size_t dblast_determinism_workspace_bytes(int N, int rows, int b, int V, int M) {
+  if (N < 1 || rows < 1 || b < 1 || V < 1 || M < 0) return 0;
+  return det_layout(N, rows, b, V, M).total;
+}
+
+dblast_status dblast_target_determinism(const void* target, dblast_dtype dtype, int N, int rows,
+                                        int b, int V, float temperature, int M, uint64_t seed,
+                                        float* collision, float* d_exact, float* d_hat,
+                                        int32_t* samples, void* ws, size_t ws_bytes,
+                                        dblast_stream_t stream) {
+  if (!target || !aligned16(target)) return DBLAST_ERR_INVALID_ARG;
+  if (dtype != DBLAST_BF16 && dtype != DBLAST_F32) return DBLAST_ERR_INVALID_ARG;
+  if (N < 1 || rows < 1 || V < 1 || b < 1 || b > 32 || b > rows || M < 0 || M > (1 << 24))
+    return DBLAST_ERR_INVALID_ARG;
+  if (!(temperature > 0.f)) return DBLAST_ERR_INVALID_ARG;
+  if ((d_hat || samples) && M < 1) return DBLAST_ERR_INVALID_ARG;
+  if ((long long)N * rows > (1LL << 24)) return DBLAST_ERR_INVALID_ARG;
+  const DetLayout d = det_layout(N, rows, b, V, M);
+  if (!ws || !aligned16(ws) || ws_bytes < d.total) return DBLAST_ERR_WORKSPACE;
+  dblast_head h{};
+  h.V = V;
+  h.dtype = dtype;
+  dblast_block_args a{};
+  a.N = N;
+  a.B = rows - 1;  // the target-statistics kernels index rows as n (B + 1) + i
+  StepCtx c{};
+  c.head = &h;
+  c.args = &a;
+  c.wl.N = N;
+  c.wl.B = rows - 1;
+  c.wl.V = V;
+  c.wl.nt = d.nt;
+  c.wl.Rt = d.Rt;
+  c.wl.off_partt = d.off_partt;
+  c.wl.off_lt2 = d.off_lt2;
+  c.wl.off_coll = d.off_coll;
+  c.ws = static_cast<unsigned char*>(ws);
+  c.stream = reinterpret_cast<cudaStream_t>(stream);
+  c.k2 = LOG2E / temperature;
+  c.Bt = rows;
+  dblast_verify_out o{};
+  o.target = target;
+  o.has_bonus = 1;
+  g_calls.fetch_add(1, std::memory_order_relaxed);
+  return cuda_status(dbg(launch_determinism(c, &o, rows, b, M, seed, collision, d_exact, d_hat,
+                                            samples, d.off_pval),
+                         "determinism", c.stream));
 }
 
 const char* dblast_status_string(dblast_status s) {

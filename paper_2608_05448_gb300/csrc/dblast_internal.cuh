@@ -48,13 +48,14 @@ struct PrepLayout {
 //   partv float2 [nt,Mpad] | av float4 [AV_SPLIT,M] | ties u32 [N]
 //   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
 //   token and the consistent-branch set C_i as a bit mask over z)
+//   coll f32 [Rt]  (collision probability sum_v p(v)^2 of every target row)
 constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
 constexpr int AV_SPLIT = 8;   // partial sums of the verify records per row
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
       off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
-      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, total;
+      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, off_coll, total;
 };
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
@@ -287,5 +288,8 @@ cudaError_t launch_verify_pass_simt(const StepCtx& c);
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
 cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* out);
 cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
+cudaError_t launch_determinism(const StepCtx& c, const dblast_verify_out* o, int rows, int b,
+                               int M, uint64_t seed, float* collision, float* d_exact,
+                               float* d_hat, int32_t* samples, size_t off_pval);
 
 }  // namespace dblast

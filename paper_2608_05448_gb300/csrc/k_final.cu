@@ -495,7 +495,8 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
 // ---------------------------------------------------------------- target side
 // One block per target row: a half-warp per tile of 128 tokens (8 per lane),
 // the tile records partt and the row's lse2t = log2 sum_v 2^{t_v k2} (also as
-// a float pair lt2 for the verify pass).
+// a float pair lt2 for the verify pass), and the row's collision probability
+// coll = sum_v p(v)^2 (App. B), from the same exponentials squared.
 constexpr int TS_NT = 256;
 constexpr int TS_HW = TS_NT / 16;  // half-warps per block
 constexpr int TS_NF = 4;           // tiles in flight per half-warp
@@ -504,15 +505,16 @@ template <typename Tin>
 __global__ void __launch_bounds__(TS_NT)
     k_target_stats(const Tin* __restrict__ target, int V, int nt, int B, int Bt, int Rt, float k2,
                    bool vec, float2* __restrict__ partt, float2* __restrict__ lt2,
-                   float* __restrict__ lse_out) {
+                   float* __restrict__ coll, float* __restrict__ lse_out) {
   __shared__ float smx[TS_HW];
   __shared__ FF ssum[TS_HW];
+  __shared__ float ssq[TS_HW];
   const int row = blockIdx.x;
   const int n = row / Bt, i = row - n * Bt;
   const int rl = n * (B + 1) + i;
   const Tin* tr = target + (size_t)row * V;
   const int hw = threadIdx.x >> 4, hl = threadIdx.x & 15;
-  float rmax = -INFINITY;
+  float rmax = -INFINITY, rsq = 0.f;
   FF rsum{0.f, 0.f};
   // every lane of both half-warps runs the shuffles; `valid` gates the results
   auto tile = [&](int t, const float (&x)[8], bool valid) {
@@ -521,18 +523,29 @@ __global__ void __launch_bounds__(TS_NT)
     for (int j = 1; j < 8; ++j) mx = fmaxf(mx, x[j]);
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(FULLMASK, mx, o));
-    float s = 0.f;
+    float s = 0.f, s2 = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) s += exp2f((x[j] - mx) * k2);
+    for (int j = 0; j < 8; ++j) {
+      const float e = exp2f((x[j] - mx) * k2);
+      s += e;
+      s2 = fmaf(e, e, s2);
+    }
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(FULLMASK, s, o);
+    for (int o = 8; o > 0; o >>= 1) {
+      s += __shfl_xor_sync(FULLMASK, s, o);
+      s2 += __shfl_xor_sync(FULLMASK, s2, o);
+    }
     if (!valid) return;
     if (hl == 0) partt[(size_t)t * Rt + rl] = make_float2(mx, s);
     if (mx > rmax) {
-      rsum = ff_mulf(rsum, exp2f((rmax - mx) * k2));
+      const float f = exp2f((rmax - mx) * k2);
+      rsum = ff_mulf(rsum, f);
+      rsq *= f * f;
       rmax = mx;
     }
-    rsum = ff_addf(rsum, s * exp2f((mx - rmax) * k2));
+    const float g = exp2f((mx - rmax) * k2);
+    rsum = ff_addf(rsum, s * g);
+    rsq = fmaf(s2, g * g, rsq);
   };
   // TS_NF tiles in flight per half-warp; the loop bounds are uniform over the block
   const int iters = ceil_div(nt, TS_HW);
@@ -552,6 +565,7 @@ __global__ void __launch_bounds__(TS_NT)
   if (hl == 0) {
     smx[hw] = rmax;
     ssum[hw] = rsum;
+    ssq[hw] = rsq;
   }
   __syncthreads();
   if (threadIdx.x < 32) {
@@ -561,13 +575,23 @@ __global__ void __launch_bounds__(TS_NT)
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) M2 = fmaxf(M2, __shfl_xor_sync(FULLMASK, M2, o));
     FF S{0.f, 0.f};
-    if (M2 != -INFINITY && ml != -INFINITY) S = ff_mulf(ssum[l], exp2f((ml - M2) * k2));
+    float Q = 0.f;
+    if (M2 != -INFINITY && ml != -INFINITY) {
+      const float f = exp2f((ml - M2) * k2);
+      S = ff_mulf(ssum[l], f);
+      Q = ssq[l] * f * f;
+    }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) S = ff_add(S, ff_shfl_xor(S, o));
+    for (int o = 16; o > 0; o >>= 1) {
+      S = ff_add(S, ff_shfl_xor(S, o));
+      Q += __shfl_xor_sync(FULLMASK, Q, o);
+    }
     if (l == 0) {
       const FF L = (M2 == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
                                                      : ff_add(ff_prod(M2, k2), ff_log2(S));
       lt2[rl] = ff_st(L);
+      const float sf = ff_f(S);
+      coll[rl] = sf > 0.f ? Q / (sf * sf) : 0.f;
       if (lse_out) lse_out[row] = ff_f(L) * LN2;
     }
   }
@@ -590,7 +614,7 @@ __device__ __forceinline__ float ex2a(float x) {
 __global__ void __launch_bounds__(32 * TS2_NW)
     k_target_stats_tiles(const __nv_bfloat16* __restrict__ target, int V, int nt, int B, int Bt,
                          int Rt, float k2, float2* __restrict__ partt, float2* __restrict__ lt2,
-                         float* __restrict__ lse_out) {
+                         float* __restrict__ coll, float* __restrict__ lse_out) {
   __shared__ __align__(16) uint4 stg[TS2_NW][2][32 * 16];  // 48 KB
   const int row = blockIdx.x;
   const int n = row / Bt, i = row - n * Bt;
@@ -619,7 +643,7 @@ __global__ void __launch_bounds__(32 * TS2_NW)
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  float rmax = -INFINITY;
+  float rmax = -INFINITY, rsq = 0.f;
   FF rsum{0.f, 0.f};
   int buf = 0;
   if (w < groups) stage(w, 0);
@@ -644,7 +668,7 @@ __global__ void __launch_bounds__(32 * TS2_NW)
                                        *reinterpret_cast<const __nv_bfloat162*>(&q.w))));
     }
     const float mx = fmaxf(__low2float(m2), __high2float(m2));
-    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+    float s4[4] = {0.f, 0.f, 0.f, 0.f}, q4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
       const uint4 q = ws[l * 16 + (j ^ (l & 7))];
@@ -652,18 +676,25 @@ __global__ void __launch_bounds__(32 * TS2_NW)
 #pragma unroll
       for (int h = 0; h < 4; ++h) {
         const float a = __uint_as_float(u[h] << 16), b = __uint_as_float(u[h] & 0xFFFF0000u);
-        s4[h] += ex2a((a - mx) * k2) + ex2a((b - mx) * k2);
+        const float ea = ex2a((a - mx) * k2), eb = ex2a((b - mx) * k2);
+        s4[h] += ea + eb;
+        q4[h] = fmaf(ea, ea, fmaf(eb, eb, q4[h]));
       }
     }
     __syncwarp();  // every lane has read this buffer before it is refilled
     if (t < nt) {
       const float s = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      const float s2 = (q4[0] + q4[1]) + (q4[2] + q4[3]);
       partt[(size_t)t * Rt + rl] = make_float2(mx, s);
       if (mx > rmax) {
-        rsum = ff_mulf(rsum, exp2f((rmax - mx) * k2));
+        const float f = exp2f((rmax - mx) * k2);
+        rsum = ff_mulf(rsum, f);
+        rsq *= f * f;
         rmax = mx;
       }
-      rsum = ff_addf(rsum, s * exp2f((mx - rmax) * k2));
+      const float g = exp2f((mx - rmax) * k2);
+      rsum = ff_addf(rsum, s * g);
+      rsq = fmaf(s2, g * g, rsq);
     }
   }
   // lanes, then warps
@@ -671,27 +702,41 @@ __global__ void __launch_bounds__(32 * TS2_NW)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M1 = fmaxf(M1, __shfl_xor_sync(FULLMASK, M1, o));
   FF S1{0.f, 0.f};
-  if (M1 != -INFINITY && rmax != -INFINITY) S1 = ff_mulf(rsum, exp2f((rmax - M1) * k2));
+  float Q1 = 0.f;
+  if (M1 != -INFINITY && rmax != -INFINITY) {
+    const float f = exp2f((rmax - M1) * k2);
+    S1 = ff_mulf(rsum, f);
+    Q1 = rsq * f * f;
+  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) S1 = ff_add(S1, ff_shfl_xor(S1, o));
+  for (int o = 16; o > 0; o >>= 1) {
+    S1 = ff_add(S1, ff_shfl_xor(S1, o));
+    Q1 += __shfl_xor_sync(FULLMASK, Q1, o);
+  }
   // each warp's partial goes into the first entry of its own (now idle) buffer
   if (l == 0) stg[w][0][0] = make_uint4(__float_as_uint(M1), __float_as_uint(S1.hi),
-                                        __float_as_uint(S1.lo), 0u);
+                                        __float_as_uint(S1.lo), __float_as_uint(Q1));
   __syncthreads();
   if (threadIdx.x == 0) {
     float M2 = -INFINITY;
     for (int k = 0; k < TS2_NW; ++k) M2 = fmaxf(M2, __uint_as_float(stg[k][0][0].x));
     FF S{0.f, 0.f};
+    float Q = 0.f;
     if (M2 != -INFINITY)
       for (int k = 0; k < TS2_NW; ++k) {
         const uint4 e = stg[k][0][0];
         const float mk = __uint_as_float(e.x);
-        if (mk != -INFINITY)
-          S = ff_add(S, ff_mulf(FF{__uint_as_float(e.y), __uint_as_float(e.z)}, exp2f((mk - M2) * k2)));
+        if (mk != -INFINITY) {
+          const float f = exp2f((mk - M2) * k2);
+          S = ff_add(S, ff_mulf(FF{__uint_as_float(e.y), __uint_as_float(e.z)}, f));
+          Q = fmaf(__uint_as_float(e.w), f * f, Q);
+        }
       }
     const FF L = (M2 == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
                                                    : ff_add(ff_prod(M2, k2), ff_log2(S));
     lt2[rl] = ff_st(L);
+    const float sf = ff_f(S);
+    coll[rl] = sf > 0.f ? Q / (sf * sf) : 0.f;
     if (lse_out) lse_out[row] = ff_f(L) * LN2;
   }
 }
@@ -706,7 +751,8 @@ static cudaError_t target_typed(const StepCtx& c, const dblast_verify_out* o) {
     if (vec) {
       k_target_stats_tiles<<<rows, 32 * TS2_NW, 0, c.stream>>>(
           static_cast<const __nv_bfloat16*>(o->target), w.V, w.nt, w.B, Bt, w.Rt, c.k2,
-          wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), o->lse_target);
+          wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), wsp<float>(c, w.off_coll),
+          o->lse_target);
       debug_kernel("k_target_stats_tiles", c.stream);
       count_launches(1);
       return cudaGetLastError();
@@ -714,7 +760,8 @@ static cudaError_t target_typed(const StepCtx& c, const dblast_verify_out* o) {
   }
   k_target_stats<Tin><<<rows, TS_NT, 0, c.stream>>>(
       static_cast<const Tin*>(o->target), w.V, w.nt, w.B, Bt, w.Rt, c.k2, vec,
-      wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), o->lse_target);
+      wsp<float2>(c, w.off_partt), wsp<float2>(c, w.off_lt2), wsp<float>(c, w.off_coll),
+      o->lse_target);
   debug_kernel("k_target_stats", c.stream);
   count_launches(1);
   return cudaGetLastError();
@@ -776,8 +823,9 @@ __global__ void __launch_bounds__(VF_NT)
                    const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
                    const float2* __restrict__ partv, const float2* __restrict__ partt,
                    const float4* __restrict__ avp, const int32_t* __restrict__ tok,
-                   const uint32_t* __restrict__ ties_draft, int V, int K, int rr, int B, int Bt,
-                   int nt, int M, int Mpad, int Rt, float k2, uint64_t seed,
+                   const uint32_t* __restrict__ ties_draft, const float* __restrict__ coll, int V,
+                   int K, int rr, int B, int Bt, int nt, int M, int Mpad, int Rt, float k2,
+                   uint64_t seed,
                    int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
                    dblast_verify_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
@@ -822,17 +870,27 @@ __global__ void __launch_bounds__(VF_NT)
     const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
     // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha (products in lane order)
+    // App. B: collision probabilities of the block's target rows and
+    // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
+    float cC = 1.f;
+    if (lane < B) {
+      cC = coll[(size_t)n * (B + 1) + lane];
+      if (out.collision) out.collision[n * B + lane] = cC;
+    }
     float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const float ta = __shfl_up_sync(FULLMASK, cA, o);
       const float tl = __shfl_up_sync(FULLMASK, cAl, o);
+      const float tc = __shfl_up_sync(FULLMASK, cC, o);
       if (lane >= o) {
         cA *= ta;
         cAl *= tl;
+        cC *= tc;
       }
     }
     FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
+    FF ed{lane < B ? cC : 0.f, 0.f};
     FF R{0.f, 0.f};
     if (L < B && lane < AV_SPLIT) {
       const float4 q = avp[(size_t)lane * M + n * B + L];
@@ -843,6 +901,7 @@ __global__ void __launch_bounds__(VF_NT)
       R = ff_add(R, ff_shfl_xor(R, o));
       el = ff_add(el, ff_shfl_xor(el, o));
       ea = ff_add(ea, ff_shfl_xor(ea, o));
+      ed = ff_add(ed, ff_shfl_xor(ed, o));
     }
     if (L < B && lane < K) {  // normalisers of the rejected row: L_z - log2 w_z
       const size_t mz = (size_t)(n * B + L) * K + lane;
@@ -852,6 +911,7 @@ __global__ void __launch_bounds__(VF_NT)
     if (lane == 0) {
       if (out.exp_len) out.exp_len[n] = ff_f(el);
       if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
+      if (out.determinism) out.determinism[n] = ff_f(ed) / (float)B;
       sL = L;
       sties = ties;
       sR = R;
@@ -926,8 +986,8 @@ static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out*
       wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2), wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
       wsp<float2>(c, w.off_partt), wsp<float4>(c, w.off_av), wsp<int32_t>(c, w.off_tok),
-      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, Bt, w.nt, w.M, w.Mpad, w.Rt, c.k2,
-      c.args->seed, c.args->pos, c.args->round, *o);
+      wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.rr, w.B, Bt,
+      w.nt, w.M, w.Mpad, w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o);
   debug_kernel("k_verify_final", c.stream);
   count_launches(2);
   return le != cudaSuccess ? le : cudaGetLastError();
@@ -1118,8 +1178,9 @@ __global__ void __launch_bounds__(VF_NT)
                     const int32_t* __restrict__ xhat, const uint32_t* __restrict__ cmask,
                     const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
                     const float2* __restrict__ partt, const int32_t* __restrict__ tok,
-                    const uint32_t* __restrict__ ties_draft, int V, int K, int B, int Bt, int nt,
-                    int Rt, float k2, uint64_t seed, int64_t* __restrict__ pos,
+                    const uint32_t* __restrict__ ties_draft, const float* __restrict__ coll,
+                    int V, int K, int B, int Bt, int nt, int Rt, float k2, uint64_t seed,
+                    int64_t* __restrict__ pos,
                     uint32_t* __restrict__ rnd, dblast_verify_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<VF_NT> fs;
@@ -1186,21 +1247,32 @@ __global__ void __launch_bounds__(VF_NT)
     const int L = rej ? (__ffs(rej) - 1) : B;
     const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    // App. B: collision probabilities of the block's target rows and
+    // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
+    float cC = 1.f;
+    if (lane < B) {
+      cC = coll[(size_t)n * (B + 1) + lane];
+      if (out.collision) out.collision[n * B + lane] = cC;
+    }
     float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const float ta = __shfl_up_sync(FULLMASK, cA, o);
       const float tl = __shfl_up_sync(FULLMASK, cAl, o);
+      const float tc = __shfl_up_sync(FULLMASK, cC, o);
       if (lane >= o) {
         cA *= ta;
         cAl *= tl;
+        cC *= tc;
       }
     }
     FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
+    FF ed{lane < B ? cC : 0.f, 0.f};
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       el = ff_add(el, ff_shfl_xor(el, o));
       ea = ff_add(ea, ff_shfl_xor(ea, o));
+      ed = ff_add(ed, ff_shfl_xor(ed, o));
     }
     // the atoms of the rejected row: token, q_greedy, the tile (first atom of a tile only)
     if (L < B && lane == L) {
@@ -1229,6 +1301,7 @@ __global__ void __launch_bounds__(VF_NT)
     if (lane == 0) {
       if (out.exp_len) out.exp_len[n] = ff_f(el);
       if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
+      if (out.determinism) out.determinism[n] = ff_f(ed) / (float)B;
       sL = L;
       sties = ties;
     }
@@ -1305,8 +1378,8 @@ static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out
       static_cast<const Tin*>(o->target), wsp<float>(c, w.off_log2pi),
       wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask), wsp<float>(c, w.off_qtok),
       wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
-      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.B, c.Bt, w.nt, w.Rt, c.k2, c.args->seed,
-      c.args->pos, c.args->round, *o);
+      wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.B, c.Bt, w.nt,
+      w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o);
   debug_kernel("k_greedy_verify", c.stream);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
@@ -1315,6 +1388,108 @@ static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out
 cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {
   return c.head->dtype == DBLAST_F32 ? greedy_verify_typed<float>(c, o)
                                      : greedy_verify_typed<__nv_bfloat16>(c, o);
+}
+
+// ---------------------------------------------------------------- early determinism
+// App. B.  The target statistics give every row's tile records, log-sum-exp
+// and collision probability; k_target_sample draws x_i^(m) ~ p_i (one block
+// per (i, m, n), the two-level inverse CDF of the bonus draw with the
+// stream-4 uniform) and keeps p_i(x_i^(m)); k_determinism_reduce forms
+// D_exact from the collision probabilities and D-hat from the samples.
+template <typename Tin>
+__global__ void __launch_bounds__(VF_NT)
+    k_target_sample(const Tin* __restrict__ target, const float2* __restrict__ partt,
+                    const float2* __restrict__ lt2, int V, int nt, int rows, int b, int M, int Rt,
+                    float k2, uint64_t seed, float* __restrict__ pval, int32_t* __restrict__ samples) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ FindShared<VF_NT> fs;
+  const int i = blockIdx.x, m = blockIdx.y, n = blockIdx.z;
+  const int rl = n * rows + i;
+  const FF Lt = ff_ld(lt2 + rl);
+  const TargetTokenProb<Tin> pv{target + (size_t)rl * V, k2, Lt};
+  const float u = decision_uniform(seed, 4u, (uint32_t)m, (uint32_t)n, (uint32_t)i);
+  const FindOut f = block_find<VF_NT>(nt, V, TargetTileMass{partt + rl, (size_t)Rt, k2, Lt}, pv,
+                                      FF{u, 0.f}, 1.f, fs);
+  if (threadIdx.x == 0) {
+    const int x = f.x >= 0 ? f.x : 0;
+    const size_t o = ((size_t)n * M + m) * b + i;
+    pval[o] = pv(x);
+    if (samples) samples[o] = x;
+  }
+}
+
+constexpr int DR_NT = 256;
+__global__ void __launch_bounds__(DR_NT)
+    k_determinism_reduce(const float* __restrict__ coll, const float* __restrict__ pval, int rows,
+                         int b, int M, float* __restrict__ collision, float* __restrict__ d_exact,
+                         float* __restrict__ d_hat) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ FF red[DR_NT / 32];
+  const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) {
+    FF d{0.f, 0.f};
+    float c = 1.f;
+    for (int i = 0; i < b; ++i) {
+      const float ci = coll[(size_t)n * rows + i];
+      if (collision) collision[n * b + i] = ci;
+      c *= ci;
+      d = ff_addf(d, c);
+    }
+    if (d_exact) d_exact[n] = ff_f(d) / (float)b;
+  }
+  if (!d_hat) return;  // uniform over the block
+  FF acc{0.f, 0.f};
+  for (int m = tid; m < M; m += DR_NT) {
+    const float* pv = pval + ((size_t)n * M + m) * b;
+    float c = 1.f;
+    for (int i = 0; i < b; ++i) {
+      c *= pv[i];
+      acc = ff_addf(acc, c);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc = ff_add(acc, ff_shfl_xor(acc, o));
+  if (lane == 0) red[warp] = acc;
+  __syncthreads();
+  if (tid == 0) {
+    FF t{0.f, 0.f};
+    for (int w = 0; w < DR_NT / 32; ++w) t = ff_add(t, red[w]);
+    d_hat[n] = ff_f(t) / ((float)M * (float)b);
+  }
+}
+
+template <typename Tin>
+static cudaError_t determinism_typed(const StepCtx& c, const dblast_verify_out* o, int rows, int b,
+                                     int M, uint64_t seed, float* collision, float* d_exact,
+                                     float* d_hat, int32_t* samples, size_t off_pval) {
+  const WsLayout& w = c.wl;
+  cudaError_t e = launch_target_stats(c, o);
+  if (e == cudaSuccess && (d_hat || samples)) {
+    e = launch_dep(k_target_sample<Tin>, dim3(b, M, w.N), dim3(VF_NT), 0, c.stream,
+                   static_cast<const Tin*>(o->target), wsp<float2>(c, w.off_partt),
+                   wsp<float2>(c, w.off_lt2), w.V, w.nt, rows, b, M, w.Rt, c.k2, seed,
+                   wsp<float>(c, off_pval), samples);
+    debug_kernel("k_target_sample", c.stream);
+    count_launches(1);
+  }
+  if (e == cudaSuccess) {
+    e = launch_dep(k_determinism_reduce, dim3(w.N), dim3(DR_NT), 0, c.stream,
+                   wsp<float>(c, w.off_coll), wsp<float>(c, off_pval), rows, b, M, collision,
+                   d_exact, d_hat);
+    debug_kernel("k_determinism_reduce", c.stream);
+    count_launches(1);
+  }
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t launch_determinism(const StepCtx& c, const dblast_verify_out* o, int rows, int b,
+                               int M, uint64_t seed, float* collision, float* d_exact,
+                               float* d_hat, int32_t* samples, size_t off_pval) {
+  return c.head->dtype == DBLAST_F32
+             ? determinism_typed<float>(c, o, rows, b, M, seed, collision, d_exact, d_hat,
+                                        samples, off_pval)
+             : determinism_typed<__nv_bfloat16>(c, o, rows, b, M, seed, collision, d_exact, d_hat,
+                                                samples, off_pval);
 }
 
 }  // namespace dblast

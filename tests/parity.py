@@ -73,6 +73,9 @@ def compare(gpu, orc_list, seqs, stats=None):
         _close("accept_prob", gpu["accept_prob"][n][:j], o["accept_prob"][:j])
         _close("alpha", gpu["alpha"][n][:jj], o["alpha"][:jj], atol=1e-6)
         _close("lse_target", gpu["lse_target"][n], o["lse_target"], rtol=1e-5, atol=1e-4)
+        if "collision" in gpu:
+            _close("collision", gpu["collision"][n], o["collision"], atol=1e-7)
+            _close("determinism", gpu["determinism"][n], o["determinism"], atol=1e-7)
         stats["positions"] += j
         if j == B:
             _close("exp_len", gpu["exp_len"][n], o["exp_len"], atol=1e-6)
@@ -120,6 +123,9 @@ def compare_greedy(gpu, orc_list, seqs, stats=None):
         _close("accept_prob", gpu["accept_prob"][n][:j], o["accept_prob"][:j])
         _close("alpha", gpu["alpha"][n][:j], o["alpha"][:j], atol=1e-6)
         _close("lse_target", gpu["lse_target"][n], o["lse_target"], rtol=1e-5, atol=1e-4)
+        if "collision" in gpu:
+            _close("collision", gpu["collision"][n], o["collision"], atol=1e-7)
+            _close("determinism", gpu["determinism"][n], o["determinism"], atol=1e-7)
         stats["positions"] += j
         if j == B:
             _close("exp_len", gpu["exp_len"][n], o["exp_len"], atol=1e-6)

@@ -101,3 +101,19 @@ def test_status_strings():
     lib = bd.lib()
     for s in range(7):
         assert lib.dblast_status_string(s)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(b=0), 1), (dict(b=33, rows=40), 1), (dict(b=6, rows=5), 1),
+    (dict(M=0, d_hat=True), 1), (dict(T=0.0), 1), (dict(ws_bytes=0), 3),
+])
+def test_determinism_bad_arguments_are_rejected_before_launch(kw, status):
+    lib = bd.lib()
+    a = dict(N=2, rows=5, b=4, V=100, T=1.0, M=3, d_hat=False, ws_bytes=1 << 30)
+    a.update(kw)
+    p = ctypes.c_void_p(1 << 20)
+    got = lib.dblast_target_determinism(p, 0, a["N"], a["rows"], a["b"], a["V"], a["T"],
+                                        a["M"], 0, p, p, p if a["d_hat"] else None, None, p,
+                                        a["ws_bytes"], None)
+    assert got == status
+    assert lib.dblast_determinism_workspace_bytes(2, 17, 15, 151936, 20) > 2 * 17 * 1187 * 8
