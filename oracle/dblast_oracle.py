@@ -32,6 +32,8 @@ Definitions followed (section / equation of the paper):
   (Algorithm 1; Appendix A, "Distributional correctness").
 * Expected accepted length of the drafted block, sum_i prod_{j<=i} A_j
   (Eq. 3), and the overlap alpha_i = sum_v min(p_i(v), q(v|x_<i)).
+* Target sampling transform: temperature, top-k, top-p (Sec. 3.2, Sec. 4),
+  applied to every target row before verification (filter_target).
 * Target-block early determinism D_b and its M-sample estimator (App. B),
   for target rows that do not depend on the sampled prefix.
 * Greedy-branch mode (Sec. 3.1, "Drafter sampling during inference"; App. A,
@@ -170,8 +172,61 @@ def posterior(log_pi, logq_at_x):
     return logw
 
 
+def filter_target(t_row, T, top_k=0, top_p=0.0):
+    """The target sampling transform: temperature, then top-k, then top-p.
+
+    Sec. 3.2 / Sec. 4 (the target distribution after temperature, top-p and
+    top-k; top-k 20 with top-p 0.8 or 0.95 in every evaluation).  Readings
+    (the paper does not spell them out): top-k keeps the k largest logits,
+    ties at the k-th value going to the lower token index, so exactly
+    min(k, V) tokens stay (k = 0: off); top-p then orders the kept tokens by
+    probability (the same order) and keeps each token whose preceding
+    cumulative mass, renormalised over the top-k set, is below top_p (the
+    smallest prefix reaching top_p; 0 or >= 1: off).  The result is
+    renormalised over the kept set.  Returns (p' [V], kept token indices,
+    margin of the top-p cut: the distance of top_p to the nearest cumulative
+    mass that decides it, +inf when top-p is off).
+    """
+    t = f64(t_row)
+    V = t.shape[0]
+    st = t / T
+    p = np.exp(st - logsumexp(st))
+    order = np.lexsort((np.arange(V), -t))      # logit descending, index ascending
+    kk = V if (top_k <= 0 or top_k >= V) else int(top_k)
+    keep = order[:kk]
+    margin = np.inf
+    if 0.0 < top_p < 1.0:
+        pk = p[keep] / np.sum(p[keep])
+        before = np.concatenate([[0.0], np.cumsum(pk)[:-1]])
+        n_keep = int(np.sum(before < top_p))
+        margin = top_p - before[n_keep - 1]
+        if n_keep < kk:
+            margin = min(margin, before[n_keep] - top_p)
+        keep = keep[:n_keep]
+    out = np.zeros(V, dtype=np.float64)
+    out[keep] = p[keep] / np.sum(p[keep])
+    return out, keep, float(margin)
+
+
+def target_distributions(target, T, top_k, top_p, ties):
+    """p_i for every target row: softmax(t_i / T), filtered by top-k / top-p
+    when either is on (filter_target); a top-p cut within TIE_TOL is recorded
+    as a tie of kind "top_p" at row i.  Also returns the unfiltered natural
+    log-sum-exp of t_i / T."""
+    st = target / T
+    lse_t = logsumexp(st, axis=-1)
+    if top_k <= 0 and not (0.0 < top_p < 1.0):
+        return np.exp(st - lse_t[:, None]), lse_t
+    p = np.empty_like(st)
+    for i in range(target.shape[0]):
+        p[i], _, margin = filter_target(target[i], T, top_k, top_p)
+        if margin < TIE_TOL:
+            ties.append(("top_p", i, margin))
+    return p, lse_t
+
+
 def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
-                              seed, n, pos, round_):
+                              seed, n, pos, round_, top_k=0, top_p=0.0):
     """One draft+verify step for sequence n (all arrays fp64 numpy).
 
     head: dict with W [V,H] (any dtype), U, Vf [K,H,r], e [K,H]|None,
@@ -214,9 +269,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     q_tok = qmix[np.arange(B), tokens]
 
     # target distributions p_i = softmax(t_i / T)
-    st = target / T
-    lse_t = logsumexp(st, axis=-1)
-    p = np.exp(st - lse_t[:, None])                           # [B+hb, V]
+    p, lse_t = target_distributions(target, T, top_k, top_p, ties)  # [B+hb, V]
     p_tok = p[np.arange(B), tokens]
 
     alpha = np.sum(np.minimum(p[:B], qmix), axis=-1)
@@ -336,7 +389,7 @@ def greedy_conditional(pi, xhat, C, V):
 
 
 def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
-                                     seed, n, pos, round_):
+                                     seed, n, pos, round_, top_k=0, top_p=0.0):
     """One greedy-branch draft+verify step for sequence n (Algorithm 1 of App. A).
 
     Same inputs and outputs as draft_and_verify_sequence.  The category is
@@ -380,9 +433,7 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
         logw = np.log(pit)
 
     # target distributions p_i = softmax(t_i / T)
-    st = target / T
-    lse_t = logsumexp(st, axis=-1)
-    p = np.exp(st - lse_t[:, None])
+    p, lse_t = target_distributions(target, T, top_k, top_p, ties)
     p_tok = p[np.arange(B), tokens]
     alpha = np.sum(np.minimum(p[:B], q), axis=-1)
     ratio = p_tok / q_tok
@@ -497,12 +548,13 @@ def prepare_head(head):
 
 
 def draft_and_verify(head, hidden, anchor, target, has_bonus, T, Z_T, seed,
-                     pos, round_, seqs=None, mode="soft"):
+                     pos, round_, seqs=None, mode="soft", top_k=0, top_p=0.0):
     """Run the step for the sequences in ``seqs`` (default: all).
 
     hidden: [N, B, H]; anchor: [N, H] or None; target: [N, B+has_bonus, V];
     pos: [N] int; round_: [N] int; mode "soft" (tokens drawn from the branch
-    distributions) or "greedy" (greedy branches, App. A).  Returns a list of
+    distributions) or "greedy" (greedy branches, App. A); top_k / top_p: the
+    target filter of filter_target (0: off).  Returns a list of
     per-sequence dicts (see draft_and_verify_sequence and
     greedy_draft_and_verify_sequence) in the order of ``seqs``.
     """
@@ -518,7 +570,7 @@ def draft_and_verify(head, hidden, anchor, target, has_bonus, T, Z_T, seed,
         t = f64(target[n])
         out.append(step(
             hd, h, a, t, bool(has_bonus), float(T), float(Z_T), int(seed),
-            int(n), int(pos[n]), int(round_[n])))
+            int(n), int(pos[n]), int(round_[n]), int(top_k), float(top_p)))
     return out
 
 

@@ -61,7 +61,7 @@ def compare(gpu, orc_list, seqs, stats=None):
             continue
         assert int(gpu["z_hat"][n]) == o["zhat"], ("z_hat", n)
         _close("pi", gpu["pi"][n], o["pi"], atol=1e-7)
-        j = min([i for k, i, _ in ties if k == "draft"], default=B)
+        j = min([i for k, i, _ in ties if k in ("draft", "top_p")], default=B)
         _close("lse", gpu["lse"][n], o["lse"], rtol=1e-5, atol=1e-4)
         assert list(gpu["tokens"][n][:j].tolist()) == [int(x) for x in o["tokens"][:j]], \
             ("tokens", n, gpu["tokens"][n].tolist(), o["tokens"].tolist())
@@ -112,7 +112,7 @@ def compare_greedy(gpu, orc_list, seqs, stats=None):
             continue
         assert int(gpu["z_hat"][n]) == o["zhat"], ("z_hat", n)
         _close("pi", gpu["pi"][n], o["pi"], atol=1e-7)
-        j = min([i for k, i, _ in ties if k == "greedy"], default=B)
+        j = min([i for k, i, _ in ties if k in ("greedy", "top_p")], default=B)
         assert list(gpu["tokens"][n][:j].tolist()) == [int(x) for x in o["tokens"][:j]], \
             ("tokens", n, gpu["tokens"][n].tolist(), o["tokens"].tolist())
         jj = min(j + 1, B)
