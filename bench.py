@@ -104,7 +104,7 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
-def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft"):
+def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft", top_k=0, top_p=0.0):
     """Time the fp64 oracle, as it stands, on one sequence of the workload."""
     import torch
     from oracle import dblast_oracle as orc
@@ -117,7 +117,7 @@ def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft"):
     while True:
         orc.draft_and_verify(head_cpu, blk_cpu["hidden"], None, blk_cpu["target"],
                              blk_cpu["has_bonus"], T, Z_T, 0, pos.numpy(), rnd.numpy(),
-                             seqs=[n_done % cfg["N"]], mode=mode)
+                             seqs=[n_done % cfg["N"]], mode=mode, top_k=top_k, top_p=top_p)
         n_done += 1
         el = time.perf_counter() - t0
         if el > budget_s / 3 or n_done >= 4:
@@ -326,6 +326,10 @@ def main():
     ap.add_argument("--config", default="qwen3_8b_b32")
     ap.add_argument("--T", type=float, default=1.0)
     ap.add_argument("--kernels", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--top-k", type=int, default=0,
+                    help="target filter: top-k (0 = off; the paper uses 20)")
+    ap.add_argument("--top-p", type=float, default=0.0,
+                    help="target filter: top-p (0 = off; the paper uses 0.8 / 0.95)")
     ap.add_argument("--mode", default="soft", choices=["soft", "greedy"],
                     help="draft tokens sampled from the z-hat branch (soft) or the "
                          "greedy-branch decoder")
@@ -392,7 +396,8 @@ def main():
     def step(vout):
         dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, args.T, cfg["Z_T"], seed,
                                 blk["target"], blk["has_bonus"], impl=args.kernels,
-                                dout=dout, vout=vout, mode=args.mode)
+                                dout=dout, vout=vout, mode=args.mode, top_k=args.top_k,
+                                top_p=args.top_p)
 
     for _ in range(args.warmup):
         step(vouts[0])
@@ -466,7 +471,7 @@ def main():
         main.wait_event(copied[b])
         dblast_draft_and_verify(head, ws, h_dev[b], pos, rnd, args.T, cfg["Z_T"], seed, t_dev[b],
                                 blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0],
-                                mode=args.mode)
+                                mode=args.mode, top_k=args.top_k, top_p=args.top_p)
         freed[b].record(main)
         for kk, v in res_host.items():
             v.copy_(vouts[0][kk], non_blocking=True)
@@ -505,7 +510,8 @@ def main():
             "dtype": "bf16" if cfg["dtype"] == "bf16" else "f32", "data": "synthetic",
             "config": {"workload": cfg["name"], "N": N, "B": B, "K": cfg["K"], "r": cfg["r"],
                        "H": cfg["H"], "V": cfg["V"], "T": args.T, "Z_T": cfg["Z_T"],
-                       "sigma": cfg["sigma"], "mode": args.mode,
+                       "sigma": cfg["sigma"], "mode": args.mode, "top_k": args.top_k,
+                       "top_p": args.top_p,
                        "kernels": "tcgen05" if st["tc_launches"] > 0 else "simt",
                        "parallelism": "replicas" if world > 1 else "single",
                        "l2": "no flush: inputs larger than L2 (W %.2f GB, target %.0f MB)" % (
@@ -532,7 +538,8 @@ def main():
         }
         if world == 1 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline(cfg, head_t, blk, args.T, cfg["Z_T"],
-                                                mode=args.mode)
+                                                mode=args.mode, top_k=args.top_k,
+                                                top_p=args.top_p)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

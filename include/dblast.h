@@ -154,6 +154,19 @@ typedef struct {
   float* determinism;   /* [N]        target-block early determinism D_B = (1/B) sum_j prod_{i<=j}
                                        collision_i (App. B, Eq. appendix-early-determinism, for
                                        target rows that do not depend on the drafted prefix) */
+  /* Target filter (inputs), applied to every target row after the temperature
+   * and before verification (Sec. 3.2, Sec. 4: temperature, top-k, top-p):
+   * top-k keeps the k largest logits, ties at the k-th value to the lower
+   * token index (0 or >= V: off); top-p then keeps, in the order (logit desc,
+   * index asc), every token whose preceding mass renormalised over the
+   * top-k set is below top_p (0 or >= 1: off).  p' is renormalised over the
+   * kept set and used for p_tok, acceptance, alpha, the residual, the bonus
+   * token and collision/determinism; lse_target stays the unfiltered
+   * log-sum-exp.  With a filter on, at most 256 tokens may stay (top-p needs
+   * top_k in 1..256, or V <= 256) and V <= 524288; else DBLAST_ERR_UNSUPPORTED.
+   * tie_flags bit5: a top-p cut within 1e-6 of top_p on some row. */
+  int top_k;
+  float top_p;
 } dblast_verify_out;
 
 /* Bytes of the prep buffer for this head (depends on V, K, r, e != NULL). */

@@ -19,7 +19,7 @@ DTYPES = {torch.bfloat16: 0, torch.float32: 1}
 IMPLS = {"auto": 0, "simt": 1, "tcgen05": 2}
 MODES = {"soft": 0, "greedy": 1}
 
-TIE_ZHAT, TIE_DRAFT, TIE_ACCEPT, TIE_RESID, TIE_RMASS = 1, 2, 4, 8, 16
+TIE_ZHAT, TIE_DRAFT, TIE_ACCEPT, TIE_RESID, TIE_RMASS, TIE_TOPP = 1, 2, 4, 8, 16, 32
 
 
 class DBLastError(RuntimeError):
@@ -64,7 +64,9 @@ class CVerifyOut(ctypes.Structure):
     _fields_ = [("target", ctypes.c_void_p), ("has_bonus", ctypes.c_int)] + [
         (n, ctypes.c_void_p) for n in
         ("p_tok", "accept_prob", "alpha", "lse_target", "accepted", "emitted",
-         "n_emitted", "exp_len", "alpha_len", "tie_flags", "collision", "determinism")]
+         "n_emitted", "exp_len", "alpha_len", "tie_flags", "collision", "determinism")] + [
+        ("top_k", ctypes.c_int), ("top_p", ctypes.c_float)]
+    POINTERS = 12  # the output pointers after (target, has_bonus)
 
 
 EXPORTS = ["dblast_prep_bytes", "dblast_workspace_bytes", "dblast_head_prepare",
@@ -265,10 +267,11 @@ def _draft_struct(d):
     return CDraftOut(*[_ptr(d.get(k)) for k, _ in CDraftOut._fields_])
 
 
-def _verify_struct(target, has_bonus, v):
+def _verify_struct(target, has_bonus, v, top_k=0, top_p=0.0):
     v = v or {}
-    return CVerifyOut(_ptr(target), int(has_bonus),
-                      *[_ptr(v.get(k)) for k, _ in CVerifyOut._fields_[2:]])
+    names = [k for k, _ in CVerifyOut._fields_[2:2 + CVerifyOut.POINTERS]]
+    return CVerifyOut(_ptr(target), int(has_bonus), *[_ptr(v.get(k)) for k in names],
+                      int(top_k), float(top_p))
 
 
 def dblast_draft_block(head, ws, hidden, pos, round_, T, Z_T, seed, anchor=None,
@@ -284,14 +287,14 @@ def dblast_draft_block(head, ws, hidden, pos, round_, T, Z_T, seed, anchor=None,
 
 
 def dblast_verify_block(head, ws, hidden, pos, round_, T, Z_T, seed, target, has_bonus,
-                        anchor=None, impl="auto", out=None, mode="soft"):
+                        anchor=None, impl="auto", out=None, mode="soft", top_k=0, top_p=0.0):
     args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode)
     N, B, _ = hidden.shape
     _cuda_contig(target, "target", head.dtype)
     if tuple(target.shape) != (N, B + int(has_bonus), head.V):
         raise ValueError("target must be [N, B + has_bonus, V]")
     out = out if out is not None else alloc_verify_out(N, B, has_bonus, hidden.device)
-    v = _verify_struct(target, has_bonus, out)
+    v = _verify_struct(target, has_bonus, out, top_k, top_p)
     _check(lib().dblast_verify_block(ctypes.byref(head.c), ctypes.byref(args),
                                      ctypes.byref(v), ws.ptr, ws.nbytes, _stream()),
            "dblast_verify_block")
@@ -300,9 +303,10 @@ def dblast_verify_block(head, ws, hidden, pos, round_, T, Z_T, seed, target, has
 
 def dblast_draft_and_verify(head, ws, hidden, pos, round_, T, Z_T, seed, target,
                             has_bonus, anchor=None, impl="auto", dout=None, vout=None,
-                            mode="soft"):
+                            mode="soft", top_k=0, top_p=0.0):
     """One fused draft+verify step; returns (draft_out, verify_out) dicts.
-    mode: "soft" (sampled draft tokens) or "greedy" (greedy branches)."""
+    mode: "soft" (sampled draft tokens) or "greedy" (greedy branches);
+    top_k / top_p: the target filter (0: off)."""
     args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, mode)
     N, B, _ = hidden.shape
     _cuda_contig(target, "target", head.dtype)
@@ -311,7 +315,7 @@ def dblast_draft_and_verify(head, ws, hidden, pos, round_, T, Z_T, seed, target,
     dout = dout if dout is not None else alloc_draft_out(N, B, head.K, hidden.device, mode)
     vout = vout if vout is not None else alloc_verify_out(N, B, has_bonus, hidden.device)
     d = _draft_struct(dout)
-    v = _verify_struct(target, has_bonus, vout)
+    v = _verify_struct(target, has_bonus, vout, top_k, top_p)
     _check(lib().dblast_draft_and_verify(ctypes.byref(head.c), ctypes.byref(args),
                                          ctypes.byref(d), ctypes.byref(v), ws.ptr,
                                          ws.nbytes, _stream()),

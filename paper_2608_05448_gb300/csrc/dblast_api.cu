@@ -145,6 +145,10 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_xhat = take((size_t)w.M * K * sizeof(int32_t));
   w.off_cmask = take((size_t)w.M * sizeof(uint32_t));
   w.off_coll = take((size_t)w.Rt * sizeof(float));
+  w.off_ftok = take((size_t)w.Rt * FILTER_MAX_K * sizeof(int32_t));
+  w.off_fp = take((size_t)w.Rt * FILTER_MAX_K * sizeof(float));
+  w.off_fcnt = take((size_t)w.Rt * sizeof(int32_t));
+  w.off_ftie = take((size_t)w.Rt * sizeof(uint32_t));
   w.total = o;
   return w;
 }
@@ -215,6 +219,28 @@ static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, 
   return DBLAST_OK;
 }
 
+// top-k / top-p of a verify call: on, and the number of tokens it keeps at most
+static bool filter_on(const dblast_head* h, const dblast_verify_out* o) {
+  const bool k_on = o->top_k >= 1 && o->top_k < h->V;
+  const bool p_on = o->top_p > 0.f && o->top_p < 1.f;
+  return k_on || p_on;
+}
+static dblast_status check_filter(const dblast_head* h, const dblast_verify_out* o) {
+  if (o->top_k < 0 || !(o->top_p >= 0.f)) return DBLAST_ERR_INVALID_ARG;
+  if (!filter_on(h, o)) return DBLAST_OK;
+  const int k_eff = (o->top_k >= 1 && o->top_k < h->V) ? o->top_k : h->V;
+  if (k_eff > FILTER_MAX_K || ceil_div(h->V, TILE_V) > FILTER_MAX_TILES)
+    return DBLAST_ERR_UNSUPPORTED;
+  return DBLAST_OK;
+}
+// the dblast_verify_out the filter kernel reads: top_k clamped to what stays
+static dblast_verify_out filter_args(const dblast_head* h, const dblast_verify_out* o) {
+  dblast_verify_out f = *o;
+  f.top_k = (o->top_k >= 1 && o->top_k < h->V) ? o->top_k : h->V;
+  if (!(f.top_p > 0.f && f.top_p < 1.f)) f.top_p = 1.f;
+  return f;
+}
+
 static dblast_status cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return DBLAST_OK;
   fprintf(stderr, "dblast: CUDA error %s\n", cudaGetErrorString(e));
@@ -260,6 +286,12 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
 }
 
 static cudaError_t verify_passes(const StepCtx& c, dblast_verify_out* out) {
+  // with a target filter p' has at most k tokens: one kernel verifies against
+  // it in either mode (the filter itself ran after the target statistics)
+  if (filter_on(c.head, out)) {
+    const dblast_verify_out f = filter_args(c.head, out);
+    return dbg(launch_filtered_verify(c, &f), "filtered_verify", c.stream);
+  }
   // greedy-branch mode has no vocabulary-wide verify pass: q_greedy has at
   // most K atoms, so one kernel reads p at them and draws the residual
   if (c.greedy) return dbg(launch_greedy_verify_finalize(c, out), "verify_finalize", c.stream);
@@ -276,6 +308,10 @@ static dblast_status verify_impl(StepCtx c, dblast_verify_out* out) {
   c.Bt = c.args->B + (out->has_bonus ? 1 : 0);
   g_calls.fetch_add(1, std::memory_order_relaxed);
   cudaError_t e = dbg(launch_target_stats(c, out), "target_stats", c.stream);
+  if (e == cudaSuccess && filter_on(c.head, out)) {
+    const dblast_verify_out f = filter_args(c.head, out);
+    e = dbg(launch_target_filter(c, &f), "target_filter", c.stream);
+  }
   if (e == cudaSuccess) e = verify_passes(c, out);
   return cuda_status(e);
 }
@@ -342,6 +378,10 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   if (e == cudaSuccess) e = cudaEventRecord(ss->ev[2], c.stream);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[2], 0);
   if (e == cudaSuccess) e = launch_target_stats(side, vout);
+  if (e == cudaSuccess && filter_on(c.head, vout)) {
+    const dblast_verify_out f = filter_args(c.head, vout);
+    e = launch_target_filter(side, &f);
+  }
   if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
   if (e == cudaSuccess)
     e = c.greedy ? launch_greedy_draft_finalize(c, dout) : launch_draft_finalize(c, dout);
@@ -370,6 +410,8 @@ dblast_status dblast_verify_block(const dblast_head* h, const dblast_block_args*
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
   if (!out || !out->target || !aligned16(out->target)) return DBLAST_ERR_INVALID_ARG;
+  st = check_filter(h, out);
+  if (st != DBLAST_OK) return st;
   StepCtx c;
   st = make_ctx(h, a, ws, ws_bytes, out->has_bonus ? 1 : 0, stream, &c);
   if (st != DBLAST_OK) return st;
@@ -383,6 +425,8 @@ dblast_status dblast_draft_and_verify(const dblast_head* h, const dblast_block_a
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
   if (!vout || !vout->target || !aligned16(vout->target)) return DBLAST_ERR_INVALID_ARG;
+  st = check_filter(h, vout);
+  if (st != DBLAST_OK) return st;
   StepCtx c;
   st = make_ctx(h, a, ws, ws_bytes, vout->has_bonus ? 1 : 0, stream, &c);
   if (st != DBLAST_OK) return st;

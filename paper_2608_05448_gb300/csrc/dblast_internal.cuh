@@ -21,8 +21,13 @@ constexpr float LN2 = 0.6931471805599453f;
 constexpr float TIE_TOL = 1e-6f;
 
 enum TieBits : uint32_t {
-  TIE_ZHAT = 1u, TIE_DRAFT = 2u, TIE_ACCEPT = 4u, TIE_RESID = 8u, TIE_RMASS = 16u
+  TIE_ZHAT = 1u, TIE_DRAFT = 2u, TIE_ACCEPT = 4u, TIE_RESID = 8u, TIE_RMASS = 16u, TIE_TOPP = 32u
 };
+
+// target filter (top-k / top-p): at most FILTER_MAX_K kept tokens per row,
+// and vocabularies of at most FILTER_MAX_TILES tiles
+constexpr int FILTER_MAX_K = 256;
+constexpr int FILTER_MAX_TILES = 4096;
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -49,13 +54,16 @@ struct PrepLayout {
 //   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
 //   token and the consistent-branch set C_i as a bit mask over z)
 //   coll f32 [Rt]  (collision probability sum_v p(v)^2 of every target row)
+//   ftok i32 [Rt, FILTER_MAX_K] | fp f32 [Rt, FILTER_MAX_K] | fcnt i32 [Rt] | ftie u32 [Rt]
+//   (target filter: kept tokens by index, their filtered probabilities, count, top-p tie)
 constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
 constexpr int AV_SPLIT = 8;   // partial sums of the verify records per row
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
       off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
-      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, off_coll, total;
+      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, off_coll, off_ftok,
+      off_fp, off_fcnt, off_ftie, total;
 };
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
@@ -288,6 +296,8 @@ cudaError_t launch_verify_pass_simt(const StepCtx& c);
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
 cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* out);
 cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
+cudaError_t launch_target_filter(const StepCtx& c, const dblast_verify_out* o);
+cudaError_t launch_filtered_verify(const StepCtx& c, const dblast_verify_out* o);
 cudaError_t launch_determinism(const StepCtx& c, const dblast_verify_out* o, int rows, int b,
                                int M, uint64_t seed, float* collision, float* d_exact,
                                float* d_hat, int32_t* samples, size_t off_pval);

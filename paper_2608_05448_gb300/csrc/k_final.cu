@@ -1492,4 +1492,554 @@ cudaError_t launch_determinism(const StepCtx& c, const dblast_verify_out* o, int
                                                 samples, off_pval);
 }
 
+// ---------------------------------------------------------------- target filter
+// Sec. 3.2 / Sec. 4: verification against the target after temperature,
+// top-k and top-p.  k_target_filter (one block per target row) finds the kept
+// set from the tile records of the target statistics: the k largest logits
+// (ties to the lower index) lie in the tiles whose maximum is at least the
+// k-th largest tile maximum, so only those tiles are read.  A radix select
+// on order-preserving keys gives the k-th largest value and how many of its
+// equal values are needed; an ordered compaction (two passes over per-warp
+// segments, ballots for the in-order ranks) lists the kept tokens by index.
+// top-p ranks the k tokens by (logit desc, index asc) and keeps those whose
+// preceding mass is below top_p.  Output per row: kept tokens by index,
+// p' renormalised over them, sum p'^2, and a flag for a top-p cut within
+// TIE_TOL.  k_filtered_verify then verifies against p' (its support has at
+// most k tokens, so no vocabulary-wide pass is needed in either mode).
+constexpr int TF_NT = 256;
+constexpr int TF_W = TF_NT / 32;
+
+__device__ __forceinline__ uint32_t fkey(float f) {
+  if (f == 0.f) f = 0.f;  // -0 ranks with +0
+  const uint32_t b = __float_as_uint(f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+struct FilterShared {
+  int hist[256];
+  int wcnt[TF_W][2];
+  int wbase[TF_W][2];
+  int digit, above;
+  int C;
+  uint32_t tie;
+  FF red[TF_W];
+  float smax;
+};
+
+// The key of the k-th largest (1-based) of n keys get(i), and in *rem how many
+// elements equal to that key belong to the k largest.
+template <typename GET>
+__device__ uint32_t radix_kth_largest(int n, int k, const GET& get, FilterShared& sh, int* rem) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  uint32_t prefix = 0u, mask = 0u;
+  int r = k;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int b = tid; b < 256; b += TF_NT) sh.hist[b] = 0;
+    __syncthreads();
+    for (int i = tid; i < n; i += TF_NT) {
+      const uint32_t key = get(i);
+      if ((key & mask) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // lane l owns digits 255 - 8l ... 248 - 8l (descending)
+      int c[8], loc = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = sh.hist[255 - 8 * lane - j];
+        loc += c[j];
+      }
+      int incl = loc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(FULLMASK, incl, o);
+        if (lane >= o) incl += t;
+      }
+      const int excl = incl - loc;
+      const unsigned hit = __ballot_sync(FULLMASK, incl >= r);
+      const int l0 = hit ? __ffs(hit) - 1 : 31;
+      if (lane == l0) {
+        int acc = excl, j = 0;
+        while (j < 7 && acc + c[j] < r) acc += c[j++];
+        sh.digit = 255 - 8 * lane - j;
+        sh.above = acc;
+      }
+    }
+    __syncthreads();
+    prefix |= (uint32_t)sh.digit << shift;
+    mask |= 255u << shift;
+    r -= sh.above;
+    __syncthreads();
+  }
+  *rem = r;
+  return prefix;
+}
+
+// Ordered compaction in two passes over per-warp segments of n elements:
+// cls(i) = 0 (drop), 1 (keep), 2 (keep if among the first `E` of class 2 in
+// index order); emit(i, pos) is called for every kept element with its rank.
+template <typename CLS, typename EMIT>
+__device__ int ordered_compact(int n, int E, const CLS& cls, const EMIT& emit, FilterShared& sh) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int seg = ceil_div(ceil_div(n, TF_W), 32) * 32;
+  const int s0 = min(n, warp * seg), s1 = min(n, s0 + seg);
+  int c1 = 0, c2 = 0;
+  for (int b = s0; b < s1; b += 32) {
+    const int i = b + lane;
+    const int c = i < s1 ? cls(i) : 0;
+    c1 += __popc(__ballot_sync(FULLMASK, c == 1));
+    c2 += __popc(__ballot_sync(FULLMASK, c == 2));
+  }
+  if (lane == 0) {
+    sh.wcnt[warp][0] = c1;
+    sh.wcnt[warp][1] = c2;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int a = 0, b = 0;
+    for (int w = 0; w < TF_W; ++w) {
+      sh.wbase[w][0] = a;
+      sh.wbase[w][1] = b;
+      a += sh.wcnt[w][0];
+      b += sh.wcnt[w][1];
+    }
+    sh.C = a + min(b, E);
+  }
+  __syncthreads();
+  int b1 = sh.wbase[warp][0], b2 = sh.wbase[warp][1];
+  const unsigned lt = (1u << lane) - 1u;
+  for (int b = s0; b < s1; b += 32) {
+    const int i = b + lane;
+    const int c = i < s1 ? cls(i) : 0;
+    const unsigned m1 = __ballot_sync(FULLMASK, c == 1), m2 = __ballot_sync(FULLMASK, c == 2);
+    const int r1 = b1 + __popc(m1 & lt), r2 = b2 + __popc(m2 & lt);
+    if (c == 1 || (c == 2 && r2 < E)) emit(i, r1 + min(r2, E));
+    b1 += __popc(m1);
+    b2 += __popc(m2);
+  }
+  const int total = sh.C;
+  __syncthreads();
+  return total;
+}
+
+template <typename Tin>
+__global__ void __launch_bounds__(TF_NT)
+    k_target_filter(const Tin* __restrict__ target, const float2* __restrict__ partt, int V,
+                    int nt, int B, int Bt, int Rt, int kf, float top_p, float k2,
+                    int32_t* __restrict__ ftok, float* __restrict__ fp, int32_t* __restrict__ fcnt,
+                    float* __restrict__ coll, uint32_t* __restrict__ ftie) {
+  __shared__ FilterShared sh;
+  __shared__ int clist[FILTER_MAX_TILES];
+  __shared__ int stok[FILTER_MAX_K];
+  __shared__ float sval[FILTER_MAX_K];
+  __shared__ float sw[FILTER_MAX_K];
+  __shared__ FF scum[FILTER_MAX_K];
+  __shared__ int skeep[FILTER_MAX_K];
+  const int row = blockIdx.x, tid = threadIdx.x;
+  const int n = row / Bt, i = row - n * Bt;
+  const int rl = n * (B + 1) + i;
+  const Tin* tr = target + (size_t)row * V;
+  const int k = min(kf, V);
+  // candidate tiles: maximum >= the k-th largest tile maximum
+  uint32_t theta = 0u;
+  if (k < nt) {
+    int rem;
+    theta = radix_kth_largest(nt, k, [&](int t) { return fkey(partt[(size_t)t * Rt + rl].x); },
+                              sh, &rem);
+  }
+  const int C = ordered_compact(
+      nt, 0, [&](int t) { return fkey(partt[(size_t)t * Rt + rl].x) >= theta ? 1 : 0; },
+      [&](int t, int pos) { clist[pos] = t; }, sh);
+  // the k-th largest logit of the candidate tiles, and its equal values needed
+  auto cand = [&](int j) {
+    const int v = clist[j >> 7] * TILE_V + (j & (TILE_V - 1));
+    return v < V ? fkey(ldf(tr + v)) : 0u;
+  };
+  int E;
+  const uint32_t tau = radix_kth_largest(C * TILE_V, k, cand, sh, &E);
+  // kept tokens in index order
+  const int cnt = ordered_compact(
+      C * TILE_V, E,
+      [&](int j) {
+        const int v = clist[j >> 7] * TILE_V + (j & (TILE_V - 1));
+        if (v >= V) return 0;
+        const uint32_t key = fkey(ldf(tr + v));
+        return key > tau ? 1 : (key == tau ? 2 : 0);
+      },
+      [&](int j, int pos) {
+        const int v = clist[j >> 7] * TILE_V + (j & (TILE_V - 1));
+        stok[pos] = v;
+        sval[pos] = ldf(tr + v);
+      },
+      sh);
+  __syncthreads();
+  // weights relative to the largest kept logit
+  if (tid == 0) {
+    float m = -INFINITY;
+    for (int j = 0; j < cnt; ++j) m = fmaxf(m, sval[j]);
+    sh.smax = m;
+  }
+  __syncthreads();
+  const FF cmax = ff_prod(sh.smax, k2);
+  for (int j = tid; j < cnt; j += TF_NT)
+    sw[j] = (sval[j] == -INFINITY || sh.smax == -INFINITY) ? 0.f : exp2_rel(sval[j], k2, cmax);
+  __syncthreads();
+  // top-p: rank by (logit desc, index asc), cumulative mass before each rank
+  const bool use_p = top_p > 0.f && top_p < 1.f;
+  if (tid == 0) sh.tie = 0u;
+  if (use_p) {
+    for (int j = tid; j < cnt; j += TF_NT) {
+      int rk = 0;
+      for (int l = 0; l < cnt; ++l)
+        rk += (sval[l] > sval[j] || (sval[l] == sval[j] && stok[l] < stok[j])) ? 1 : 0;
+      skeep[j] = rk;
+    }
+    __syncthreads();
+    for (int j = tid; j < cnt; j += TF_NT) scum[skeep[j]] = FF{sw[j], 0.f};
+    __syncthreads();
+    if (tid == 0) {  // exclusive prefix sums in rank order (k <= FILTER_MAX_K)
+      FF acc{0.f, 0.f};
+      for (int r = 0; r < cnt; ++r) {
+        const FF w = scum[r];
+        scum[r] = acc;
+        acc = ff_add(acc, w);
+      }
+      sh.red[0] = acc;
+    }
+    __syncthreads();
+    const FF W = sh.red[0];
+    const FF thr = ff_mulf(W, top_p);
+    const float Wf = ff_f(W);
+    for (int j = tid; j < cnt; j += TF_NT) {
+      const FF before = scum[skeep[j]];
+      skeep[j] = ff_gt(thr, before) ? 1 : 0;
+      if (fabsf(ff_f(ff_sub(before, thr))) < TIE_TOL * Wf) atomicOr(&sh.tie, 1u);
+    }
+  } else {
+    for (int j = tid; j < cnt; j += TF_NT) skeep[j] = 1;
+  }
+  __syncthreads();
+  // renormalise over the kept tokens, collision probability, ordered output
+  if (tid < 32) {
+    FF Wk{0.f, 0.f};
+    for (int j = tid; j < cnt; j += 32)
+      if (skeep[j]) Wk = ff_addf(Wk, sw[j]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) Wk = ff_add(Wk, ff_shfl_xor(Wk, o));
+    const float inv = 1.f / ff_f(Wk);
+    float c2 = 0.f;
+    int base = 0;
+    for (int j0 = 0; j0 < cnt; j0 += 32) {
+      const int j = j0 + tid;
+      const bool kp = j < cnt && skeep[j];
+      const unsigned m = __ballot_sync(FULLMASK, kp);
+      if (kp) {
+        const int pos = base + __popc(m & ((1u << tid) - 1u));
+        const float pj = sw[j] * inv;
+        ftok[(size_t)rl * FILTER_MAX_K + pos] = stok[j];
+        fp[(size_t)rl * FILTER_MAX_K + pos] = pj;
+        c2 = fmaf(pj, pj, c2);
+      }
+      base += __popc(m);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c2 += __shfl_xor_sync(FULLMASK, c2, o);
+    if (tid == 0) {
+      fcnt[rl] = base;
+      coll[rl] = c2;
+      ftie[rl] = sh.tie;
+    }
+  }
+}
+
+// q(v|x_<i) at one token for the verify kernels: the soft mixture from the
+// stash and the branch corrections, or q_greedy from the consistent branches.
+struct SoftQ {
+  const float* srow;  // stash row of position i
+  const float* wu;
+  const float* cm;    // codes of position i, [K, rr]
+  const FF* Cz;       // [K] L_z - log2 w_z (+inf if w_z = 0)
+  int K, rr;
+  float k2;
+  __device__ float operator()(int v) const {
+    float q = 0.f;
+    const float base = srow[v];
+    for (int z = 0; z < K; ++z) {
+      const FF c = Cz[z];
+      if (c.hi == INFINITY) continue;
+      q += exp2_rel2(base, corr_at(wu, cm + z * rr, v, z, K, rr), k2, c);
+    }
+    return q;
+  }
+};
+struct GreedyQ {
+  const int* X;       // x-hat of position i, [K]
+  const float* pi;
+  uint32_t c;         // C_i
+  float S;            // sum of pi over C_i
+  int K;
+  __device__ float operator()(int v) const {
+    float q = 0.f;
+    for (int z = 0; z < K; ++z)
+      if (((c >> z) & 1u) && X[z] == v) q += pi[z];
+    return S > 0.f ? q / S : 0.f;
+  }
+};
+
+// Inverse CDF over at most FILTER_MAX_K masses in index order by one warp:
+// the smallest j whose cumulative mass exceeds u times the total (the
+// total is the warp's own sum).  Returns j (-1 if the total is 0) and the
+// margin of the decision relative to the total.
+template <typename MASS>
+__device__ int warp_inverse_cdf(int cnt, const MASS& mass, float u, float* margin, float* total) {
+  const int lane = threadIdx.x & 31;
+  FF tot{0.f, 0.f};
+  for (int j = lane; j < cnt; j += 32) tot = ff_addf(tot, mass(j));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tot = ff_add(tot, ff_shfl_xor(tot, o));
+  *total = ff_f(tot);
+  *margin = 0.f;
+  if (!(tot.hi > 0.f)) return -1;
+  const FF target = ff_mulf(tot, u);
+  FF base{0.f, 0.f};
+  int last = -1;
+  for (int j0 = 0; j0 < cnt; j0 += 32) {
+    const int j = j0 + lane;
+    const float w = j < cnt ? mass(j) : 0.f;
+    FF incl{w, 0.f};
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const FF t = ff_shfl_up(incl, o);
+      if (lane >= o) incl = ff_add(t, incl);
+    }
+    FF ex1 = ff_shfl_up(incl, 1);
+    if (lane == 0) ex1 = FF{0.f, 0.f};
+    const FF hi = ff_add(base, incl), lo = ff_add(base, ex1);
+    const unsigned hit = __ballot_sync(FULLMASK, j < cnt && ff_gt(hi, target));
+    const unsigned pos = __ballot_sync(FULLMASK, j < cnt && w > 0.f);
+    if (pos) last = j0 + 31 - __clz(pos);
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      const float m = fminf(ff_f(ff_sub(target, lo)), ff_f(ff_sub(hi, target))) / ff_f(tot);
+      *margin = __shfl_sync(FULLMASK, m, l);
+      return j0 + l;
+    }
+    base = FF{__shfl_sync(FULLMASK, hi.hi, 31), __shfl_sync(FULLMASK, hi.lo, 31)};
+  }
+  return last;  // rounding left the target at the total: the last positive mass
+}
+
+// One block per sequence: verification against the filtered target p'.
+// alpha_i and the residual mass need q only at the kept tokens of row i.
+template <bool GREEDY>
+__global__ void __launch_bounds__(VF_NT)
+    k_filtered_verify(const int32_t* __restrict__ ftok, const float* __restrict__ fp,
+                      const int32_t* __restrict__ fcnt, const uint32_t* __restrict__ ftie,
+                      const float* __restrict__ coll, const float* __restrict__ stash,
+                      const float* __restrict__ wu, const float* __restrict__ codes,
+                      const float2* __restrict__ lse2, const float2* __restrict__ w2,
+                      const int32_t* __restrict__ xhat, const uint32_t* __restrict__ cmask,
+                      const float* __restrict__ log2pi, const float* __restrict__ qtok_ws,
+                      const int32_t* __restrict__ tok, const uint32_t* __restrict__ ties_draft,
+                      int V, int K, int rr, int B, int Bt, float k2, uint64_t seed,
+                      int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
+                      dblast_verify_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ FF Cz[32][32];       // soft: per position, L_z - log2 w_z
+  __shared__ int X[1024];         // greedy: x-hat [B, K]
+  __shared__ float piS[32], Ssum[32];
+  __shared__ float alphaS[32];
+  __shared__ int sL, sx;
+  __shared__ uint32_t sties;
+  const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t p0 = pos[n];
+  const uint32_t rd = rnd[n];
+  const size_t m0 = (size_t)n * B;
+  if (GREEDY) {
+    for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[m0 * K + j];
+    if (tid < K) piS[tid] = exp2f(log2pi[n * K + tid]);
+  } else {
+    for (int j = tid; j < B * K; j += VF_NT) {
+      const int i = j / K, z = j - i * K;
+      const FF wz = ff_ld(w2 + (m0 + i) * K + z);
+      Cz[i][z] = (wz.hi == -INFINITY) ? FF{INFINITY, 0.f} : ff_sub(ff_ld(lse2 + (m0 + i) * K + z), wz);
+    }
+  }
+  __syncthreads();
+  if (GREEDY && tid < B) {
+    const uint32_t c = cmask[m0 + tid];
+    float S = 0.f;
+    for (int z = 0; z < K; ++z)
+      if ((c >> z) & 1u) S += piS[z];
+    Ssum[tid] = S;
+  }
+  __syncthreads();
+  auto qfun = [&](int i, int v) -> float {
+    if constexpr (GREEDY) {
+      return GreedyQ{X + i * K, piS, cmask[m0 + i], Ssum[i], K}(v);
+    } else {
+      return SoftQ{stash + (m0 + i) * V, wu, codes + (m0 + i) * K * rr, Cz[i], K, rr, k2}(v);
+    }
+  };
+  // alpha_i = sum over the kept tokens of min(p'(v), q(v)): one warp per position
+  for (int i = warp; i < B; i += VF_NT / 32) {
+    const int rl = n * (B + 1) + i;
+    const int cnt = fcnt[rl];
+    FF a{0.f, 0.f};
+    for (int j = lane; j < cnt; j += 32) {
+      const int v = ftok[(size_t)rl * FILTER_MAX_K + j];
+      a = ff_addf(a, fminf(fp[(size_t)rl * FILTER_MAX_K + j], qfun(i, v)));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a = ff_add(a, ff_shfl_xor(a, o));
+    if (lane == 0) alphaS[i] = ff_f(a);
+  }
+  __syncthreads();
+  if (tid < 32) {
+    uint32_t ties = ties_draft[n];
+    float A = 0.f, alpha = 0.f, ptok = 0.f, qtok = 1.f, u2 = 0.f;
+    bool acc_ok = false;
+    uint32_t ftb = 0u;
+    for (int r = lane; r < Bt; r += 32) ftb |= ftie[n * (B + 1) + r];
+    if (__any_sync(FULLMASK, ftb != 0u)) ties |= TIE_TOPP;
+    if (lane < B) {
+      const int m = n * B + lane;
+      const int rl = n * (B + 1) + lane;
+      const int x = tok[m];
+      // p'(x_i): binary search among the kept tokens (sorted by index)
+      int lo = 0, hi = fcnt[rl];
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (ftok[(size_t)rl * FILTER_MAX_K + mid] < x) lo = mid + 1;
+        else hi = mid;
+      }
+      ptok = (lo < fcnt[rl] && ftok[(size_t)rl * FILTER_MAX_K + lo] == x)
+                 ? fp[(size_t)rl * FILTER_MAX_K + lo] : 0.f;
+      qtok = qtok_ws[m];
+      const float ratio = ptok / qtok;
+      A = fminf(1.f, ratio);
+      alpha = alphaS[lane];
+      u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
+      acc_ok = u2 < ratio;
+      if (out.p_tok) out.p_tok[m] = ptok;
+      if (out.accept_prob) out.accept_prob[m] = A;
+      if (out.alpha) out.alpha[m] = alpha;
+    }
+    const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
+    const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
+    const int L = rej ? (__ffs(rej) - 1) : B;
+    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    float cC = 1.f;
+    if (lane < B) {
+      cC = coll[(size_t)n * (B + 1) + lane];
+      if (out.collision) out.collision[n * B + lane] = cC;
+    }
+    float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float ta = __shfl_up_sync(FULLMASK, cA, o);
+      const float tl = __shfl_up_sync(FULLMASK, cAl, o);
+      const float tc = __shfl_up_sync(FULLMASK, cC, o);
+      if (lane >= o) {
+        cA *= ta;
+        cAl *= tl;
+        cC *= tc;
+      }
+    }
+    FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f}, ed{lane < B ? cC : 0.f, 0.f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      el = ff_add(el, ff_shfl_xor(el, o));
+      ea = ff_add(ea, ff_shfl_xor(ea, o));
+      ed = ff_add(ed, ff_shfl_xor(ed, o));
+    }
+    // the residual or bonus token, by this warp
+    int extra = -1;
+    if (L < B || Bt > B) {
+      const int irow = L < B ? L : B;
+      const int rl = n * (B + 1) + irow;
+      const int cnt = fcnt[rl];
+      const int32_t* tk = ftok + (size_t)rl * FILTER_MAX_K;
+      const float* pk = fp + (size_t)rl * FILTER_MAX_K;
+      const float u3 = decision_uniform(seed, 3u, rd, (uint32_t)n, (uint32_t)(p0 + irow));
+      float margin = 0.f, total = 0.f;
+      int j = -1;
+      bool from_p = L >= B;
+      if (L < B) {
+        j = warp_inverse_cdf(cnt, [&](int jj) { return fmaxf(pk[jj] - qfun(L, tk[jj]), 0.f); },
+                             u3, &margin, &total);
+        if (total < TIE_TOL) ties |= TIE_RMASS;
+        if (j < 0) {
+          from_p = true;
+          ties |= TIE_RMASS;
+        }
+      }
+      if (from_p) j = warp_inverse_cdf(cnt, [&](int jj) { return pk[jj]; }, u3, &margin, &total);
+      if (margin < TIE_TOL) ties |= TIE_RESID;
+      extra = j >= 0 ? tk[j] : (cnt > 0 ? tk[0] : 0);
+    }
+    if (lane == 0) {
+      if (out.exp_len) out.exp_len[n] = ff_f(el);
+      if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
+      if (out.determinism) out.determinism[n] = ff_f(ed) / (float)B;
+      sL = L;
+      sx = extra;
+      sties = ties;
+    }
+  }
+  __syncthreads();
+  const int L = sL, extra = sx;
+  if (tid == 0) {
+    const int ne = L + (extra >= 0 ? 1 : 0);
+    if (out.accepted) out.accepted[n] = L;
+    if (out.n_emitted) out.n_emitted[n] = ne;
+    if (out.tie_flags) out.tie_flags[n] = sties;
+    pos[n] = p0 + ne;
+    rnd[n] = rd + 1u;
+  }
+  if (out.emitted) {
+    for (int j = tid; j < B + 1; j += VF_NT) {
+      int val = -1;
+      if (j < L) val = tok[n * B + j];
+      else if (j == L && extra >= 0) val = extra;
+      out.emitted[(size_t)n * (B + 1) + j] = val;
+    }
+  }
+}
+
+template <typename Tin>
+static cudaError_t filter_typed(const StepCtx& c, const dblast_verify_out* o) {
+  const WsLayout& w = c.wl;
+  const int rows = w.N * c.Bt;
+  k_target_filter<Tin><<<rows, TF_NT, 0, c.stream>>>(
+      static_cast<const Tin*>(o->target), wsp<float2>(c, w.off_partt), w.V, w.nt, w.B, c.Bt, w.Rt,
+      o->top_k > 0 ? o->top_k : w.V, o->top_p, c.k2, wsp<int32_t>(c, w.off_ftok),
+      wsp<float>(c, w.off_fp), wsp<int32_t>(c, w.off_fcnt), wsp<float>(c, w.off_coll),
+      wsp<uint32_t>(c, w.off_ftie));
+  debug_kernel("k_target_filter", c.stream);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_target_filter(const StepCtx& c, const dblast_verify_out* o) {
+  return c.head->dtype == DBLAST_F32 ? filter_typed<float>(c, o) : filter_typed<__nv_bfloat16>(c, o);
+}
+
+cudaError_t launch_filtered_verify(const StepCtx& c, const dblast_verify_out* o) {
+  const WsLayout& w = c.wl;
+  auto k = c.greedy ? k_filtered_verify<true> : k_filtered_verify<false>;
+  cudaError_t le = launch_dep(k, dim3(w.N), dim3(VF_NT), 0, c.stream,
+      wsp<int32_t>(c, w.off_ftok), wsp<float>(c, w.off_fp), wsp<int32_t>(c, w.off_fcnt),
+      wsp<uint32_t>(c, w.off_ftie), wsp<float>(c, w.off_coll), wsp<float>(c, w.off_stash),
+      prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2),
+      wsp<float2>(c, w.off_w2), wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask),
+      wsp<float>(c, w.off_log2pi), wsp<float>(c, w.off_qtok), wsp<int32_t>(c, w.off_tok),
+      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, c.Bt, c.k2, c.args->seed,
+      c.args->pos, c.args->round, *o);
+  debug_kernel("k_filtered_verify", c.stream);
+  count_launches(1);
+  return le != cudaSuccess ? le : cudaGetLastError();
+}
+
 }  // namespace dblast

@@ -16,24 +16,27 @@ RTOL = 1e-4
 ATOL_PROB = 1e-7
 
 
-def run_gpu(head_t, blk, T, Z_T, seed, pos, rnd, impl="auto", head=None, ws=None, mode="soft"):
+def run_gpu(head_t, blk, T, Z_T, seed, pos, rnd, impl="auto", head=None, ws=None, mode="soft",
+            top_k=0, top_p=0.0):
     from paper_2608_05448_gb300 import Head, Workspace, dblast_draft_and_verify
     head = head or Head.from_dict(head_t)
     N, B, _ = blk["hidden"].shape
     ws = ws or Workspace(head, N, B, blk["has_bonus"])
     dout, vout = dblast_draft_and_verify(head, ws, blk["hidden"], pos, rnd, T, Z_T, seed,
                                          blk["target"], blk["has_bonus"],
-                                         anchor=blk.get("anchor"), impl=impl, mode=mode)
+                                         anchor=blk.get("anchor"), impl=impl, mode=mode,
+                                         top_k=top_k, top_p=top_p)
     torch.cuda.synchronize()
     out = {k: v.cpu() for k, v in dout.items()}
     out.update({k: v.cpu() for k, v in vout.items()})
     return out
 
 
-def run_oracle(head_t, blk, T, Z_T, seed, pos, rnd, seqs, mode="soft"):
+def run_oracle(head_t, blk, T, Z_T, seed, pos, rnd, seqs, mode="soft", top_k=0, top_p=0.0):
     return orc.draft_and_verify(head_t, blk["hidden"], blk.get("anchor"), blk["target"],
                                 blk["has_bonus"], T, Z_T, seed, pos.cpu().numpy(),
-                                rnd.cpu().numpy(), seqs=seqs, mode=mode)
+                                rnd.cpu().numpy(), seqs=seqs, mode=mode, top_k=top_k,
+                                top_p=top_p)
 
 
 def _close(name, got, want, rtol=RTOL, atol=ATOL_PROB):

@@ -117,3 +117,26 @@ def test_determinism_bad_arguments_are_rejected_before_launch(kw, status):
                                         a["ws_bytes"], None)
     assert got == status
     assert lib.dblast_determinism_workspace_bytes(2, 17, 15, 151936, 20) > 2 * 17 * 1187 * 8
+
+
+@pytest.mark.parametrize("top_k,top_p,status", [
+    (-1, 0.0, 1), (0, float("nan"), 1), (0, -0.5, 1),
+    (300, 0.0, 2),        # more than 256 kept tokens
+    (0, 0.9, 2),          # top-p over the whole 1000-token vocabulary
+    (20, 0.9, 0), (2000, 0.0, 0), (0, 1.0, 0),
+])
+def test_filter_arguments_are_checked_before_launch(top_k, top_p, status):
+    lib = bd.lib()
+    h = fake_head(V=1000, H=64, K=4, r=8)
+    h.prep_bytes = lib.dblast_prep_bytes(ctypes.byref(h))
+    a = _args()
+    p = ctypes.c_void_p(1 << 20)
+    v = bd.CVerifyOut()
+    v.target = p
+    v.top_k = top_k
+    v.top_p = top_p
+    need = lib.dblast_workspace_bytes(ctypes.byref(h), 2, 3, 1)
+    # an accepted filter gets as far as the workspace check (3), with a buffer one byte short
+    got = lib.dblast_verify_block(ctypes.byref(h), ctypes.byref(a), ctypes.byref(v), p,
+                                  need - 1, None)
+    assert got == (3 if status == 0 else status)
