@@ -32,6 +32,10 @@ Definitions followed (section / equation of the paper):
   (Algorithm 1; Appendix A, "Distributional correctness").
 * Expected accepted length of the drafted block, sum_i prod_{j<=i} A_j
   (Eq. 3), and the overlap alpha_i = sum_v min(p_i(v), q(v|x_<i)).
+* Training-side objectives, forward only (Sec. 3.2): block NLL (Eqs.
+  independent-nll, dependent-nll) and the acceptance-oriented surrogate J_AL
+  with r_l, S_l, l_tau (Eqs. acceptance-length-objective, subblock-objective)
+  on given target blocks.
 * Target sampling transform: temperature, top-k, top-p (Sec. 3.2, Sec. 4),
   applied to every target row before verification (filter_target).
 * Target-block early determinism D_b and its M-sample estimator (App. B),
@@ -325,6 +329,80 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 lse_target=lse_t, ties=ties, first_tie=first_tie,
                 collision=collision_probability(p[:B]),
                 determinism=early_determinism_exact(p[:B]))
+
+
+# ---------------------------------------------- training-side objectives (forward)
+def block_nll(log_pi, logq_at_x):
+    """Block negative log-likelihood of a target block under the proposal.
+
+    Eq. dependent-nll: -log sum_z q(z|y) prod_i q_i(x*_i|y,z); with K = 1 it
+    is Eq. independent-nll, -sum_i log q_i(x*_i|y).  log_pi: [K];
+    logq_at_x: [b, K] with logq_at_x[i, z] = log q_i(x*_i|y,z).
+    """
+    with np.errstate(invalid="ignore"):
+        return float(-logsumexp(log_pi + np.sum(logq_at_x, axis=0)))
+
+
+def al_surrogate(q_cond, p_tok, tau):
+    """The acceptance-oriented surrogate of one target block (Sec. 3.2).
+
+    q_cond[i] = q(x*_i|y,x*_<i) (the proposal conditional, Eq.
+    dep-next-token), p_tok[i] = p(x*_i|y,x*_<i).  A_j = min(1, p/q) (Eq. 2),
+    r_l = q(x*_{1:l}|y) / p(x*_{1:l}|y) = prod_{j<=l} q_j / p_j (the prefix
+    importance ratio), S_l = sum_{i<=l} prod_{j<=i} A_j, l_tau = the first l
+    with r_l < tau (b if none), and J = sum_{l <= l_tau} (log r_l + log S_l)
+    (Eq. subblock-objective for one sampled block; the loss is -J, Eq.
+    training-loss).  Returns dict(A, r, S, l_tau (1-based), J, margin: the
+    relative distance of the decisive r_l to tau).
+    """
+    q = np.asarray(q_cond, dtype=np.float64)
+    p = np.asarray(p_tok, dtype=np.float64)
+    b = q.shape[0]
+    with np.errstate(divide="ignore"):
+        A = np.minimum(1.0, p / q)
+        r = np.cumprod(q / p)
+    S = np.cumsum(np.cumprod(A))
+    below = np.nonzero(r < tau)[0]
+    l_tau = int(below[0]) + 1 if below.size else b
+    with np.errstate(divide="ignore"):
+        J = float(np.sum(np.log(r[:l_tau]) + np.log(S[:l_tau])))
+    margin = float(np.min(np.abs(r[:l_tau] - tau)) / tau) if tau > 0 else np.inf
+    return dict(A=A, r=r, S=S, l_tau=l_tau, J=J, margin=margin)
+
+
+def al_objective_sequence(head, h, anchor, target, tokens, T, Z_T, tau,
+                          top_k=0, top_p=0.0):
+    """Forward pass of the training objectives on one given target block.
+
+    tokens: the target block x*_{1:b} (sampled from the target); target:
+    [b (+1), V] target logits whose first b rows give p_i.  The proposal is
+    the soft latent mixture (Eq. 5) with the category prior at Z_T; its
+    conditionals along x* are Eqs. category-posterior and dep-next-token.
+    p is the target after the same filter as verification
+    (target_distributions).  Returns block NLL (Eq. dependent-nll), the AL
+    surrogate terms (al_surrogate), q_cond, p_tok and the ties of the
+    top-p cuts and of the l_tau decision (kind "tau", within TIE_TOL).
+    """
+    b = len(tokens)
+    a = h[0] if anchor is None else anchor
+    ties = []
+    _, pi = category_prior(head["Wp"], head["bp"], a, Z_T)
+    with np.errstate(divide="ignore"):
+        log_pi = np.log(pi)
+    hz = branch_hidden(h, head["U"], head["Vf"], head["e"])
+    s = component_logits(head["W"], hz, head["vbias"]) / T
+    logq = s - logsumexp(s, axis=-1)[:, :, None]
+    x = np.asarray(tokens, dtype=np.int64)
+    logq_at_x = logq[np.arange(b), :, x]                        # [b, K]
+    logw = posterior(log_pi, logq_at_x)
+    q_cond = np.sum(np.exp(logw + logq_at_x), axis=-1)
+    p, _ = target_distributions(target[:b], T, top_k, top_p, ties)
+    p_tok = p[np.arange(b), x]
+    al = al_surrogate(q_cond, p_tok, tau)
+    if al["margin"] < TIE_TOL:
+        ties.append(("tau", al["l_tau"] - 1, al["margin"]))
+    return dict(nll=block_nll(log_pi, logq_at_x), q_cond=q_cond, p_tok=p_tok,
+                ties=ties, **al)
 
 
 # --------------------------------------------------------- greedy-branch mode
