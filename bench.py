@@ -272,6 +272,44 @@ def run_determinism(args, cfg):
         "data": "synthetic"}}), flush=True)
 
 
+def run_al(args, cfg):
+    """Training-side objectives, forward only (block NLL and J_AL at tau = 0.1)
+    on target blocks of the workload: one JSON line with ms per call and
+    blocks/s, with and without the paper's target filter."""
+    import numpy as np
+    import torch
+    import synth
+    from paper_2608_05448_gb300 import Head, Workspace, dblast_al_objective
+    dev = torch.device("cuda", 0)
+    head_t = synth.make_head(cfg, dev)
+    blk = synth.make_block(cfg, head_t, 0, dev)
+    head = Head.from_dict(head_t)
+    N, B = cfg["N"], cfg["B"]
+    ws = Workspace(head, N, B, blk["has_bonus"])
+    pos, rnd = synth.initial_state(cfg, dev)
+    # target blocks: the target's own top tokens, a fixed input of the timed calls
+    g = torch.Generator(device=dev).manual_seed(7)
+    probs = torch.softmax(blk["target"][:, :B].float() / args.T, dim=-1)
+    tokens = torch.multinomial(probs.reshape(-1, probs.shape[-1]), 1, generator=g)
+    tokens = tokens.reshape(N, B).int().contiguous()
+    del probs
+    for top_k, top_p in ((0, 0.0), (20, 0.95)):
+        res = {}
+
+        def step(k):
+            res["o"] = dblast_al_objective(head, ws, blk["hidden"], pos, rnd, args.T, 1.0, 3,
+                                           tokens, blk["target"], blk["has_bonus"], tau=0.1,
+                                           top_k=top_k, top_p=top_p)
+        ms = _timed_steps(step, args.steps, args.warmup) / args.steps
+        o = {k: v.float().cpu() for k, v in res["o"].items()}
+        print(json.dumps({"al_objective": {
+            "workload": cfg["name"], "N": N, "B": B, "T": args.T, "top_k": top_k,
+            "top_p": top_p, "tau": 0.1, "ms_per_call": ms, "blocks_per_s": N / (ms * 1e-3),
+            "nll_mean": float(o["nll"].mean()),
+            "j_al_mean": float(o["j_al"][torch.isfinite(o["j_al"])].mean()),
+            "l_tau_mean": float(o["l_tau"].mean()), "data": "synthetic"}}), flush=True)
+
+
 def run_serve(args):
     """Serving steps (N=256, B=8 and 32): four rounds with fresh hidden states
     and targets per round and per-sequence state (positions, round counters,
@@ -339,6 +377,9 @@ def main():
                     help="entropy-sweep report (K=16 vs K=1 cells), one JSON line per cell")
     ap.add_argument("--determinism", action="store_true",
                     help="target-block early determinism report (b = 15, M = 20), one JSON line")
+    ap.add_argument("--al", action="store_true",
+                    help="training-side objectives (block NLL, J_AL), forward only, one JSON line "
+                         "per filter setting")
     ap.add_argument("--serve", action="store_true",
                     help="serving report (N=256, B=8/32, four rounds), one JSON line per round")
     ap.add_argument("--n-seqs", type=int, default=None,
@@ -355,11 +396,13 @@ def main():
     if args.impl == "reference":
         run_reference(args, cfg, rank)
         return
-    if args.sweep or args.serve or args.determinism:
+    if args.sweep or args.serve or args.determinism or args.al:
         import torch
         torch.cuda.set_device(0)
         if args.determinism:
             run_determinism(args, cfg)
+        if args.al:
+            run_al(args, cfg)
         if args.sweep:
             run_sweep(args)
         if args.serve:

@@ -245,6 +245,48 @@ dblast_status dblast_target_lse_noalloc(const void* target, int rows, int V, dbl
                                         float temperature, float* lse_out,
                                         dblast_stream_t stream);
 
+/* Training-side objectives, forward only, on given target blocks (Sec. 3.2).
+ * For each sequence n the target block x*_{1:B} = tokens[n] (sampled from the
+ * target) is scored under the soft latent-mixture proposal (Eq. 5; the
+ * prior at args->z_temperature, branch distributions at args->temperature):
+ *   q_cond[n, i] = q(x*_i|y, x*_<i) (Eqs. category-posterior, dep-next-token)
+ *   p_tok[n, i]  = p(x*_i), the target after the filter top_k / top_p (as in
+ *                  dblast_verify_out)
+ *   accept_prob  = A_i = min(1, p/q) (Eq. 2)
+ *   r[n, l]      = prod_{j<=l} q_cond_j / p_tok_j, the prefix importance ratio
+ *   S[n, l]      = sum_{i<=l} prod_{j<=i} A_j
+ *   l_tau[n]     = the first l (1-based) with r_l < tau, else B
+ *   j_al[n]      = sum_{l<=l_tau} (log r_l + log S_l) (Eq. subblock-objective;
+ *                  the training loss is -j_al, Eq. training-loss)
+ *   nll[n]       = -log sum_z q(z|y) prod_i q_i(x*_i|y,z) (Eq. dependent-nll;
+ *                  K = 1: Eq. independent-nll)
+ *   tie_flags[n] bit5: a top-p cut within 1e-6; bit6: an r_l within 1e-6
+ *                (relative) of tau among l <= l_tau.
+ * Natural logarithms.  args->mode must be DBLAST_MODE_SOFT; args->seed, pos
+ * and round are read (the latent draw of the shared draft kernels) but not
+ * advanced.  Uses the step workspace (dblast_workspace_bytes with the same
+ * N, B, has_bonus).  Every output may be NULL. */
+typedef struct {
+  const int32_t* tokens; /* [N, B] target block x*_{1:B} */
+  const void* target;    /* [N, B + has_bonus, V] target logits (head dtype) */
+  int has_bonus;
+  int top_k;
+  float top_p;
+  float tau;             /* truncation threshold, >= 0 (the paper: 0.1) */
+  float* nll;            /* [N] */
+  float* j_al;           /* [N] */
+  int32_t* l_tau;        /* [N] */
+  float* r;              /* [N, B] */
+  float* S;              /* [N, B] */
+  float* accept_prob;    /* [N, B] */
+  float* q_cond;         /* [N, B] */
+  float* p_tok;          /* [N, B] */
+  uint32_t* tie_flags;   /* [N] */
+} dblast_al_args;
+dblast_status dblast_al_objective(const dblast_head* head, const dblast_block_args* args,
+                                  const dblast_al_args* al, void* workspace,
+                                  size_t workspace_bytes, dblast_stream_t stream);
+
 /* Target-block early determinism of given target rows (App. B).
  *   collision[n, i] = sum_v p_{n,i}(v)^2 for the first b rows of sequence n,
  *   d_exact[n]      = (1/b) sum_j prod_{i<=j} collision[n, i]

@@ -53,6 +53,14 @@ class CDraftOut(ctypes.Structure):
                 ("z_hat", "pi", "tokens", "lse", "logw", "q_tok", "branch_tokens")]
 
 
+class CAlArgs(ctypes.Structure):
+    _fields_ = [("tokens", ctypes.c_void_p), ("target", ctypes.c_void_p),
+                ("has_bonus", ctypes.c_int), ("top_k", ctypes.c_int), ("top_p", ctypes.c_float),
+                ("tau", ctypes.c_float)] + [
+        (n, ctypes.c_void_p) for n in ("nll", "j_al", "l_tau", "r", "S", "accept_prob",
+                                       "q_cond", "p_tok", "tie_flags")]
+
+
 class CStats(ctypes.Structure):
     _fields_ = [("calls", ctypes.c_uint64), ("kernel_launches", ctypes.c_uint64),
                 ("tc_launches", ctypes.c_uint64),
@@ -73,7 +81,8 @@ EXPORTS = ["dblast_prep_bytes", "dblast_workspace_bytes", "dblast_head_prepare",
            "dblast_draft_block", "dblast_verify_block", "dblast_draft_and_verify",
            "dblast_device_status", "dblast_set_wait_limit", "dblast_stats_reset",
            "dblast_stats_get", "dblast_target_lse_noalloc", "dblast_status_string",
-           "dblast_version", "dblast_determinism_workspace_bytes", "dblast_target_determinism"]
+           "dblast_version", "dblast_determinism_workspace_bytes", "dblast_target_determinism",
+           "dblast_al_objective"]
 
 
 def load_library(path=None, build_if_missing=True):
@@ -114,6 +123,9 @@ def load_library(path=None, build_if_missing=True):
                                               ctypes.c_int, ctypes.c_float, ctypes.c_void_p,
                                               ctypes.c_void_p]
     lib.dblast_target_lse_noalloc.restype = ctypes.c_int
+    lib.dblast_al_objective.argtypes = [P(CHead), P(CBlockArgs), P(CAlArgs), ctypes.c_void_p, S,
+                                        ctypes.c_void_p]
+    lib.dblast_al_objective.restype = ctypes.c_int
     lib.dblast_determinism_workspace_bytes.argtypes = [ctypes.c_int] * 5
     lib.dblast_determinism_workspace_bytes.restype = S
     lib.dblast_target_determinism.argtypes = [
@@ -383,4 +395,31 @@ def dblast_target_determinism(target, b, temperature, M=0, seed=0, samples=False
         int(seed) & ((1 << 64) - 1), _ptr(out["collision"]), _ptr(out["d_exact"]),
         _ptr(out.get("d_hat")), _ptr(out.get("samples")), _ptr(ws), nbytes, _stream()),
         "dblast_target_determinism")
+    return out
+
+
+def dblast_al_objective(head, ws, hidden, pos, round_, T, Z_T, seed, tokens, target, has_bonus,
+                        tau=0.1, top_k=0, top_p=0.0, anchor=None, impl="auto"):
+    """Forward pass of the training-side objectives on given target blocks
+    tokens [N, B] (int32): block NLL, J_AL and its terms (r, S, l_tau, A,
+    q_cond, p_tok).  Returns a dict of CUDA tensors."""
+    args = _block_args(head, hidden, pos, round_, T, Z_T, seed, anchor, impl, "soft")
+    N, B, _ = hidden.shape
+    _cuda_contig(tokens, "tokens", torch.int32)
+    _cuda_contig(target, "target", head.dtype)
+    if tuple(tokens.shape) != (N, B) or tuple(target.shape) != (N, B + int(has_bonus), head.V):
+        raise ValueError("tokens must be [N, B] and target [N, B + has_bonus, V]")
+    dev = hidden.device
+    f = torch.float32
+    out = dict(nll=torch.empty(N, dtype=f, device=dev), j_al=torch.empty(N, dtype=f, device=dev),
+               l_tau=torch.empty(N, dtype=torch.int32, device=dev),
+               r=torch.empty(N, B, dtype=f, device=dev), S=torch.empty(N, B, dtype=f, device=dev),
+               accept_prob=torch.empty(N, B, dtype=f, device=dev),
+               q_cond=torch.empty(N, B, dtype=f, device=dev),
+               p_tok=torch.empty(N, B, dtype=f, device=dev),
+               tie_flags=torch.empty(N, dtype=torch.int32, device=dev))
+    al = CAlArgs(_ptr(tokens), _ptr(target), int(has_bonus), int(top_k), float(top_p), float(tau),
+                 *[_ptr(out[k]) for k, _ in CAlArgs._fields_[6:]])
+    _check(lib().dblast_al_objective(ctypes.byref(head.c), ctypes.byref(args), ctypes.byref(al),
+                                     ws.ptr, ws.nbytes, _stream()), "dblast_al_objective")
     return out

@@ -483,6 +483,45 @@ dblast_status dblast_stats_get(dblast_stats* out) {
   return DBLAST_OK;
 }
 
+dblast_status dblast_al_objective(const dblast_head* h, const dblast_block_args* a,
+                                  const dblast_al_args* al, void* ws, size_t ws_bytes,
+                                  dblast_stream_t stream) {
+  dblast_status st = check_head(h, true);
+  if (st == DBLAST_OK) st = check_args(h, a);
+  if (st != DBLAST_OK) return st;
+  if (!al || !al->tokens || !al->target || !aligned16(al->target)) return DBLAST_ERR_INVALID_ARG;
+  if (a->mode != DBLAST_MODE_SOFT || !(al->tau >= 0.f) || al->tau == INFINITY)
+    return DBLAST_ERR_INVALID_ARG;
+  dblast_verify_out vo{};
+  vo.target = al->target;
+  vo.has_bonus = al->has_bonus ? 1 : 0;
+  vo.top_k = al->top_k;
+  vo.top_p = al->top_p;
+  st = check_filter(h, &vo);
+  if (st != DBLAST_OK) return st;
+  StepCtx c;
+  st = make_ctx(h, a, ws, ws_bytes, vo.has_bonus, stream, &c);
+  if (st != DBLAST_OK) return st;
+  c.target = al->target;
+  c.Bt = a->B + vo.has_bonus;
+  g_calls.fetch_add(1, std::memory_order_relaxed);
+  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t),
+                                  c.stream);
+  if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
+  if (e == cudaSuccess)
+    e = dbg(c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c), "draft_pass", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_draft_finalize(c, nullptr, al->tokens), "draft_finalize", c.stream);
+  if (e == cudaSuccess) e = dbg(launch_target_stats(c, &vo), "target_stats", c.stream);
+  const bool filtered = filter_on(h, &vo);
+  if (e == cudaSuccess && filtered) {
+    const dblast_verify_out f = filter_args(h, &vo);
+    e = dbg(launch_target_filter(c, &f), "target_filter", c.stream);
+  }
+  if (e == cudaSuccess) e = dbg(launch_al_objective(c, al, filtered), "al_objective", c.stream);
+  return cuda_status(e);
+}
+
 // Workspace of dblast_target_determinism: the target statistics of the
 // N x rows target rows (tile records, log-sum-exp, collision probability) and
 // p_i(x_i^(m)) of every sample.

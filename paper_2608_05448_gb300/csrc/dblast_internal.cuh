@@ -21,7 +21,8 @@ constexpr float LN2 = 0.6931471805599453f;
 constexpr float TIE_TOL = 1e-6f;
 
 enum TieBits : uint32_t {
-  TIE_ZHAT = 1u, TIE_DRAFT = 2u, TIE_ACCEPT = 4u, TIE_RESID = 8u, TIE_RMASS = 16u, TIE_TOPP = 32u
+  TIE_ZHAT = 1u, TIE_DRAFT = 2u, TIE_ACCEPT = 4u, TIE_RESID = 8u, TIE_RMASS = 16u, TIE_TOPP = 32u,
+  TIE_TAU = 64u
 };
 
 // target filter (top-k / top-p): at most FILTER_MAX_K kept tokens per row,
@@ -290,7 +291,9 @@ bool tc_supported(const dblast_head* h);
 cudaError_t launch_prior(const StepCtx& c);
 cudaError_t launch_codes(const StepCtx& c);
 cudaError_t launch_draft_pass_simt(const StepCtx& c);
-cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* out);
+cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* out,
+                                  const int32_t* given = nullptr);
+cudaError_t launch_al_objective(const StepCtx& c, const dblast_al_args* al, bool filtered);
 cudaError_t launch_target_stats(const StepCtx& c, const dblast_verify_out* out);
 cudaError_t launch_verify_pass_simt(const StepCtx& c);
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* out);

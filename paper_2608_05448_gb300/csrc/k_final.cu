@@ -342,7 +342,8 @@ __global__ void __launch_bounds__(DT_NT)
                   const float* __restrict__ codes, const int32_t* __restrict__ zhat, int nt, int V,
                   int K, int rr, int B, int M, int Mpad, float k2, uint64_t seed,
                   const int64_t* __restrict__ pos, const uint32_t* __restrict__ rnd,
-                  float2* __restrict__ lse2, int32_t* __restrict__ tok, float2* __restrict__ lq2,
+                  const int32_t* __restrict__ given, float2* __restrict__ lse2,
+                  int32_t* __restrict__ tok, float2* __restrict__ lq2,
                   uint32_t* __restrict__ ties) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<DT_NT> fs;
@@ -375,11 +376,17 @@ __global__ void __launch_bounds__(DT_NT)
   const float* srow = stash + (size_t)m * V;
   const DraftTileMass tm{partd + (size_t)z * Mpad + m, (size_t)K * Mpad, L};
   const BranchTokenProb em{srow, wu, cm + z * rr, z, K, rr, k2, L};
-  const FindOut f = block_find<DT_NT>(nt, V, tm, em, FF{u, 0.f}, 1.f, fs);
-  const int x = f.x >= 0 ? f.x : 0;
-  if (tid == 0) {
-    tok[m] = x;
-    if (f.tie || f.x < 0) atomicOr(&ties[n], (uint32_t)TIE_DRAFT);
+  int x;
+  if (given) {  // a given block (training-side objectives): no draw
+    x = min(max(given[m], 0), V - 1);
+    if (tid == 0) tok[m] = x;
+  } else {
+    const FindOut f = block_find<DT_NT>(nt, V, tm, em, FF{u, 0.f}, 1.f, fs);
+    x = f.x >= 0 ? f.x : 0;
+    if (tid == 0) {
+      tok[m] = x;
+      if (f.tie || f.x < 0) atomicOr(&ties[n], (uint32_t)TIE_DRAFT);
+    }
   }
   if (tid < K) {  // log2 q_z(x) = (base_x + corr_z(x)) k2 - L_z, products exact
     const FF s = ff_add(ff_prod(srow[x], k2), ff_prod(corr_at(wu, cm + tid * rr, x, tid, K, rr), k2));
@@ -465,7 +472,8 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp) {
+cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp,
+                                  const int32_t* given) {
   const WsLayout& w = c.wl;
   const dblast_block_args* a = c.args;
   const int K = c.head->K;
@@ -476,7 +484,8 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
   if (le == cudaSuccess) le = launch_dep(k_draft_token, dim3(w.M), dim3(DT_NT), 0, c.stream,
       wsp<float2>(c, w.off_partd), wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_stash),
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<int32_t>(c, w.off_zhat), w.nt,
-      w.V, K, w.rr, w.B, w.M, w.Mpad, c.k2, a->seed, a->pos, a->round, wsp<float2>(c, w.off_lse2),
+      w.V, K, w.rr, w.B, w.M, w.Mpad, c.k2, a->seed, a->pos, a->round, given,
+      wsp<float2>(c, w.off_lse2),
       wsp<int32_t>(c, w.off_tok), wsp<float2>(c, w.off_lq2), wsp<uint32_t>(c, w.off_ties));
   debug_kernel("k_draft_token", c.stream);
   dblast_draft_out out{};
@@ -1629,6 +1638,7 @@ __global__ void __launch_bounds__(TF_NT)
                     int32_t* __restrict__ ftok, float* __restrict__ fp, int32_t* __restrict__ fcnt,
                     float* __restrict__ coll, uint32_t* __restrict__ ftie) {
   __shared__ FilterShared sh;
+  __shared__ uint32_t tkey[FILTER_MAX_TILES];  // keys of the row's tile maxima
   __shared__ int clist[FILTER_MAX_TILES];
   __shared__ int stok[FILTER_MAX_K];
   __shared__ float sval[FILTER_MAX_K];
@@ -1640,15 +1650,16 @@ __global__ void __launch_bounds__(TF_NT)
   const int rl = n * (B + 1) + i;
   const Tin* tr = target + (size_t)row * V;
   const int k = min(kf, V);
+  for (int t = tid; t < nt; t += TF_NT) tkey[t] = fkey(partt[(size_t)t * Rt + rl].x);
+  __syncthreads();
   // candidate tiles: maximum >= the k-th largest tile maximum
   uint32_t theta = 0u;
   if (k < nt) {
     int rem;
-    theta = radix_kth_largest(nt, k, [&](int t) { return fkey(partt[(size_t)t * Rt + rl].x); },
-                              sh, &rem);
+    theta = radix_kth_largest(nt, k, [&](int t) { return tkey[t]; }, sh, &rem);
   }
   const int C = ordered_compact(
-      nt, 0, [&](int t) { return fkey(partt[(size_t)t * Rt + rl].x) >= theta ? 1 : 0; },
+      nt, 0, [&](int t) { return tkey[t] >= theta ? 1 : 0; },
       [&](int t, int pos) { clist[pos] = t; }, sh);
   // the k-th largest logit of the candidate tiles, and its equal values needed
   auto cand = [&](int j) {
@@ -1674,10 +1685,11 @@ __global__ void __launch_bounds__(TF_NT)
       sh);
   __syncthreads();
   // weights relative to the largest kept logit
-  if (tid == 0) {
+  if (tid < 32) {
     float m = -INFINITY;
-    for (int j = 0; j < cnt; ++j) m = fmaxf(m, sval[j]);
-    sh.smax = m;
+    for (int j = tid; j < cnt; j += 32) m = fmaxf(m, sval[j]);
+    m = warp_max(m);
+    if (tid == 0) sh.smax = m;
   }
   __syncthreads();
   const FF cmax = ff_prod(sh.smax, k2);
@@ -1697,17 +1709,12 @@ __global__ void __launch_bounds__(TF_NT)
     __syncthreads();
     for (int j = tid; j < cnt; j += TF_NT) scum[skeep[j]] = FF{sw[j], 0.f};
     __syncthreads();
-    if (tid == 0) {  // exclusive prefix sums in rank order (k <= FILTER_MAX_K)
-      FF acc{0.f, 0.f};
-      for (int r = 0; r < cnt; ++r) {
-        const FF w = scum[r];
-        scum[r] = acc;
-        acc = ff_add(acc, w);
-      }
-      sh.red[0] = acc;
-    }
+    // exclusive prefix sums in rank order (cnt <= FILTER_MAX_K == TF_NT)
+    static_assert(FILTER_MAX_K <= TF_NT, "one thread per rank");
+    const BlockScan bs = block_scan_ff<TF_NT>(tid < cnt ? scum[tid] : FF{0.f, 0.f}, sh.red);
+    if (tid < cnt) scum[tid] = bs.excl;
     __syncthreads();
-    const FF W = sh.red[0];
+    const FF W = bs.total;
     const FF thr = ff_mulf(W, top_p);
     const float Wf = ff_f(W);
     for (int j = tid; j < cnt; j += TF_NT) {
@@ -2038,6 +2045,130 @@ cudaError_t launch_filtered_verify(const StepCtx& c, const dblast_verify_out* o)
       wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, c.Bt, c.k2, c.args->seed,
       c.args->pos, c.args->round, *o);
   debug_kernel("k_filtered_verify", c.stream);
+  count_launches(1);
+  return le != cudaSuccess ? le : cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- training-side objectives
+// Sec. 3.2, forward only, on a given target block x*: the draft pass and the
+// draft finalize kernels run with the given tokens in place of draws, so
+// q(x*_i|x*_<i) (Eqs. category-posterior, dep-next-token) and log2 q_z(x*_i)
+// come from the step's own kernels; one warp per sequence then forms
+// p(x*_i) (filtered like verification), A_i, r_l, S_l, l_tau, J_AL and the
+// block NLL (Eq. dependent-nll) from sum_i log2 q_z(x*_i) and the prior.
+template <typename Tin>
+__global__ void __launch_bounds__(32)
+    k_al_objective(const Tin* __restrict__ target, const int32_t* __restrict__ tok,
+                   const float* __restrict__ qtok_ws, const float2* __restrict__ lq2,
+                   const float* __restrict__ log2pi, const float2* __restrict__ lt2,
+                   const int32_t* __restrict__ ftok, const float* __restrict__ fp,
+                   const int32_t* __restrict__ fcnt, const uint32_t* __restrict__ ftie,
+                   bool filtered, int V, int K, int B, int Bt, float k2, float tau,
+                   dblast_al_args al) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  const int n = blockIdx.x, lane = threadIdx.x;
+  const size_t m0 = (size_t)n * B;
+  const bool on = lane < B;
+  uint32_t ties = 0u;
+  float p = 1.f, q = 1.f;
+  if (on) {
+    const int m = (int)m0 + lane;
+    const int rl = n * (B + 1) + lane;
+    const int x = tok[m];
+    q = qtok_ws[m];
+    if (filtered) {
+      int lo = 0, hi = fcnt[rl];
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (ftok[(size_t)rl * FILTER_MAX_K + mid] < x) lo = mid + 1;
+        else hi = mid;
+      }
+      p = (lo < fcnt[rl] && ftok[(size_t)rl * FILTER_MAX_K + lo] == x)
+              ? fp[(size_t)rl * FILTER_MAX_K + lo] : 0.f;
+      if (ftie[rl]) ties |= TIE_TOPP;
+    } else {
+      const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
+      p = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), ff_ld(lt2 + rl)));
+    }
+  }
+  const float A = on ? fminf(1.f, p / q) : 1.f;
+  // log2 r_l: prefix sums of log2 q - log2 p; S_l: prefix sums of prod A
+  FF lr{on ? log2f(q) - log2f(p) : 0.f, 0.f};
+  float cA = A;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const FF t = ff_shfl_up(lr, o);
+    const float ta = __shfl_up_sync(FULLMASK, cA, o);
+    if (lane >= o) {
+      lr = ff_add(t, lr);
+      cA *= ta;
+    }
+  }
+  FF S{on ? cA : 0.f, 0.f};
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const FF t = ff_shfl_up(S, o);
+    if (lane >= o) S = ff_add(t, S);
+  }
+  const float l2tau = tau > 0.f ? log2f(tau) : -INFINITY;
+  const float lrf = ff_f(lr);
+  const unsigned below = __ballot_sync(FULLMASK, on && lrf < l2tau);
+  const int l_tau = below ? __ffs(below) : B;
+  const bool in = lane < l_tau;
+  if (__ballot_sync(FULLMASK, in && tau > 0.f && fabsf(lrf - l2tau) * LN2 < TIE_TOL))
+    ties |= TIE_TAU;
+  FF jt{in ? lrf + ff_f(ff_log2(S)) : 0.f, 0.f};
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) jt = ff_add(jt, ff_shfl_xor(jt, o));
+  // block NLL: -log sum_z pi_z prod_i q_z(x*_i), in base 2 over the lanes z
+  FF sz{-INFINITY, 0.f};
+  if (lane < K) {
+    const float lp = log2pi[n * K + lane];
+    if (lp != -INFINITY) {
+      sz = FF{lp, 0.f};
+      for (int i = 0; i < B; ++i) sz = ff_add(sz, ff_ld(lq2 + (m0 + i) * K + lane));
+    }
+  }
+  const float mx = warp_max(sz.hi);
+  float e = (sz.hi == -INFINITY || mx == -INFINITY) ? 0.f : ff_exp2(ff_addf(sz, -mx));
+  e = warp_sum(e);
+  ties = __reduce_or_sync(FULLMASK, ties);
+  if (on) {
+    const int m = (int)m0 + lane;
+    if (al.r) al.r[m] = exp2f(lrf);
+    if (al.S) al.S[m] = ff_f(S);
+    if (al.accept_prob) al.accept_prob[m] = A;
+    if (al.q_cond) al.q_cond[m] = q;
+    if (al.p_tok) al.p_tok[m] = p;
+  }
+  if (lane == 0) {
+    if (al.j_al) al.j_al[n] = ff_f(jt) * LN2;
+    if (al.l_tau) al.l_tau[n] = l_tau;
+    if (al.nll) al.nll[n] = (mx == -INFINITY) ? INFINITY : -(mx + log2f(e)) * LN2;
+    if (al.tie_flags) al.tie_flags[n] = ties;
+  }
+}
+
+cudaError_t launch_al_objective(const StepCtx& c, const dblast_al_args* al, bool filtered) {
+  const WsLayout& w = c.wl;
+  cudaError_t le;
+  if (c.head->dtype == DBLAST_F32)
+    le = launch_dep(k_al_objective<float>, dim3(w.N), dim3(32), 0, c.stream,
+                    static_cast<const float*>(al->target), wsp<int32_t>(c, w.off_tok),
+                    wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lq2),
+                    wsp<float>(c, w.off_log2pi), wsp<float2>(c, w.off_lt2),
+                    wsp<int32_t>(c, w.off_ftok), wsp<float>(c, w.off_fp),
+                    wsp<int32_t>(c, w.off_fcnt), wsp<uint32_t>(c, w.off_ftie), filtered, w.V,
+                    c.head->K, w.B, c.Bt, c.k2, al->tau, *al);
+  else
+    le = launch_dep(k_al_objective<__nv_bfloat16>, dim3(w.N), dim3(32), 0, c.stream,
+                    static_cast<const __nv_bfloat16*>(al->target), wsp<int32_t>(c, w.off_tok),
+                    wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lq2),
+                    wsp<float>(c, w.off_log2pi), wsp<float2>(c, w.off_lt2),
+                    wsp<int32_t>(c, w.off_ftok), wsp<float>(c, w.off_fp),
+                    wsp<int32_t>(c, w.off_fcnt), wsp<uint32_t>(c, w.off_ftie), filtered, w.V,
+                    c.head->K, w.B, c.Bt, c.k2, al->tau, *al);
+  debug_kernel("k_al_objective", c.stream);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
 }
