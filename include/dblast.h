@@ -163,7 +163,7 @@ typedef struct {
    * kept set and used for p_tok, acceptance, alpha, the residual, the bonus
    * token and collision/determinism; lse_target stays the unfiltered
    * log-sum-exp.  With a filter on, at most 256 tokens may stay (top-p needs
-   * top_k in 1..256, or V <= 256) and V <= 524288; else DBLAST_ERR_UNSUPPORTED.
+   * top_k in 1..256, or V <= 256) and V <= 262144; else DBLAST_ERR_UNSUPPORTED.
    * tie_flags bit5: a top-p cut within 1e-6 of top_p on some row. */
   int top_k;
   float top_p;

@@ -28,7 +28,8 @@ enum TieBits : uint32_t {
 // target filter (top-k / top-p): at most FILTER_MAX_K kept tokens per row,
 // and vocabularies of at most FILTER_MAX_TILES tiles
 constexpr int FILTER_MAX_K = 256;
-constexpr int FILTER_MAX_TILES = 4096;
+constexpr int FILTER_MAX_TILES = 2048;
+constexpr int FILTER_STAGE = 4096;  // candidate tokens staged in shared memory (else read twice)
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }

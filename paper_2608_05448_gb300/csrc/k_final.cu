@@ -75,10 +75,24 @@ template <int NT> __device__ int block_max_i(int v, int* sh) {
   return -block_min_i<NT>(-v, sh);
 }
 
+// (W U_z)_v . c: the branch correction of token v (rr % 4 == 0: 16-byte loads,
+// the WU rows and the code rows then start on 16-byte boundaries)
 __device__ __forceinline__ float corr_at(const float* __restrict__ wu, const float* __restrict__ c,
                                          int v, int z, int K, int rr) {
   const float* wr = wu + ((size_t)v * K + z) * rr;
   float acc = 0.f;
+  if ((rr & 3) == 0) {
+    const float4* w4 = reinterpret_cast<const float4*>(wr);
+    const float4* c4 = reinterpret_cast<const float4*>(c);
+    for (int k = 0; k < (rr >> 2); ++k) {
+      const float4 a = w4[k], b = c4[k];
+      acc = fmaf(a.x, b.x, acc);
+      acc = fmaf(a.y, b.y, acc);
+      acc = fmaf(a.z, b.z, acc);
+      acc = fmaf(a.w, b.w, acc);
+    }
+    return acc;
+  }
   for (int k = 0; k < rr; ++k) acc = fmaf(wr[k], c[k], acc);
   return acc;
 }
@@ -1197,6 +1211,9 @@ __global__ void __launch_bounds__(VF_NT)
   __shared__ float piS[32];
   __shared__ int atok[32], atile[32];
   __shared__ float aq[32], amass[32];
+  __shared__ uint32_t cmS[32];
+  __shared__ float SS[32];
+  __shared__ float T[1024];  // min(p, q) of each distinct atom, at its first branch
   __shared__ int sL, sna;
   __shared__ uint32_t sties;
   __shared__ float sR;
@@ -1205,6 +1222,39 @@ __global__ void __launch_bounds__(VF_NT)
   const uint32_t rd = rnd[n];
   for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[(size_t)n * B * K + j];
   if (tid < K) piS[tid] = exp2f(log2pi[n * K + tid]);
+  if (tid < B) cmS[tid] = cmask[(size_t)n * B + tid];
+  __syncthreads();
+  if (tid < B) {
+    float S = 0.f;
+    for (int k = 0; k < K; ++k)
+      if ((cmS[tid] >> k) & 1u) S += piS[k];
+    SS[tid] = S;
+  }
+  __syncthreads();
+  // one term min(p(a), q(a)) per distinct token a of the branches in C_i, a
+  // thread per (i, z): the first branch of C_i with that token carries it
+  for (int t = tid; t < B * K; t += VF_NT) {
+    const int i = t / K, z = t - i * K;
+    const uint32_t c = cmS[i];
+    float term = 0.f;
+    if ((c >> z) & 1u) {
+      const int a = X[t];
+      bool first = true;
+      float qa = 0.f;
+      for (int k = 0; k < K; ++k) {
+        if (!((c >> k) & 1u) || X[i * K + k] != a) continue;
+        if (k < z) first = false;
+        qa += piS[k];
+      }
+      if (first) {
+        const float ta = ldf(target + ((size_t)n * Bt + i) * V + a);
+        const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + i);
+        const float pa = (ta == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(ta, k2), Lt));
+        term = fminf(pa, SS[i] > 0.f ? qa / SS[i] : 0.f);
+      }
+    }
+    T[t] = term;
+  }
   __syncthreads();
   if (tid < 32) {
     uint32_t ties = ties_draft[n];
@@ -1212,38 +1262,19 @@ __global__ void __launch_bounds__(VF_NT)
     bool acc_ok = false;
     uint32_t c = 0u;
     float S = 0.f;
-    FF Lt{0.f, 0.f};
-    const Tin* trow = target;
     if (lane < B) {
       const int m = n * B + lane;
       const int x = min(max(tok[m], 0), V - 1);
-      Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
-      trow = target + ((size_t)n * Bt + lane) * V;
-      const float tx = ldf(trow + x);
+      const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
+      const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
       ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
       qtok = qtok_ws[m];
       const float ratio = ptok / qtok;
       A = fminf(1.f, ratio);
-      // alpha_i: one term min(p(a), q(a)) per distinct token a of the branches in C_i
-      c = cmask[m];
-      for (int k = 0; k < K; ++k)
-        if ((c >> k) & 1u) S += piS[k];
+      c = cmS[lane];
+      S = SS[lane];
       FF al{0.f, 0.f};
-      for (int k = 0; k < K; ++k) {
-        if (!((c >> k) & 1u)) continue;
-        const int a = X[lane * K + k];
-        bool first = true;
-        float qa = 0.f;
-        for (int k2i = 0; k2i < K; ++k2i) {
-          if (!((c >> k2i) & 1u) || X[lane * K + k2i] != a) continue;
-          if (k2i < k) first = false;
-          qa += piS[k2i];
-        }
-        if (!first) continue;
-        const float ta = ldf(trow + a);
-        const float pa = (ta == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(ta, k2), Lt));
-        al = ff_addf(al, fminf(pa, S > 0.f ? qa / S : 0.f));
-      }
+      for (int k = 0; k < K; ++k) al = ff_addf(al, T[lane * K + k]);
       alpha = ff_f(al);
       u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
       acc_ok = u2 < ratio;
@@ -1427,6 +1458,102 @@ __global__ void __launch_bounds__(VF_NT)
   }
 }
 
+// All M draws of one target row in one block: the inclusive prefix of the
+// tile masses is scanned once into shared memory; each warp then takes a
+// draw, finds its tile by binary search and scans the tile's 128 tokens
+// (four per lane).  The decisions are those of the block-wide two-level draw
+// of k_target_sample.
+constexpr int TSR_MAX_TILES = 5120;  // prefix in shared memory (40 KB)
+template <typename Tin>
+__global__ void __launch_bounds__(VF_NT)
+    k_target_sample_row(const Tin* __restrict__ target, const float2* __restrict__ partt,
+                        const float2* __restrict__ lt2, int V, int nt, int rows, int b, int M,
+                        int Rt, float k2, uint64_t seed, float* __restrict__ pval,
+                        int32_t* __restrict__ samples) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  extern __shared__ FF pre[];  // [nt] inclusive prefix of the tile masses
+  __shared__ FF sh[VF_NT / 32];
+  const int i = blockIdx.x, n = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int rl = n * rows + i;
+  const FF Lt = ff_ld(lt2 + rl);
+  const TargetTokenProb<Tin> pv{target + (size_t)rl * V, k2, Lt};
+  const TargetTileMass tm{partt + rl, (size_t)Rt, k2, Lt};
+  const int chunk = ceil_div(nt, VF_NT);
+  const int t0 = min(nt, tid * chunk), t1 = min(nt, t0 + chunk);
+  FF loc{0.f, 0.f};
+  for (int t = t0; t < t1; ++t) {
+    const float w = tm(t);
+    loc = ff_addf(loc, w);
+    pre[t] = FF{w, 0.f};  // the mass for now, the prefix below
+  }
+  const BlockScan sc = block_scan_ff<VF_NT>(loc, sh);
+  FF run = sc.excl;
+  for (int t = t0; t < t1; ++t) {
+    run = ff_add(run, pre[t]);
+    pre[t] = run;
+  }
+  __syncthreads();
+  for (int m = warp; m < M; m += VF_NT / 32) {
+    const FF target{decision_uniform(seed, 4u, (uint32_t)m, (uint32_t)n, (uint32_t)i), 0.f};
+    int lo = 0, hi = nt;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (ff_gt(pre[mid], target)) hi = mid;
+      else lo = mid + 1;
+    }
+    int tt = lo;
+    if (tt >= nt) {  // rounding left the target at the total: the last tile with mass
+      tt = nt - 1;
+      while (tt > 0 && !(ff_gt(pre[tt], pre[tt - 1]))) --tt;
+    }
+    const FF before = tt > 0 ? pre[tt - 1] : FF{0.f, 0.f};
+    float e[4];
+    FF cum[4];
+    FF acc{0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int v = tt * TILE_V + lane * 4 + j;
+      e[j] = v < V ? pv(v) : 0.f;
+      acc = ff_addf(acc, e[j]);
+      cum[j] = acc;
+    }
+    FF incl = acc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const FF t = ff_shfl_up(incl, o);
+      if (lane >= o) incl = ff_add(t, incl);
+    }
+    FF excl = ff_shfl_up(incl, 1);
+    if (lane == 0) excl = FF{0.f, 0.f};
+    const FF base = ff_add(before, excl);
+    int jj = 4;
+#pragma unroll
+    for (int j = 3; j >= 0; --j)
+      if (ff_gt(ff_add(base, cum[j]), target)) jj = j;
+    const unsigned hit = __ballot_sync(FULLMASK, jj < 4);
+    int x;
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      x = tt * TILE_V + l * 4 + __shfl_sync(FULLMASK, jj, l);
+    } else {  // the last token with mass
+      int lj = -1;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (e[j] > 0.f) lj = j;
+      const unsigned pos = __ballot_sync(FULLMASK, lj >= 0);
+      const int l = pos ? 31 - __clz(pos) : 0;
+      x = tt * TILE_V + l * 4 + max(__shfl_sync(FULLMASK, lj, l), 0);
+    }
+    if (lane == 0) {
+      x = min(x, V - 1);
+      const size_t o = ((size_t)n * M + m) * b + i;
+      pval[o] = pv(x);
+      if (samples) samples[o] = x;
+    }
+  }
+}
+
 constexpr int DR_NT = 256;
 __global__ void __launch_bounds__(DR_NT)
     k_determinism_reduce(const float* __restrict__ coll, const float* __restrict__ pval, int rows,
@@ -1474,11 +1601,24 @@ static cudaError_t determinism_typed(const StepCtx& c, const dblast_verify_out* 
   const WsLayout& w = c.wl;
   cudaError_t e = launch_target_stats(c, o);
   if (e == cudaSuccess && (d_hat || samples)) {
-    e = launch_dep(k_target_sample<Tin>, dim3(b, M, w.N), dim3(VF_NT), 0, c.stream,
-                   static_cast<const Tin*>(o->target), wsp<float2>(c, w.off_partt),
-                   wsp<float2>(c, w.off_lt2), w.V, w.nt, rows, b, M, w.Rt, c.k2, seed,
-                   wsp<float>(c, off_pval), samples);
-    debug_kernel("k_target_sample", c.stream);
+    if (w.nt <= TSR_MAX_TILES) {
+      const size_t sm = (size_t)w.nt * sizeof(FF);
+      e = sm > 48 * 1024 ? cudaFuncSetAttribute(k_target_sample_row<Tin>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm)
+                         : cudaSuccess;
+      if (e == cudaSuccess)
+        e = launch_dep(k_target_sample_row<Tin>, dim3(b, w.N), dim3(VF_NT), sm, c.stream,
+                       static_cast<const Tin*>(o->target), wsp<float2>(c, w.off_partt),
+                       wsp<float2>(c, w.off_lt2), w.V, w.nt, rows, b, M, w.Rt, c.k2, seed,
+                       wsp<float>(c, off_pval), samples);
+      debug_kernel("k_target_sample_row", c.stream);
+    } else {
+      e = launch_dep(k_target_sample<Tin>, dim3(b, M, w.N), dim3(VF_NT), 0, c.stream,
+                     static_cast<const Tin*>(o->target), wsp<float2>(c, w.off_partt),
+                     wsp<float2>(c, w.off_lt2), w.V, w.nt, rows, b, M, w.Rt, c.k2, seed,
+                     wsp<float>(c, off_pval), samples);
+      debug_kernel("k_target_sample", c.stream);
+    }
     count_launches(1);
   }
   if (e == cudaSuccess) {
@@ -1537,12 +1677,15 @@ struct FilterShared {
 
 // The key of the k-th largest (1-based) of n keys get(i), and in *rem how many
 // elements equal to that key belong to the k largest.
+// Digits from bit 31 down to lo_shift (keys whose lower bits are all zero
+// need fewer passes: 16 for keys of bf16 values).
 template <typename GET>
-__device__ uint32_t radix_kth_largest(int n, int k, const GET& get, FilterShared& sh, int* rem) {
+__device__ uint32_t radix_kth_largest(int n, int k, const GET& get, FilterShared& sh, int* rem,
+                                      int lo_shift) {
   const int tid = threadIdx.x, lane = tid & 31;
   uint32_t prefix = 0u, mask = 0u;
   int r = k;
-  for (int shift = 24; shift >= 0; shift -= 8) {
+  for (int shift = 24; shift >= lo_shift; shift -= 8) {
     for (int b = tid; b < 256; b += TF_NT) sh.hist[b] = 0;
     __syncthreads();
     for (int i = tid; i < n; i += TF_NT) {
@@ -1640,6 +1783,7 @@ __global__ void __launch_bounds__(TF_NT)
   __shared__ FilterShared sh;
   __shared__ uint32_t tkey[FILTER_MAX_TILES];  // keys of the row's tile maxima
   __shared__ int clist[FILTER_MAX_TILES];
+  __shared__ uint32_t ckey[FILTER_STAGE];      // keys of the candidate tokens, when they fit
   __shared__ int stok[FILTER_MAX_K];
   __shared__ float sval[FILTER_MAX_K];
   __shared__ float sw[FILTER_MAX_K];
@@ -1650,31 +1794,40 @@ __global__ void __launch_bounds__(TF_NT)
   const int rl = n * (B + 1) + i;
   const Tin* tr = target + (size_t)row * V;
   const int k = min(kf, V);
-  for (int t = tid; t < nt; t += TF_NT) tkey[t] = fkey(partt[(size_t)t * Rt + rl].x);
+  // keys of bf16 values have 16 significant bits: two radix digits
+  constexpr bool BF = std::is_same<Tin, __nv_bfloat16>::value;
+  constexpr uint32_t KMASK = BF ? 0xFFFF0000u : 0xFFFFFFFFu;
+  constexpr int LO = BF ? 16 : 0;
+  for (int t = tid; t < nt; t += TF_NT) tkey[t] = fkey(partt[(size_t)t * Rt + rl].x) & KMASK;
   __syncthreads();
   // candidate tiles: maximum >= the k-th largest tile maximum
   uint32_t theta = 0u;
   if (k < nt) {
     int rem;
-    theta = radix_kth_largest(nt, k, [&](int t) { return tkey[t]; }, sh, &rem);
+    theta = radix_kth_largest(nt, k, [&](int t) { return tkey[t]; }, sh, &rem, LO);
   }
   const int C = ordered_compact(
       nt, 0, [&](int t) { return tkey[t] >= theta ? 1 : 0; },
       [&](int t, int pos) { clist[pos] = t; }, sh);
   // the k-th largest logit of the candidate tiles, and its equal values needed
-  auto cand = [&](int j) {
+  auto gkey = [&](int j) {
     const int v = clist[j >> 7] * TILE_V + (j & (TILE_V - 1));
-    return v < V ? fkey(ldf(tr + v)) : 0u;
+    return v < V ? (fkey(ldf(tr + v)) & KMASK) : 0u;
   };
+  const bool staged = C * TILE_V <= FILTER_STAGE;
+  if (staged)
+    for (int j = tid; j < C * TILE_V; j += TF_NT) ckey[j] = gkey(j);
+  __syncthreads();
+  auto cand = [&](int j) { return staged ? ckey[j] : gkey(j); };
   int E;
-  const uint32_t tau = radix_kth_largest(C * TILE_V, k, cand, sh, &E);
+  const uint32_t tau = radix_kth_largest(C * TILE_V, k, cand, sh, &E, LO);
   // kept tokens in index order
   const int cnt = ordered_compact(
       C * TILE_V, E,
       [&](int j) {
         const int v = clist[j >> 7] * TILE_V + (j & (TILE_V - 1));
         if (v >= V) return 0;
-        const uint32_t key = fkey(ldf(tr + v));
+        const uint32_t key = cand(j);
         return key > tau ? 1 : (key == tau ? 2 : 0);
       },
       [&](int j, int pos) {
@@ -1848,10 +2001,11 @@ __global__ void __launch_bounds__(VF_NT)
                       const int32_t* __restrict__ xhat, const uint32_t* __restrict__ cmask,
                       const float* __restrict__ log2pi, const float* __restrict__ qtok_ws,
                       const int32_t* __restrict__ tok, const uint32_t* __restrict__ ties_draft,
-                      int V, int K, int rr, int B, int Bt, float k2, uint64_t seed,
+                      int V, int K, int rr, int B, int Bt, int kf, float k2, uint64_t seed,
                       int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
                       dblast_verify_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
+  extern __shared__ float qS[];   // [B][kf]: q(v|x_<i) at the kept tokens of row i
   __shared__ FF Cz[32][32];       // soft: per position, L_z - log2 w_z
   __shared__ int X[1024];         // greedy: x-hat [B, K]
   __shared__ float piS[32], Ssum[32];
@@ -1888,15 +2042,20 @@ __global__ void __launch_bounds__(VF_NT)
       return SoftQ{stash + (m0 + i) * V, wu, codes + (m0 + i) * K * rr, Cz[i], K, rr, k2}(v);
     }
   };
+  // q at every (position, kept token), all threads; then
   // alpha_i = sum over the kept tokens of min(p'(v), q(v)): one warp per position
+  for (int pq = tid; pq < B * kf; pq += VF_NT) {
+    const int i = pq / kf, j = pq - i * kf;
+    const int rl = n * (B + 1) + i;
+    if (j < fcnt[rl]) qS[pq] = qfun(i, ftok[(size_t)rl * FILTER_MAX_K + j]);
+  }
+  __syncthreads();
   for (int i = warp; i < B; i += VF_NT / 32) {
     const int rl = n * (B + 1) + i;
     const int cnt = fcnt[rl];
     FF a{0.f, 0.f};
-    for (int j = lane; j < cnt; j += 32) {
-      const int v = ftok[(size_t)rl * FILTER_MAX_K + j];
-      a = ff_addf(a, fminf(fp[(size_t)rl * FILTER_MAX_K + j], qfun(i, v)));
-    }
+    for (int j = lane; j < cnt; j += 32)
+      a = ff_addf(a, fminf(fp[(size_t)rl * FILTER_MAX_K + j], qS[i * kf + j]));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) a = ff_add(a, ff_shfl_xor(a, o));
     if (lane == 0) alphaS[i] = ff_f(a);
@@ -1974,7 +2133,7 @@ __global__ void __launch_bounds__(VF_NT)
       int j = -1;
       bool from_p = L >= B;
       if (L < B) {
-        j = warp_inverse_cdf(cnt, [&](int jj) { return fmaxf(pk[jj] - qfun(L, tk[jj]), 0.f); },
+        j = warp_inverse_cdf(cnt, [&](int jj) { return fmaxf(pk[jj] - qS[L * kf + jj], 0.f); },
                              u3, &margin, &total);
         if (total < TIE_TOL) ties |= TIE_RMASS;
         if (j < 0) {
@@ -2036,13 +2195,14 @@ cudaError_t launch_target_filter(const StepCtx& c, const dblast_verify_out* o) {
 cudaError_t launch_filtered_verify(const StepCtx& c, const dblast_verify_out* o) {
   const WsLayout& w = c.wl;
   auto k = c.greedy ? k_filtered_verify<true> : k_filtered_verify<false>;
-  cudaError_t le = launch_dep(k, dim3(w.N), dim3(VF_NT), 0, c.stream,
+  const int kf = o->top_k;  // the kept tokens per row at most (clamped by the caller)
+  cudaError_t le = launch_dep(k, dim3(w.N), dim3(VF_NT), (size_t)w.B * kf * sizeof(float), c.stream,
       wsp<int32_t>(c, w.off_ftok), wsp<float>(c, w.off_fp), wsp<int32_t>(c, w.off_fcnt),
       wsp<uint32_t>(c, w.off_ftie), wsp<float>(c, w.off_coll), wsp<float>(c, w.off_stash),
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2),
       wsp<float2>(c, w.off_w2), wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask),
       wsp<float>(c, w.off_log2pi), wsp<float>(c, w.off_qtok), wsp<int32_t>(c, w.off_tok),
-      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, c.Bt, c.k2, c.args->seed,
+      wsp<uint32_t>(c, w.off_ties), w.V, c.head->K, w.rr, w.B, c.Bt, kf, c.k2, c.args->seed,
       c.args->pos, c.args->round, *o);
   debug_kernel("k_filtered_verify", c.stream);
   count_launches(1);
