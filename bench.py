@@ -483,12 +483,23 @@ def main():
     e2e_steps = args.e2e_steps or K_steps
     h_host = blk["hidden"].cpu().pin_memory()
     t_host = blk["target"].cpu().pin_memory()
-    res_host = {k: torch.empty_like(vouts[0][k], device="cpu").pin_memory()
-                for k in ("accepted", "n_emitted", "emitted", "exp_len")}
+    # the per-sequence results live in one device buffer (segments 16-byte
+    # aligned), so one device-to-host copy reads them back each step
+    def seg(n):
+        return (n + 3) // 4 * 4
+    sizes = [seg(N), seg(N), seg(N * (B + 1)), seg(N)]
+    offs = [sum(sizes[:j]) for j in range(4)]
+    res_dev = torch.empty(sum(sizes), dtype=torch.int32, device=dev)
+    vout_e2e = dict(vouts[0])
+    vout_e2e["accepted"] = res_dev[offs[0]:offs[0] + N]
+    vout_e2e["n_emitted"] = res_dev[offs[1]:offs[1] + N]
+    vout_e2e["emitted"] = res_dev[offs[2]:offs[2] + N * (B + 1)].view(N, B + 1)
+    vout_e2e["exp_len"] = res_dev[offs[3]:offs[3] + N].view(torch.float32)
+    res_host = torch.empty_like(res_dev, device="cpu").pin_memory()
     h_dev = [torch.empty_like(blk["hidden"]) for _ in range(2)]
     t_dev = [torch.empty_like(blk["target"]) for _ in range(2)]
     h2d = h_host.numel() * h_host.element_size() + t_host.numel() * t_host.element_size()
-    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    d2h = res_host.numel() * res_host.element_size()
     main = torch.cuda.current_stream()
     cstream = torch.cuda.Stream()
     copied = [torch.cuda.Event() for _ in range(2)]
@@ -513,11 +524,10 @@ def main():
             copy_in(b ^ 1, freed[b ^ 1] if k >= 1 else None)
         main.wait_event(copied[b])
         dblast_draft_and_verify(head, ws, h_dev[b], pos, rnd, args.T, cfg["Z_T"], seed, t_dev[b],
-                                blk["has_bonus"], impl=args.kernels, dout=dout, vout=vouts[0],
+                                blk["has_bonus"], impl=args.kernels, dout=dout, vout=vout_e2e,
                                 mode=args.mode, top_k=args.top_k, top_p=args.top_p)
         freed[b].record(main)
-        for kk, v in res_host.items():
-            v.copy_(vouts[0][kk], non_blocking=True)
+        res_host.copy_(res_dev, non_blocking=True)
     e1.record(main)
     torch.cuda.synchronize()
     ems = e0.elapsed_time(e1)

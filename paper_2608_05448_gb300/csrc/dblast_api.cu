@@ -140,7 +140,6 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_partt = take((size_t)w.nt * w.Rt * sizeof(float2));
   w.off_lt2 = take((size_t)w.Rt * sizeof(float2));
   w.off_partv = take((size_t)w.nt * w.Mpad * sizeof(float2));
-  w.off_av = take((size_t)AV_SPLIT * w.M * sizeof(float4));
   w.off_ties = take((size_t)N * sizeof(uint32_t));
   w.off_xhat = take((size_t)w.M * K * sizeof(int32_t));
   w.off_cmask = take((size_t)w.M * sizeof(uint32_t));

@@ -52,19 +52,18 @@ struct PrepLayout {
 //   zhat i32 [N] | log2pi f32 [N,K] | stash f32 [M,V] | partd float2 [nt,K,Mpad]
 //   lsep float4 [LSE_SPLIT,M,K] | lse2, lq2, w2 ff [M,K] | qtok f32 [M] | tok i32 [M]
 //   vcz float2 [M,K] | vb0 f32 [M] | partt float2 [nt,Rt] | lt2 ff [Rt]
-//   partv float2 [nt,Mpad] | av float4 [AV_SPLIT,M] | ties u32 [N]
+//   partv float2 [nt,Mpad] | ties u32 [N]
 //   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
 //   token and the consistent-branch set C_i as a bit mask over z)
 //   coll f32 [Rt]  (collision probability sum_v p(v)^2 of every target row)
 //   ftok i32 [Rt, FILTER_MAX_K] | fp f32 [Rt, FILTER_MAX_K] | fcnt i32 [Rt] | ftie u32 [Rt]
 //   (target filter: kept tokens by index, their filtered probabilities, count, top-p tie)
 constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
-constexpr int AV_SPLIT = 8;   // partial sums of the verify records per row
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
       off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
-      off_partt, off_lt2, off_partv, off_av, off_ties, off_xhat, off_cmask, off_coll, off_ftok,
+      off_partt, off_lt2, off_partv, off_ties, off_xhat, off_cmask, off_coll, off_ftok,
       off_fp, off_fcnt, off_ftie, total;
 };
 

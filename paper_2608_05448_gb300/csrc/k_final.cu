@@ -796,47 +796,10 @@ cudaError_t launch_target_stats(const StepCtx& c, const dblast_verify_out* o) {
 }
 
 // ---------------------------------------------------------------- verify side
-// Partial sums of the verify records: block (row group of 32, split), lane =
-// row.  avp[sp][m] = (alpha.hi, alpha.lo, R.hi, R.lo).
-constexpr int AVM_WARPS = 16;
-__global__ void __launch_bounds__(AVM_WARPS * 32)
-    k_verify_merge(const float2* __restrict__ partv, int nt, int M, int Mpad,
-                   float4* __restrict__ avp) {
-  griddep_wait();  // launched as a dependent of the previous kernel
-  __shared__ FF sa[AVM_WARPS][32], sr[AVM_WARPS][32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int m = blockIdx.x * 32 + lane, sp = blockIdx.y;
-  const int step = AVM_WARPS * AV_SPLIT;
-  FF a{0.f, 0.f}, r{0.f, 0.f};
-  if (m < M) {
-    int t = sp * AVM_WARPS + warp;
-    for (; t + step < nt; t += 2 * step) {
-      const float2 q0 = partv[(size_t)t * Mpad + m], q1 = partv[(size_t)(t + step) * Mpad + m];
-      a = ff_addf(ff_addf(a, q0.x), q1.x);
-      r = ff_addf(ff_addf(r, q0.y), q1.y);
-    }
-    for (; t < nt; t += step) {
-      const float2 q = partv[(size_t)t * Mpad + m];
-      a = ff_addf(a, q.x);
-      r = ff_addf(r, q.y);
-    }
-  }
-  sa[warp][lane] = a;
-  sr[warp][lane] = r;
-  __syncthreads();
-  if (warp == 0 && m < M) {
-    FF A{0.f, 0.f}, R{0.f, 0.f};
-#pragma unroll
-    for (int w = 0; w < AVM_WARPS; ++w) {
-      A = ff_add(A, sa[w][lane]);
-      R = ff_add(R, sr[w][lane]);
-    }
-    avp[(size_t)sp * M + m] = make_float4(A.hi, A.lo, R.hi, R.lo);
-  }
-}
-
-// One block per sequence: acceptance (stream 2), residual or bonus draw
-// (stream 3), expected lengths, emitted tokens, state update.
+// One block per sequence: the per-row sums of the verify records (alpha_i and
+// the residual mass, thread (s, i) over tiles s, s + S, ... with consecutive
+// threads on consecutive rows of a tile), acceptance (stream 2), residual or
+// bonus draw (stream 3), expected lengths, emitted tokens, state update.
 constexpr int VF_NT = 256;
 template <typename Tin>
 __global__ void __launch_bounds__(VF_NT)
@@ -845,7 +808,7 @@ __global__ void __launch_bounds__(VF_NT)
                    const float2* __restrict__ lse2, const float2* __restrict__ w2,
                    const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
                    const float2* __restrict__ partv, const float2* __restrict__ partt,
-                   const float4* __restrict__ avp, const int32_t* __restrict__ tok,
+                   const int32_t* __restrict__ tok,
                    const uint32_t* __restrict__ ties_draft, const float* __restrict__ coll, int V,
                    int K, int rr, int B, int Bt, int nt, int M, int Mpad, int Rt, float k2,
                    uint64_t seed,
@@ -857,9 +820,46 @@ __global__ void __launch_bounds__(VF_NT)
   __shared__ int sL;
   __shared__ uint32_t sties;
   __shared__ FF sR;
+  __shared__ FF pa[VF_NT], pr[VF_NT];
+  __shared__ FF rowA[32], rowR[32];
   const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
   const int64_t p0 = pos[n];
   const uint32_t rd = rnd[n];
+  {
+    const int S = VF_NT / B;  // tile strides per row (B <= 32)
+    FF a{0.f, 0.f}, r{0.f, 0.f};
+    if (tid < S * B) {
+      const int i = tid % B, s0 = tid / B;
+      const float2* pv = partv + (size_t)n * B + i;
+      // eight records in flight per thread
+      for (int t = s0; t < nt; t += 8 * S) {
+        float2 q[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int tj = t + j * S;
+          q[j] = tj < nt ? pv[(size_t)tj * Mpad] : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          a = ff_addf(a, q[j].x);
+          r = ff_addf(r, q[j].y);
+        }
+      }
+    }
+    pa[tid] = a;
+    pr[tid] = r;
+    __syncthreads();
+    if (tid < B) {
+      FF A{0.f, 0.f}, R{0.f, 0.f};
+      for (int s0 = 0; s0 < S; ++s0) {
+        A = ff_add(A, pa[s0 * B + tid]);
+        R = ff_add(R, pr[s0 * B + tid]);
+      }
+      rowA[tid] = A;
+      rowR[tid] = R;
+    }
+    __syncthreads();
+  }
   if (tid < 32) {
     // lane i: p(x_i), q(x_i|x_<i), acceptance
     uint32_t ties = ties_draft[n];
@@ -874,12 +874,7 @@ __global__ void __launch_bounds__(VF_NT)
       qtok = qtok_ws[m];
       const float ratio = ptok / qtok;
       A = fminf(1.f, ratio);
-      FF al{0.f, 0.f};
-      for (int sp = 0; sp < AV_SPLIT; ++sp) {
-        const float4 q = avp[(size_t)sp * M + m];
-        al = ff_add(al, FF{q.x, q.y});
-      }
-      alpha = ff_f(al);
+      alpha = ff_f(rowA[lane]);
       u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
       acc_ok = u2 < ratio;
       if (out.p_tok) out.p_tok[m] = ptok;
@@ -915,10 +910,7 @@ __global__ void __launch_bounds__(VF_NT)
     FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
     FF ed{lane < B ? cC : 0.f, 0.f};
     FF R{0.f, 0.f};
-    if (L < B && lane < AV_SPLIT) {
-      const float4 q = avp[(size_t)lane * M + n * B + L];
-      R = FF{q.z, q.w};
-    }
+    if (L < B && lane == 0) R = rowR[L];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       R = ff_add(R, ff_shfl_xor(R, o));
@@ -1001,18 +993,15 @@ template <typename Tin>
 static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out* o) {
   const int Bt = c.Bt;
   const WsLayout& w = c.wl;
-  cudaError_t le = launch_dep(k_verify_merge, dim3(ceil_div(w.M, 32), AV_SPLIT),
-                              dim3(AVM_WARPS * 32), 0, c.stream, wsp<float2>(c, w.off_partv), w.nt, w.M, w.Mpad, wsp<float4>(c, w.off_av));
-  debug_kernel("k_verify_merge", c.stream);
-  if (le == cudaSuccess) le = launch_dep(k_verify_final<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
+  cudaError_t le = launch_dep(k_verify_final<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
       static_cast<const Tin*>(o->target), wsp<float>(c, w.off_stash), prp<float>(c, c.pl.off_wu),
       wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2), wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
-      wsp<float2>(c, w.off_partt), wsp<float4>(c, w.off_av), wsp<int32_t>(c, w.off_tok),
+      wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
       wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.rr, w.B, Bt,
       w.nt, w.M, w.Mpad, w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o);
   debug_kernel("k_verify_final", c.stream);
-  count_launches(2);
+  count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
 }
 
