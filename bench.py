@@ -30,6 +30,25 @@ METRIC = "draft+verify blocks/sec and accepted tokens/sec at 1 GB300; % of roofl
 UNIT = "blocks/s"
 
 
+def job_totals(ms, counts, world, device):
+    """Whole-job figures of a replicas run: the slowest rank's time (max over
+    ranks) and the counts summed over ranks.  One rank: returned as given."""
+    if world <= 1:
+        return ms, list(counts)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    c = torch.tensor([float(x) for x in counts], device=device, dtype=torch.float64)
+    dist.all_reduce(c)
+    return float(t.item()), [int(x) for x in c.tolist()]
+
+
+def job_value(units_per_rank, world, steps, ms):
+    """The job's throughput: units processed by all ranks over the slowest rank's time."""
+    return units_per_rank * world * steps / (ms / 1e3)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -462,19 +481,11 @@ def main():
         dist.barrier()
     clk = clocks.stop()
     st = dblast_stats_get()
-    ms = ev0.elapsed_time(ev1)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
     accepted = sum(int(v["accepted"].sum()) for v in vouts)
     emitted = sum(int(v["n_emitted"].sum()) for v in vouts)
-    if world > 1:
-        tt = torch.tensor([accepted, emitted], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt)
-        accepted, emitted = int(tt[0]), int(tt[1])
+    ms, (accepted, emitted) = job_totals(ev0.elapsed_time(ev1), (accepted, emitted), world, dev)
     ms_step = ms / K_steps
-    value = N * world * K_steps / (ms / 1e3)
+    value = job_value(N, world, K_steps, ms)
 
     # end to end through the public API with host buffers (pinned), per step:
     # H2D of hidden + target, the call, D2H of the per-sequence results.  The
@@ -530,12 +541,8 @@ def main():
         res_host.copy_(res_dev, non_blocking=True)
     e1.record(main)
     torch.cuda.synchronize()
-    ems = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([ems], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ems = float(tt.item())
-    e2e_value = N * world * e2e_steps / (ems / 1e3)
+    ems, _ = job_totals(e0.elapsed_time(e1), (), world, dev)
+    e2e_value = job_value(N, world, e2e_steps, ems)
 
     if rank == 0:
         wm = work_model(cfg)
