@@ -669,6 +669,45 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Two fp32 lanes per instruction (fma/add/sub/mul .rn.f32x2): each lane is
+// rounded exactly as the scalar instruction, with half the issue slots.
+struct F2 {
+  uint64_t v;
+};
+__device__ __forceinline__ F2 f2(float lo, float hi) {
+  F2 r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r.v) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_get(F2 a, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(a.v));
+}
+__device__ __forceinline__ F2 f2_fma(F2 a, F2 b, F2 c) {
+  F2 r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r.v) : "l"(a.v), "l"(b.v), "l"(c.v));
+  return r;
+}
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+  F2 r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+__device__ __forceinline__ F2 f2_sub(F2 a, F2 b) {
+  F2 r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+__device__ __forceinline__ F2 f2_mul(F2 a, F2 b) {
+  F2 r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+__device__ __forceinline__ F2 f2_ex2(F2 a) {
+  float lo, hi;
+  f2_get(a, lo, hi);
+  return f2(ex2(lo), ex2(hi));
+}
+
 // Greedy-branch epilogue of one tile (Sec. 3.1, "Drafter sampling during
 // inference"): for every component z, the largest logit
 // l_v = base_v + b_v + D_z / (cscale sw) of this thread's 128 columns and its
@@ -1135,9 +1174,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // per-row constants: B0 here, (k2 / scale, log2 w - L + B0) per component below
       const float B0f = mok ? P.vb0[m] : 0.f;
       const float2* vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
-      float acc[32];
+      F2 acc2[16];  // columns (2j, 2j+1)
 #pragma unroll
-      for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+      for (int j = 0; j < 16; ++j) acc2[j] = f2(0.f, 0.f);
       bool ok = true;
       for (int g = 0; g < ngroups; ++g) {
         const int gs = g & 1;
@@ -1158,22 +1197,53 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive_taken(&sempty[gs]);
           }
+          const F2 czx = f2(cz.x, cz.x), czy = f2(cz.y, cz.y);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) acc[j] += ex2(fmaf(__uint_as_float(r0[j]), cz.x, cz.y));
+          for (int j = 0; j < 16; ++j)
+            acc2[j] = f2_add(acc2[j], f2_ex2(f2_fma(f2(__uint_as_float(r0[2 * j]),
+                                                       __uint_as_float(r0[2 * j + 1])),
+                                                    czx, czy)));
         }
       }
       if (!ok) break;
-      // four partial sums per quantity keep the add chains short
-      float As4[4] = {0.f, 0.f, 0.f, 0.f}, Rs4[4] = {0.f, 0.f, 0.f, 0.f};
+      // four partial sums per quantity keep the add chains short: As2[h]
+      // holds the sums of columns j with j & 3 == 2h and 2h + 1
+      F2 As2[2] = {f2(0.f, 0.f), f2(0.f, 0.f)}, Rs2[2] = {f2(0.f, 0.f), f2(0.f, 0.f)};
       const int n = m / P.B, i = m - n * P.B;
       const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
-      const float nB0 = -B0f;
-      auto accumulate = [&](int j, float sv, float tv) {
-        const float qv = ex2(fmaf(sv, P.k2, nB0)) * acc[j];
+      const F2 k2x = f2(P.k2, P.k2), nB0x = f2(-B0f, -B0f);
+      const F2 nLtx = f2(-Lt.x, -Lt.x), Ltyx = f2(Lt.y, Lt.y);
+      // columns 2jp and 2jp + 1 together
+      auto accumulate2 = [&](int jp, float s0, float s1, float t0, float t1) {
+        const F2 qv = f2_mul(f2_ex2(f2_fma(f2(s0, s1), k2x, nB0x)), acc2[jp]);
+        const F2 pv = f2_ex2(f2_sub(f2_fma(f2(t0, t1), k2x, nLtx), Ltyx));
+        float q0, q1, p0, p1;
+        f2_get(qv, q0, q1);
+        f2_get(pv, p0, p1);
+        const F2 mn = f2(fminf(p0, q0), fminf(p1, q1));
+        As2[jp & 1] = f2_add(As2[jp & 1], mn);
+        Rs2[jp & 1] = f2_add(Rs2[jp & 1], f2_sub(pv, mn));
+      };
+      // one column (ragged tail): the same arithmetic on one lane of a pair
+      auto accumulate1 = [&](int j, float sv, float tv) {
+        float a0, a1;
+        f2_get(acc2[j >> 1], a0, a1);
+        const float qv = ex2(fmaf(sv, P.k2, -B0f)) * ((j & 1) ? a1 : a0);
         const float pv = ex2(fmaf(tv, P.k2, -Lt.x) - Lt.y);
         const float mn = fminf(pv, qv);
-        As4[j & 3] += mn;
-        Rs4[j & 3] += pv - mn;
+        const int h = (j >> 1) & 1;
+        float x0, x1, y0, y1;
+        f2_get(As2[h], x0, x1);
+        f2_get(Rs2[h], y0, y1);
+        if (j & 1) {
+          x1 += mn;
+          y1 += pv - mn;
+        } else {
+          x0 += mn;
+          y0 += pv - mn;
+        }
+        As2[h] = f2(x0, x1);
+        Rs2[h] = f2(y0, y1);
       };
       const bool full_cols = v0 + 32 <= P.V;
       if (P.use_x) {
@@ -1202,11 +1272,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (full_cols) {
 #pragma unroll
-              for (int u = 0; u < 8; ++u) accumulate(k * 8 + u, sv[u], tv[u]);
+              for (int u = 0; u < 8; u += 2)
+                accumulate2((k * 8 + u) >> 1, sv[u], sv[u + 1], tv[u], tv[u + 1]);
             } else {
 #pragma unroll
               for (int u = 0; u < 8; ++u)
-                if (v0 + k * 8 + u < P.V) accumulate(k * 8 + u, sv[u], tv[u]);
+                if (v0 + k * 8 + u < P.V) accumulate1(k * 8 + u, sv[u], tv[u]);
             }
           }
         }
@@ -1217,8 +1288,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
 #pragma unroll
         for (int u = 0; u < 32; ++u)
-          if (v0 + u < P.V) accumulate(u, srow[u], __bfloat162float(trow[u]));
+          if (v0 + u < P.V) accumulate1(u, srow[u], __bfloat162float(trow[u]));
       }
+      float As4[4], Rs4[4];
+      f2_get(As2[0], As4[0], As4[1]);
+      f2_get(As2[1], As4[2], As4[3]);
+      f2_get(Rs2[0], Rs4[0], Rs4[1]);
+      f2_get(Rs2[1], Rs4[2], Rs4[3]);
       const float As = (As4[0] + As4[1]) + (As4[2] + As4[3]);
       const float Rs = (Rs4[0] + Rs4[1]) + (Rs4[2] + Rs4[3]);
       // the other column quarters of this row, then one record per (tile, row)
