@@ -140,3 +140,27 @@ def test_filter_arguments_are_checked_before_launch(top_k, top_p, status):
     got = lib.dblast_verify_block(ctypes.byref(h), ctypes.byref(a), ctypes.byref(v), p,
                                   need - 1, None)
     assert got == (3 if status == 0 else status)
+
+
+@pytest.mark.parametrize("mutate,status", [
+    (lambda a, al: setattr(al, "tokens", None), 1),
+    (lambda a, al: setattr(al, "target", None), 1),
+    (lambda a, al: setattr(al, "tau", -0.1), 1),
+    (lambda a, al: setattr(al, "tau", float("inf")), 1),
+    (lambda a, al: setattr(a, "mode", 1), 1),        # the objectives use the soft proposal
+    (lambda a, al: setattr(al, "top_k", 300), 2),
+    (lambda a, al: None, 3),                          # accepted: stops at the short workspace
+])
+def test_al_objective_arguments_are_checked_before_launch(mutate, status):
+    lib = bd.lib()
+    h = fake_head(V=1000, H=64, K=4, r=8)
+    h.prep_bytes = lib.dblast_prep_bytes(ctypes.byref(h))
+    a = _args()
+    p = ctypes.c_void_p(1 << 20)
+    al = bd.CAlArgs()
+    al.tokens, al.target, al.has_bonus, al.tau = p, p, 1, 0.1
+    mutate(a, al)
+    need = lib.dblast_workspace_bytes(ctypes.byref(h), 2, 3, 1)
+    got = lib.dblast_al_objective(ctypes.byref(h), ctypes.byref(a), ctypes.byref(al), p,
+                                  need - 1, None)
+    assert got == status
