@@ -42,6 +42,13 @@ void debug_kernel(const char* name, cudaStream_t s) {
   fprintf(stderr, "dblast debug kernel: %-20s %s\n", name, cudaGetErrorString(e));
 }
 
+// DBLAST_FUSE_TSTATS=0: target statistics as a kernel of their own (the
+// fused step's default computes them in the draft pass)
+static bool fuse_tstats_enabled() {
+  const char* e = getenv("DBLAST_FUSE_TSTATS");
+  return !(e && e[0] == '0');
+}
+
 static cudaError_t dbg(cudaError_t e, const char* what, cudaStream_t s) {
   if (e != cudaSuccess || !debug_sync()) return e;
   e = cudaStreamSynchronize(s);
@@ -215,6 +222,8 @@ static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, 
   c->greedy = a->mode == DBLAST_MODE_GREEDY;
   c->target = nullptr;
   c->Bt = a->B + (has_bonus ? 1 : 0);
+  c->fuse_tstats = false;
+  c->lse_target = nullptr;
   return DBLAST_OK;
 }
 
@@ -353,6 +362,16 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   }
   c.target = vout->target;
   c.Bt = c.args->B + (vout->has_bonus ? 1 : 0);
+  // bf16 targets with 16-byte rows: the draft pass's idle warps compute the
+  // target statistics while its tensor cores run.  It pays where the second
+  // stream's work after the draft pass (target statistics, filter) outlasts
+  // the draft finalize kernels: the greedy mode and the target filter.  In
+  // the plain stochastic step the two are about equal, and the extra memory
+  // traffic would slow the draft pass by more than it saves.
+  c.fuse_tstats = c.tc && c.head->dtype == DBLAST_BF16 && (c.head->V % 8) == 0 &&
+                  aligned16(vout->target) && (c.greedy || filter_on(c.head, vout)) &&
+                  fuse_tstats_enabled();
+  c.lse_target = vout->lse_target;
   g_calls.fetch_add(2, std::memory_order_relaxed);
   std::lock_guard<std::mutex> lk(g_side_mu);
   SideStream* ss = nullptr;
@@ -372,20 +391,24 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
     e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
     pass_event_end(0, c.stream);
   }
-  // join 1, fork 2: target statistics | draft finalize
+  // join 1, fork 2: target statistics (unless the draft pass took them) and
+  // the target filter | draft finalize
   if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[1], 0);
-  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[2], c.stream);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[2], 0);
-  if (e == cudaSuccess) e = launch_target_stats(side, vout);
-  if (e == cudaSuccess && filter_on(c.head, vout)) {
-    const dblast_verify_out f = filter_args(c.head, vout);
-    e = launch_target_filter(side, &f);
+  const bool side_work = !c.fuse_tstats || filter_on(c.head, vout);
+  if (side_work) {
+    if (e == cudaSuccess) e = cudaEventRecord(ss->ev[2], c.stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[2], 0);
+    if (e == cudaSuccess && !c.fuse_tstats) e = launch_target_stats(side, vout);
+    if (e == cudaSuccess && filter_on(c.head, vout)) {
+      const dblast_verify_out f = filter_args(c.head, vout);
+      e = launch_target_filter(side, &f);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
   }
-  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
   if (e == cudaSuccess)
     e = c.greedy ? launch_greedy_draft_finalize(c, dout) : launch_draft_finalize(c, dout);
   // join 2
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[3], 0);
+  if (e == cudaSuccess && side_work) e = cudaStreamWaitEvent(c.stream, ss->ev[3], 0);
   if (e == cudaSuccess) e = verify_passes(c, vout);
   return cuda_status(e);
 }

@@ -245,6 +245,8 @@ struct StepCtx {
   bool greedy;  // greedy-branch mode (App. A) instead of sampled draft tokens
   const void* target;  // verify only: [N, Bt, V]
   int Bt;              // target rows per sequence (B + has_bonus)
+  bool fuse_tstats;    // fused step: the draft pass computes the target statistics
+  float* lse_target;   // its natural log-sum-exp output (or null)
 };
 
 template <typename T> T* wsp(const StepCtx& c, size_t off) { return reinterpret_cast<T*>(c.ws + off); }

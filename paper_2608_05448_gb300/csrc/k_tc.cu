@@ -364,7 +364,7 @@ struct DCfg {
   static constexpr int STAGE_B = BROWS * BK * 2;           // 16 or 32 KB
   static constexpr int STAGE = DSTAGE_A + STAGE_B;         // 32 or 48 KB
   static constexpr int TX = PAIR ? 2 * STAGE : STAGE;      // bytes completing one full barrier
-  static constexpr size_t SMEM = (size_t)STAGES * STAGE + DAZ_BYTES + DVB_BYTES + 256 + 1024;
+  static constexpr size_t SMEM = (size_t)STAGES * STAGE + DAZ_BYTES + DVB_BYTES + 256 + 64 + 1024;
 };
 static_assert(DCfg<true>::SMEM <= 227 * 1024 && DCfg<false>::SMEM <= 227 * 1024, "shared memory");
 
@@ -386,6 +386,15 @@ struct Params {
   size_t split_stride;       // elements between the split-K partial outputs
   DevStatus* status;
   uint32_t spin_limit;
+  // target statistics computed by the idle warps 2-3 of the draft pass
+  // (fused step, bf16 target with V % 8 == 0); tgt == nullptr: off
+  const __nv_bfloat16* tgt;  // [t_rows, V]
+  int t_rows, t_Bt, t_B, t_Rt, t_nt;
+  float t_k2;                // log2(e) / T
+  float2* t_partt;           // [nt, Rt] tile records (tmax, sum 2^((t - tmax) k2))
+  float2* t_lt2;             // [Rt] log2 sum_v 2^(t_v k2) as a float pair
+  float* t_coll;             // [Rt] sum_v p(v)^2
+  float* t_lse;              // [t_rows] natural log-sum-exp, or null
 };
 
 // Tile `slot` of this CTA.  The CTAs of one cluster (cs of them) share a
@@ -959,6 +968,127 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
   }
 }
 
+// Target statistics on the idle warps 2-3 of the draft pass (fused step):
+// the records of the stand-alone target-statistics kernel (per 128-token tile
+// (tmax, sum 2^((t - tmax) k2)), per row the log-sum-exp pair and the
+// collision probability), computed while the tensor cores run.  Rows go
+// round-robin over the CTAs; in a row the two warps take alternate runs of
+// eight tiles, four lanes per tile (64 contiguous bytes each).  One run is in
+// registers at a time: the 56 registers of these warps hold no second one.
+__device__ __forceinline__ void ts_load(const uint4* tr, int nchunk, int c0, uint4 (&d)[4]) {
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int c = c0 + k;
+    d[k] = c < nchunk ? __ldg(tr + c)
+                      : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+  }
+}
+__device__ __forceinline__ void draft_target_stats(const Params& P, int w, int lane, float* xch) {
+  const int q = lane >> 2, ql = lane & 3;
+  const int nchunk = P.V >> 3;
+  const float k2 = P.t_k2;
+  const int ngroups = (P.t_nt + 15) >> 4;  // 16 tiles per run pair, 8 per warp
+  for (int row = blockIdx.x; row < P.t_rows; row += gridDim.x) {
+    const int n = row / P.t_Bt, i = row - n * P.t_Bt;
+    const int rl = n * (P.t_B + 1) + i;
+    const uint4* tr = reinterpret_cast<const uint4*>(P.tgt + (size_t)row * P.V);
+    float rmax = -INFINITY, rsq = 0.f;
+    FF rsum{0.f, 0.f};
+    uint4 cur[4];
+    int t = w * 8 + q;
+    ts_load(tr, nchunk, t * 16 + ql * 4, cur);
+    for (int g = 0; g < ngroups; ++g, t += 16) {
+
+      __nv_bfloat162 m2 = __float2bfloat162_rn(-INFINITY);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint4 u = cur[k];
+        m2 = __hmax2(m2, __hmax2(__hmax2(*reinterpret_cast<const __nv_bfloat162*>(&u.x),
+                                         *reinterpret_cast<const __nv_bfloat162*>(&u.y)),
+                                 __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&u.z),
+                                         *reinterpret_cast<const __nv_bfloat162*>(&u.w))));
+      }
+      float mx = fmaxf(__low2float(m2), __high2float(m2));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      float sa = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t uu[4] = {cur[k].x, cur[k].y, cur[k].z, cur[k].w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const float a = __uint_as_float(uu[h] << 16), b = __uint_as_float(uu[h] & 0xFFFF0000u);
+          const float ea = ex2((a - mx) * k2), eb = ex2((b - mx) * k2);
+          sa += ea + eb;
+          s2 = fmaf(ea, ea, fmaf(eb, eb, s2));
+        }
+      }
+      sa += __shfl_xor_sync(0xffffffffu, sa, 1);
+      sa += __shfl_xor_sync(0xffffffffu, sa, 2);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, 1);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, 2);
+      if (t < P.t_nt) {
+        if (ql == 0) P.t_partt[(size_t)t * P.t_Rt + rl] = make_float2(mx, sa);
+        if (mx > rmax) {
+          const float f = exp2f((rmax - mx) * k2);
+          rsum = ff_mulf(rsum, f);
+          rsq *= f * f;
+          rmax = mx;
+        }
+        const float gsc = exp2f((mx - rmax) * k2);
+        rsum = ff_addf(rsum, sa * gsc);
+        rsq = fmaf(s2, gsc * gsc, rsq);
+      }
+      if (g + 1 < ngroups) ts_load(tr, nchunk, (t + 16) * 16 + ql * 4, cur);
+    }
+    // the quads of this warp (the four lanes of a quad hold the same state)
+    float M1 = rmax;
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) M1 = fmaxf(M1, __shfl_xor_sync(0xffffffffu, M1, o));
+    FF S1{0.f, 0.f};
+    float Q1 = 0.f;
+    if (ql == 0 && M1 != -INFINITY && rmax != -INFINITY) {
+      const float f = exp2f((rmax - M1) * k2);
+      S1 = ff_mulf(rsum, f);
+      Q1 = rsq * f * f;
+    }
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      const FF o1{__shfl_xor_sync(0xffffffffu, S1.hi, o), __shfl_xor_sync(0xffffffffu, S1.lo, o)};
+      S1 = ff_add(S1, o1);
+      Q1 += __shfl_xor_sync(0xffffffffu, Q1, o);
+    }
+    if (lane == 0) {
+      xch[w * 4] = M1;
+      xch[w * 4 + 1] = S1.hi;
+      xch[w * 4 + 2] = S1.lo;
+      xch[w * 4 + 3] = Q1;
+    }
+    named_bar_sync(8, 64);
+    if (w == 0 && lane == 0) {
+      const float M2 = fmaxf(xch[0], xch[4]);
+      FF S{0.f, 0.f};
+      float Q = 0.f;
+      if (M2 != -INFINITY)
+        for (int k = 0; k < 2; ++k) {
+          const float mk = xch[4 * k];
+          if (mk != -INFINITY) {
+            const float f = exp2f((mk - M2) * k2);
+            S = ff_add(S, ff_mulf(FF{xch[4 * k + 1], xch[4 * k + 2]}, f));
+            Q = fmaf(xch[4 * k + 3], f * f, Q);
+          }
+        }
+      const FF L = (M2 == -INFINITY || !(S.hi > 0.f)) ? FF{-INFINITY, 0.f}
+                                                     : ff_add(ff_prod(M2, k2), ff_log2(S));
+      P.t_lt2[rl] = ff_st(L);
+      const float sf = ff_f(S);
+      P.t_coll[rl] = sf > 0.f ? Q / (sf * sf) : 0.f;
+      if (P.t_lse) P.t_lse[row] = ff_f(L) * LN2;
+    }
+    named_bar_sync(8, 64);
+  }
+}
+
 template <bool PAIR, bool GREEDY = false>
 __global__ void __launch_bounds__(D_THREADS, 1)
     k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
@@ -984,6 +1114,7 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   uint64_t* vbar = bfull + 9;               // a tile's vocabulary bias staged (256 epilogue threads)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 10);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* xch = reinterpret_cast<float*>(bars + 32);  // 64 bytes after the barrier block
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Sched S = sched_of(P);
@@ -1042,6 +1173,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
     else if (warp == 1 && lane == 0 && (!PAIR || S.rank == 0))
       draft_mma<PAIR>(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl,
                       my_tiles);
+    else if ((warp == 2 || warp == 3) && P.tgt != nullptr)
+      draft_target_stats(P, warp - 2, lane, xch);
   }
 
   tc_fence_before();
@@ -1738,6 +1871,19 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   P.partd = wsp<float2>(c, w.off_partd);
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
+  if (c.fuse_tstats) {
+    P.tgt = static_cast<const __nv_bfloat16*>(c.target);
+    P.t_rows = w.N * c.Bt;
+    P.t_Bt = c.Bt;
+    P.t_B = w.B;
+    P.t_Rt = w.Rt;
+    P.t_nt = w.nt;
+    P.t_k2 = LOG2E / c.args->temperature;
+    P.t_partt = wsp<float2>(c, w.off_partt);
+    P.t_lt2 = wsp<float2>(c, w.off_lt2);
+    P.t_coll = wsp<float>(c, w.off_coll);
+    P.t_lse = c.lse_target;
+  }
   if (c.greedy)
     return pair ? tc::launch<true, true>(ma, mb, mca, mcb, P, c.stream)
                 : tc::launch<false, true>(ma, mb, mca, mcb, P, c.stream);

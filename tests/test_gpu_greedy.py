@@ -62,7 +62,10 @@ def test_greedy_qwen3_8b_batched_sampled(impl):
 
 
 def test_greedy_split_calls_equal_fused_call():
-    """dblast_draft_block + dblast_verify_block == dblast_draft_and_verify."""
+    """dblast_draft_block + dblast_verify_block == dblast_draft_and_verify
+    (decisions identical; the fused call computes the target statistics in the
+    draft pass with another summation order, so floats agree within the parity
+    tolerances)."""
     from paper_2608_05448_gb300 import (Head, Workspace, dblast_draft_and_verify,
                                         dblast_draft_block, dblast_verify_block)
     cfg = synth.config("qwen3_8b_b32", V=3000, H=128, K=6, r=8, B=7, N=5)
@@ -84,7 +87,11 @@ def test_greedy_split_calls_equal_fused_call():
                      pos.cpu()))
     for a, b in zip(outs[0][:2], outs[1][:2]):
         for k in a:
-            assert torch.equal(a[k], b[k]), k
+            if a[k].is_floating_point():
+                atol = 1e-4 if k in ("lse_target", "lse") else 1e-6
+                assert torch.allclose(a[k], b[k], rtol=1e-4, atol=atol, equal_nan=True), k
+            else:
+                assert torch.equal(a[k], b[k]), k
     assert torch.equal(outs[0][2], outs[1][2])
 
 

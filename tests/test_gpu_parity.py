@@ -185,3 +185,32 @@ def test_serving_batch_four_rounds_sampled(B):
         assert torch.equal(rnd.cpu(), rnd0.cpu() + 1)
         del blk, gpu
     assert int(rnd[0]) == rounds
+
+
+@pytest.mark.parametrize("mode,top_k,top_p", [("soft", 20, 0.95), ("greedy", 0, 0.0)])
+def test_target_statistics_in_the_draft_pass_match_the_separate_kernel(mode, top_k, top_p):
+    """The fused step computes the target statistics in the draft pass's idle
+    warps (greedy mode, or a target filter on); with DBLAST_FUSE_TSTATS=0 a
+    kernel of its own does.  Decisions are
+    identical and the floats agree within the parity tolerances (another
+    summation order)."""
+    import os
+    cfg = synth.config("qwen3_8b_b32", V=6000, H=128, K=4, r=8, B=9, N=6)
+    head = synth.make_head(cfg, "cuda")
+    blk = synth.make_block(cfg, head, 0, "cuda")
+    res = []
+    for fuse in ("1", "0"):
+        os.environ["DBLAST_FUSE_TSTATS"] = fuse
+        try:
+            pos, rnd = synth.initial_state(cfg, "cuda")
+            res.append(parity.run_gpu(head, blk, 0.9, 1.0, 6, pos, rnd, impl="tcgen05", mode=mode,
+                                      top_k=top_k, top_p=top_p))
+        finally:
+            os.environ.pop("DBLAST_FUSE_TSTATS", None)
+    for k in res[0]:
+        a, b = res[0][k], res[1][k]
+        if a.is_floating_point():
+            atol = 1e-4 if k in ("lse_target", "lse") else 1e-6
+            assert torch.allclose(a, b, rtol=1e-4, atol=atol, equal_nan=True), k
+        else:
+            assert torch.equal(a, b), k
