@@ -556,7 +556,9 @@ def main():
         tr_path = os.path.join(ROOT, "profiles", "draft_pass_%s_traffic.json" % cfg["name"])
         if args.mode == "greedy":
             tr_path = os.path.join(ROOT, "profiles", "draft_pass_greedy_%s_traffic.json" % cfg["name"])
-        if os.path.exists(tr_path) and st["tc_launches"] > 0 and not args.n_seqs:
+        elif args.top_k > 0 or 0.0 < args.top_p < 1.0:
+            tr_path = ""  # with a filter the soft pass also reads the target: not captured
+        if tr_path and os.path.exists(tr_path) and st["tc_launches"] > 0 and not args.n_seqs:
             d = json.load(open(tr_path))
             src = os.path.join(ROOT, d.get("source", ""))
             if os.path.exists(src):
