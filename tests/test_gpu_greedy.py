@@ -135,7 +135,37 @@ def test_greedy_four_rounds_carry_state(impl):
     assert int(rnd[0]) == 4
 
 
-def test_greedy_serving_batch_sampled():
-    """Serving step at full size (N=256, B=8): sampled sequences checked."""
+@pytest.mark.parametrize("impl", IMPLS)
+def test_greedy_qwen3_4b_single_sequence_full(impl):
+    cfg = synth.config("qwen3_4b_b1")
+    _skip_unsupported(cfg, impl)
+    _case(cfg, 1.0, 1.0, seed=3, impl=impl)
+
+
+@pytest.mark.parametrize("K", [16, 1])
+def test_greedy_entropy_sweep_sampled(K):
+    """Entropy-sweep shapes at full size (N=64, r=32, V=151936), the K=16 drafter
+    and the K=1 independent-block baseline, high-entropy cell."""
+    cfg = synth.config("sweep_k16", K=K, sigma=1.0)
+    _case(cfg, 1.5, 1.0, seed=8, impl="tcgen05", seqs=[0, 63])
+
+
+def test_greedy_serving_batch_four_rounds_sampled():
+    """Serving step at full size (N=256, B=8): state carried over four rounds,
+    fresh hidden states and targets each round, sampled sequences checked."""
+    from paper_2608_05448_gb300 import Head, Workspace
     cfg = synth.config("serve_b8")
-    _case(cfg, 1.0, 1.0, seed=21, impl="tcgen05", seqs=[3, 255])
+    head_t = synth.make_head(cfg, "cuda")
+    head = Head.from_dict(head_t)
+    ws = Workspace(head, cfg["N"], cfg["B"], True)
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    seqs = [3, 255]
+    for rd in range(4):
+        blk = synth.make_block(cfg, head_t, rd, "cuda")
+        pos0, rnd0 = pos.clone(), rnd.clone()
+        gpu = parity.run_gpu(head_t, blk, 1.0, 1.0, 21, pos, rnd, head=head, ws=ws, mode="greedy")
+        orc = parity.run_oracle(head_t, blk, 1.0, 1.0, 21, pos0, rnd0, seqs, mode="greedy")
+        parity.compare_greedy(gpu, orc, seqs)
+        assert torch.equal(pos.cpu(), pos0.cpu() + gpu["n_emitted"].long())
+        del blk, gpu
+    assert int(rnd[0]) == 4
