@@ -74,3 +74,16 @@ def test_filter_top_k_one_accepts_exactly_the_target_argmax():
             ne = int(gpu["n_emitted"][n])
             assert em[ne - 1] == int(top[n, ne - 1])
         assert torch.allclose(gpu["collision"], torch.ones_like(gpu["collision"]))
+
+
+@pytest.mark.parametrize("mode", ["soft", "greedy"])
+def test_filter_qwen3_4b_single_sequence(mode):
+    cfg = synth.config("qwen3_4b_b1")
+    _case(cfg, 0.7, 1.0, 2, "tcgen05", mode, 20, 0.8)
+
+
+@pytest.mark.parametrize("mode", ["soft", "greedy"])
+def test_filter_serving_b32_sampled(mode):
+    """Serving shapes (N=256, B=32): 8,448 filtered target rows per step."""
+    cfg = synth.config("serve_b32")
+    _case(cfg, 1.0, 1.0, 4, "tcgen05", mode, 20, 0.95, seqs=[0, 255])
