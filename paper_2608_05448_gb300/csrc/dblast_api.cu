@@ -405,6 +405,13 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
     }
     if (e == cudaSuccess) e = cudaEventRecord(ss->ev[3], side.stream);
   }
+  // greedy mode with the statistics in the draft pass and no filter: nothing
+  // runs beside the draft finalize, so one kernel per sequence takes the
+  // greedy draft and verifies it
+  if (c.greedy && c.fuse_tstats && !side_work) {
+    if (e == cudaSuccess) e = launch_greedy_step_finalize(c, dout, vout);
+    return cuda_status(e);
+  }
   if (e == cudaSuccess)
     e = c.greedy ? launch_greedy_draft_finalize(c, dout) : launch_draft_finalize(c, dout);
   // join 2

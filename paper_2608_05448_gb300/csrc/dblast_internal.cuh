@@ -301,6 +301,8 @@ cudaError_t launch_verify_pass_simt(const StepCtx& c);
 cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
 cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* out);
 cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* out);
+cudaError_t launch_greedy_step_finalize(const StepCtx& c, const dblast_draft_out* dout,
+                                        const dblast_verify_out* out);
 cudaError_t launch_target_filter(const StepCtx& c, const dblast_verify_out* o);
 cudaError_t launch_filtered_verify(const StepCtx& c, const dblast_verify_out* o);
 cudaError_t launch_determinism(const StepCtx& c, const dblast_verify_out* o, int rows, int b,

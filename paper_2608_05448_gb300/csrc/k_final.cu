@@ -1069,22 +1069,20 @@ __global__ void __launch_bounds__(LSE_WARPS * 32)
 // One block per sequence, thread t = (i, z) with i = t / K: x-hat_{i,z}, the
 // block, C_i (bit z of cmask[m]: branch z drafted x_j at every j < i),
 // pi~_{i,z} and q_greedy(x_i|x_<i), and the user-visible draft outputs.
-__global__ void __launch_bounds__(1024)
-    k_greedy_draft(const float4* __restrict__ lsep, const float* __restrict__ log2pi,
-                   const int32_t* __restrict__ zhat, int B, int K, int M, int V,
-                   int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
-                   float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
-                   dblast_draft_out out) {
-  griddep_wait();  // launched as a dependent of the previous kernel
-  __shared__ int X[1024];
-  __shared__ int tokS[32];
-  __shared__ uint32_t eqS[32], cmS[32];
-  __shared__ float piS[32], sumS[32];
-  const int n = blockIdx.x, t = threadIdx.x;
-  const int i = t / K, z = t - i * K;
-  const bool ok = i < B;
-  const size_t m = (size_t)n * B + (ok ? i : 0);
-  if (ok) {
+// The draft side of one sequence, for any block size: x-hat_{i,z} (thread
+// (i, z), strided), the block, C_i (bit z of cmask[m]: branch z drafted x_j at
+// every j < i), pi~_{i,z} and q_greedy(x_i|x_<i), and the draft outputs.
+// Shared arrays: X [B K], tokS, eqS, cmS, piS, sumS [32].
+__device__ void greedy_draft_body(const float4* __restrict__ lsep, const float* __restrict__ log2pi,
+                                  const int32_t* __restrict__ zhat, int n, int B, int K, int M,
+                                  int V, int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
+                                  float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
+                                  const dblast_draft_out& out, int* X, int* tokS, uint32_t* eqS,
+                                  uint32_t* cmS, float* piS, float* sumS, float* qS) {
+  const int nt = blockDim.x;
+  for (int t = threadIdx.x; t < B * K; t += nt) {
+    const int i = t / K, z = t - i * K;
+    const size_t m = (size_t)n * B + i;
     float mx = -INFINITY;
     int ix = 0x7fffffff;
 #pragma unroll
@@ -1097,15 +1095,19 @@ __global__ void __launch_bounds__(1024)
     xhat_ws[m * K + z] = ix;
     if (out.branch_tokens) out.branch_tokens[m * K + z] = ix;
   }
-  if (t < K) piS[t] = exp2f(log2pi[n * K + t]);  // -inf (Z_T = 0) gives 0
-  if (t < 32) eqS[t] = 0u;
+  if ((int)threadIdx.x < K) piS[threadIdx.x] = exp2f(log2pi[n * K + threadIdx.x]);  // -inf gives 0
+  if (threadIdx.x < 32) eqS[threadIdx.x] = 0u;
   __syncthreads();
   const int zh = zhat[n];
-  if (t < B) tokS[t] = X[t * K + zh];
+  if ((int)threadIdx.x < B) tokS[threadIdx.x] = X[threadIdx.x * K + zh];
   __syncthreads();
-  if (ok && X[t] == tokS[i]) atomicOr(&eqS[i], 1u << z);
+  for (int t = threadIdx.x; t < B * K; t += nt) {
+    const int i = t / K, z = t - i * K;
+    if (X[t] == tokS[i]) atomicOr(&eqS[i], 1u << z);
+  }
   __syncthreads();
-  if (t < B) {  // C_t = branches that drafted x_j at every j < t
+  if ((int)threadIdx.x < B) {  // C_t = branches that drafted x_j at every j < t
+    const int t = threadIdx.x;
     uint32_t c = (K >= 32) ? 0xffffffffu : ((1u << K) - 1u);
     for (int j = 0; j < t; ++j) c &= eqS[j];
     cmS[t] = c;
@@ -1121,18 +1123,36 @@ __global__ void __launch_bounds__(1024)
     const float qt = S > 0.f ? Q / S : 0.f;
     tok_ws[mt] = tokS[t];
     qtok_ws[mt] = qt;
+    qS[t] = qt;
     cmask_ws[mt] = c;
     if (out.tokens) out.tokens[mt] = tokS[t];
     if (out.q_tok) out.q_tok[mt] = qt;
   }
   __syncthreads();
-  if (ok && out.logw) {
-    const bool in = (cmS[i] >> z) & 1u;
-    const float w = (in && sumS[i] > 0.f) ? piS[z] / sumS[i] : 0.f;
-    out.logw[m * K + z] = w > 0.f ? logf(w) : -INFINITY;
-  }
-  if (t < K && out.pi) out.pi[n * K + t] = piS[t];
-  if (t == 0 && out.z_hat) out.z_hat[n] = zh;
+  if (out.logw)
+    for (int t = threadIdx.x; t < B * K; t += nt) {
+      const int i = t / K, z = t - i * K;
+      const bool in = (cmS[i] >> z) & 1u;
+      const float w = (in && sumS[i] > 0.f) ? piS[z] / sumS[i] : 0.f;
+      out.logw[((size_t)n * B + i) * K + z] = w > 0.f ? logf(w) : -INFINITY;
+    }
+  if ((int)threadIdx.x < K && out.pi) out.pi[n * K + threadIdx.x] = piS[threadIdx.x];
+  if (threadIdx.x == 0 && out.z_hat) out.z_hat[n] = zh;
+}
+
+__global__ void __launch_bounds__(1024)
+    k_greedy_draft(const float4* __restrict__ lsep, const float* __restrict__ log2pi,
+                   const int32_t* __restrict__ zhat, int B, int K, int M, int V,
+                   int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
+                   float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
+                   dblast_draft_out out) {
+  griddep_wait();  // launched as a dependent of the previous kernel
+  __shared__ int X[1024];
+  __shared__ int tokS[32];
+  __shared__ uint32_t eqS[32], cmS[32];
+  __shared__ float piS[32], sumS[32], qS[32];
+  greedy_draft_body(lsep, log2pi, zhat, blockIdx.x, B, K, M, V, xhat_ws, tok_ws, qtok_ws, cmask_ws,
+                    out, X, tokS, eqS, cmS, piS, sumS, qS);
 }
 
 cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* outp) {
@@ -1184,16 +1204,28 @@ template <typename Tin> struct GreedyResidTokenMass {  // [p(v) - q_greedy(v)]_+
 // One block per sequence: p at the atoms of q_greedy, acceptance (stream 2),
 // alpha_i = sum over atoms of min(p, q), residual or bonus draw (stream 3),
 // expected lengths, emitted tokens, state update.
-template <typename Tin>
+// The draft side when the verify kernel also takes the greedy draft (fused
+// step): the argmax partials in, the draft outputs and workspace rows out.
+struct GreedyDraftArgs {
+  const float4* lsep;
+  const int32_t* zhat;
+  int M;
+  int32_t* xhat_ws;
+  int32_t* tok_ws;
+  float* qtok_ws;
+  uint32_t* cmask_ws;
+  dblast_draft_out out;
+};
+
+template <typename Tin, bool WITH_DRAFT>
 __global__ void __launch_bounds__(VF_NT)
     k_greedy_verify(const Tin* __restrict__ target, const float* __restrict__ log2pi,
-                    const int32_t* __restrict__ xhat, const uint32_t* __restrict__ cmask,
-                    const float* __restrict__ qtok_ws, const float2* __restrict__ lt2,
-                    const float2* __restrict__ partt, const int32_t* __restrict__ tok,
-                    const uint32_t* __restrict__ ties_draft, const float* __restrict__ coll,
+                    const int32_t* xhat, const uint32_t* cmask, const float* qtok_ws,
+                    const float2* __restrict__ lt2, const float2* __restrict__ partt,
+                    const int32_t* tok, const uint32_t* ties_draft, const float* __restrict__ coll,
                     int V, int K, int B, int Bt, int nt, int Rt, float k2, uint64_t seed,
-                    int64_t* __restrict__ pos,
-                    uint32_t* __restrict__ rnd, dblast_verify_out out) {
+                    int64_t* __restrict__ pos, uint32_t* __restrict__ rnd, dblast_verify_out out,
+                    GreedyDraftArgs gd) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<VF_NT> fs;
   __shared__ int X[1024];
@@ -1202,6 +1234,9 @@ __global__ void __launch_bounds__(VF_NT)
   __shared__ float aq[32], amass[32];
   __shared__ uint32_t cmS[32];
   __shared__ float SS[32];
+  __shared__ int tokS[32];
+  __shared__ uint32_t eqS[32];
+  __shared__ float qS[32];
   __shared__ float T[1024];  // min(p, q) of each distinct atom, at its first branch
   __shared__ int sL, sna;
   __shared__ uint32_t sties;
@@ -1209,17 +1244,27 @@ __global__ void __launch_bounds__(VF_NT)
   const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t p0 = pos[n];
   const uint32_t rd = rnd[n];
-  for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[(size_t)n * B * K + j];
-  if (tid < K) piS[tid] = exp2f(log2pi[n * K + tid]);
-  if (tid < B) cmS[tid] = cmask[(size_t)n * B + tid];
-  __syncthreads();
-  if (tid < B) {
-    float S = 0.f;
-    for (int k = 0; k < K; ++k)
-      if ((cmS[tid] >> k) & 1u) S += piS[k];
-    SS[tid] = S;
+  if constexpr (WITH_DRAFT) {
+    greedy_draft_body(gd.lsep, log2pi, gd.zhat, n, B, K, gd.M, V, gd.xhat_ws, gd.tok_ws,
+                      gd.qtok_ws, gd.cmask_ws, gd.out, X, tokS, eqS, cmS, piS, SS, qS);
+    __syncthreads();
+  } else {
+    for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[(size_t)n * B * K + j];
+    if (tid < K) piS[tid] = exp2f(log2pi[n * K + tid]);
+    if (tid < B) {
+      cmS[tid] = cmask[(size_t)n * B + tid];
+      tokS[tid] = tok[(size_t)n * B + tid];
+      qS[tid] = qtok_ws[(size_t)n * B + tid];
+    }
+    __syncthreads();
+    if (tid < B) {
+      float S = 0.f;
+      for (int k = 0; k < K; ++k)
+        if ((cmS[tid] >> k) & 1u) S += piS[k];
+      SS[tid] = S;
+    }
+    __syncthreads();
   }
-  __syncthreads();
   // one term min(p(a), q(a)) per distinct token a of the branches in C_i, a
   // thread per (i, z): the first branch of C_i with that token carries it
   for (int t = tid; t < B * K; t += VF_NT) {
@@ -1253,11 +1298,11 @@ __global__ void __launch_bounds__(VF_NT)
     float S = 0.f;
     if (lane < B) {
       const int m = n * B + lane;
-      const int x = min(max(tok[m], 0), V - 1);
+      const int x = min(max(tokS[lane], 0), V - 1);
       const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
       const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
       ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
-      qtok = qtok_ws[m];
+      qtok = qS[lane];
       const float ratio = ptok / qtok;
       A = fminf(1.f, ratio);
       c = cmS[lane];
@@ -1393,30 +1438,58 @@ __global__ void __launch_bounds__(VF_NT)
   if (out.emitted) {
     for (int j = tid; j < B + 1; j += VF_NT) {
       int val = -1;
-      if (j < L) val = tok[n * B + j];
+      if (j < L) val = tokS[j];
       else if (j == L && extra >= 0) val = extra;
       out.emitted[(size_t)n * (B + 1) + j] = val;
     }
   }
 }
 
-template <typename Tin>
-static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out* o) {
+template <typename Tin, bool WITH_DRAFT>
+static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out* o,
+                                       const dblast_draft_out* dout) {
   const WsLayout& w = c.wl;
-  cudaError_t le = launch_dep(k_greedy_verify<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
+  GreedyDraftArgs gd{};
+  if (WITH_DRAFT) {
+    gd.lsep = wsp<float4>(c, w.off_lsep);
+    gd.zhat = wsp<int32_t>(c, w.off_zhat);
+    gd.M = w.M;
+    gd.xhat_ws = wsp<int32_t>(c, w.off_xhat);
+    gd.tok_ws = wsp<int32_t>(c, w.off_tok);
+    gd.qtok_ws = wsp<float>(c, w.off_qtok);
+    gd.cmask_ws = wsp<uint32_t>(c, w.off_cmask);
+    if (dout) gd.out = *dout;
+  }
+  cudaError_t le = launch_dep(k_greedy_verify<Tin, WITH_DRAFT>, dim3(w.N), dim3(VF_NT), 0, c.stream,
       static_cast<const Tin*>(o->target), wsp<float>(c, w.off_log2pi),
       wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask), wsp<float>(c, w.off_qtok),
       wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
       wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.B, c.Bt, w.nt,
-      w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o);
+      w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o, gd);
   debug_kernel("k_greedy_verify", c.stream);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 cudaError_t launch_greedy_verify_finalize(const StepCtx& c, const dblast_verify_out* o) {
-  return c.head->dtype == DBLAST_F32 ? greedy_verify_typed<float>(c, o)
-                                     : greedy_verify_typed<__nv_bfloat16>(c, o);
+  return c.head->dtype == DBLAST_F32 ? greedy_verify_typed<float, false>(c, o, nullptr)
+                                     : greedy_verify_typed<__nv_bfloat16, false>(c, o, nullptr);
+}
+
+// Fused step, greedy mode without a filter: the argmax partials, then one
+// kernel per sequence that takes the greedy draft and verifies it.
+cudaError_t launch_greedy_step_finalize(const StepCtx& c, const dblast_draft_out* dout,
+                                        const dblast_verify_out* o) {
+  const WsLayout& w = c.wl;
+  const int K = c.head->K;
+  cudaError_t le =
+      launch_dep(k_greedy_argmax, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
+                 c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+  debug_kernel("k_greedy_argmax", c.stream);
+  count_launches(1);
+  if (le != cudaSuccess) return le;
+  return c.head->dtype == DBLAST_F32 ? greedy_verify_typed<float, true>(c, o, dout)
+                                     : greedy_verify_typed<__nv_bfloat16, true>(c, o, dout);
 }
 
 // ---------------------------------------------------------------- early determinism
