@@ -1089,7 +1089,7 @@ __device__ __forceinline__ void draft_target_stats(const Params& P, int w, int l
   }
 }
 
-template <bool PAIR, bool GREEDY = false>
+template <bool PAIR, bool GREEDY = false, bool TS = false>
 __global__ void __launch_bounds__(D_THREADS, 1)
     k_tc_pass(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
@@ -1173,8 +1173,9 @@ __global__ void __launch_bounds__(D_THREADS, 1)
     else if (warp == 1 && lane == 0 && (!PAIR || S.rank == 0))
       draft_mma<PAIR>(P, tmem, stages, full, empty, bfull, bempty, cfull, cempty, done, ctl,
                       my_tiles);
-    else if ((warp == 2 || warp == 3) && P.tgt != nullptr)
-      draft_target_stats(P, warp - 2, lane, xch);
+    else if constexpr (TS) {
+      if (warp == 2 || warp == 3) draft_target_stats(P, warp - 2, lane, xch);
+    }
   }
 
   tc_fence_before();
@@ -1628,17 +1629,17 @@ static int num_sms() {
 // The register split of k_tc_pass (setmaxnreg) assumes the kernel was built
 // with exactly DREG registers per thread: with fewer, the epilogue's increase
 // could never be granted.  Such a build is refused instead of launched.
-template <bool PAIR, bool GREEDY>
+template <bool PAIR, bool GREEDY, bool TS>
 static cudaError_t pass_kernel_ready() {
   static int state = -1;
   if (state < 0) {
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR, GREEDY>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR, GREEDY, TS>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != DREG) {
       state = 0;
     } else {
-      e = cudaFuncSetAttribute(k_tc_pass<PAIR, GREEDY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      e = cudaFuncSetAttribute(k_tc_pass<PAIR, GREEDY, TS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)DCfg<PAIR>::SMEM);
       if (e != cudaSuccess) return e;
       state = 1;
@@ -1664,7 +1665,7 @@ static cudaLaunchConfig_t cluster_config(int grid, int cs, size_t smem, cudaStre
 }
 
 // clusters of cs CTAs that can be resident at once (cached per form and size)
-template <bool PAIR, bool GREEDY>
+template <bool PAIR, bool GREEDY, bool TS>
 static int max_clusters(int cs) {
   static int cache[5] = {0, 0, 0, 0, 0};
   if (cs < 1 || cs > 4) return 0;
@@ -1672,31 +1673,31 @@ static int max_clusters(int cs) {
     cudaLaunchAttribute at[1];
     cudaLaunchConfig_t cfg = cluster_config(cs * num_sms(), cs, DCfg<PAIR>::SMEM, 0, at);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass<PAIR, GREEDY>, &cfg) != cudaSuccess || n < 1)
+    if (cudaOccupancyMaxActiveClusters(&n, k_tc_pass<PAIR, GREEDY, TS>, &cfg) != cudaSuccess || n < 1)
       n = 1;
     cache[cs] = n;
   }
   return cache[cs];
 }
 
-template <bool PAIR, bool GREEDY = false>
+template <bool PAIR, bool GREEDY = false, bool TS = false>
 static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& ca,
                           const CUtensorMap& cb, const Params& P, cudaStream_t s) {
-  cudaError_t e = pass_kernel_ready<PAIR, GREEDY>();
+  cudaError_t e = pass_kernel_ready<PAIR, GREEDY, TS>();
   if (e != cudaSuccess) return e;
   if (P.n_tiles <= 0) return cudaSuccess;
   if (!PAIR && P.cs == 1) {
     const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
-    e = launch_dep(k_tc_pass<false, GREEDY>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a,
+    e = launch_dep(k_tc_pass<false, GREEDY, TS>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a,
                    b, ca, cb, P);
   } else {
-    const int ncl = std::min(P.n_tiles, max_clusters<PAIR, GREEDY>(P.cs));
+    const int ncl = std::min(P.n_tiles, max_clusters<PAIR, GREEDY, TS>(P.cs));
     cudaLaunchAttribute at[2];
     cudaLaunchConfig_t cfg = cluster_config(ncl * P.cs, P.cs, DCfg<PAIR>::SMEM, s, at);
     at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.numAttrs = 2;
-    e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR, GREEDY>, a, b, ca, cb, P);
+    e = cudaLaunchKernelEx(&cfg, k_tc_pass<PAIR, GREEDY, TS>, a, b, ca, cb, P);
   }
   if (e != cudaSuccess) return e;
   debug_kernel("k_tc_pass", s);
@@ -1885,8 +1886,14 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
     P.t_lse = c.lse_target;
   }
   if (c.greedy)
-    return pair ? tc::launch<true, true>(ma, mb, mca, mcb, P, c.stream)
-                : tc::launch<false, true>(ma, mb, mca, mcb, P, c.stream);
+    return c.fuse_tstats
+               ? (pair ? tc::launch<true, true, true>(ma, mb, mca, mcb, P, c.stream)
+                       : tc::launch<false, true, true>(ma, mb, mca, mcb, P, c.stream))
+               : (pair ? tc::launch<true, true>(ma, mb, mca, mcb, P, c.stream)
+                       : tc::launch<false, true>(ma, mb, mca, mcb, P, c.stream));
+  if (c.fuse_tstats)
+    return pair ? tc::launch<true, false, true>(ma, mb, mca, mcb, P, c.stream)
+                : tc::launch<false, false, true>(ma, mb, mca, mcb, P, c.stream);
   return pair ? tc::launch<true>(ma, mb, mca, mcb, P, c.stream)
               : tc::launch<false>(ma, mb, mca, mcb, P, c.stream);
 }
