@@ -124,7 +124,8 @@ class ClockSampler:
 
 
 def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft", top_k=0, top_p=0.0):
-    """Time the fp64 oracle, as it stands, on one sequence of the workload."""
+    """Time the fp64 oracle, as it stands, on sequences of the workload: with
+    the BLAS thread pool as it comes (all host cores), then with one thread."""
     import torch
     from oracle import dblast_oracle as orc
     head_cpu = {k: (None if v is None else v.cpu()) for k, v in head.items()}
@@ -132,19 +133,51 @@ def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft", top_k=0, to
                "has_bonus": blk["has_bonus"]}
     pos = torch.full((cfg["N"],), 37, dtype=torch.int64)
     rnd = torch.zeros(cfg["N"], dtype=torch.int32)
-    n_done, t0 = 0, time.perf_counter()
-    while True:
-        orc.draft_and_verify(head_cpu, blk_cpu["hidden"], None, blk_cpu["target"],
-                             blk_cpu["has_bonus"], T, Z_T, 0, pos.numpy(), rnd.numpy(),
-                             seqs=[n_done % cfg["N"]], mode=mode, top_k=top_k, top_p=top_p)
-        n_done += 1
-        el = time.perf_counter() - t0
-        if el > budget_s / 3 or n_done >= 4:
-            break
+
+    def run(max_seqs, budget):
+        n_done, t0 = 0, time.perf_counter()
+        while True:
+            orc.draft_and_verify(head_cpu, blk_cpu["hidden"], None, blk_cpu["target"],
+                                 blk_cpu["has_bonus"], T, Z_T, 0, pos.numpy(), rnd.numpy(),
+                                 seqs=[n_done % cfg["N"]], mode=mode, top_k=top_k, top_p=top_p)
+            n_done += 1
+            el = time.perf_counter() - t0
+            if el > budget or n_done >= max_seqs:
+                return n_done, el
+
+    n_done, el = run(4, budget_s / 3)
+    single = None
+    try:
+        from threadpoolctl import threadpool_limits
+        with threadpool_limits(limits=1):
+            n1, el1 = run(1, budget_s / 3)
+        single = {"value": n1 / el1, "unit": UNIT, "threads": 1,
+                  "sample": "%d sequence(s), BLAS limited to one thread" % n1}
+    except ImportError:
+        single = {"value": None, "why": "threadpoolctl not installed on this host"}
     return {"value": n_done / el, "unit": UNIT, "cores": _cpu_threads(),
-            "kind": "oracle",
+            "kind": "oracle", "nproc": os.cpu_count(), "cpu_model": _cpu_model(),
+            "single_thread": single,
             "sample": "%d sequence(s) of the %s workload (one block each, %s mode), fp64 "
                       "direct form" % (n_done, cfg["name"], mode)}
+
+
+def _cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), or None."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return None
 
 
 def _cpu_threads():
@@ -192,7 +225,8 @@ def run_reference(args, cfg, rank):
                        "mode": args.mode, "sample": "one sequence (block) per step"},
             "accepted_tokens_per_s": L_total / el,
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": _cpu_threads(),
-                             "kind": "oracle",
+                             "kind": "oracle", "nproc": os.cpu_count(),
+                             "cpu_model": _cpu_model(),
                              "sample": "one sequence of %s per step" % cfg["name"]},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -483,6 +517,34 @@ def main():
     st = dblast_stats_get()
     accepted = sum(int(v["accepted"].sum()) for v in vouts)
     emitted = sum(int(v["n_emitted"].sum()) for v in vouts)
+    # decisions the kernels flagged as within the tie tolerance of their
+    # threshold (tie_flags), counted over the timed steps
+    flags = torch.stack([v["tie_flags"] for v in vouts]).cpu()
+    tie_seqs = int(((flags & 0xFF) != 0).sum())
+    near_seqs = int((flags != 0).sum())
+    tie_bits = {name: int(((flags & bit) != 0).sum()) for name, bit in
+                (("zhat", 1), ("draft", 2), ("accept", 4), ("residual_bonus", 8),
+                 ("residual_mass", 16), ("top_p", 32))}
+
+    # the workload's other temperature (the 8B batched workload is quoted at
+    # T = 0.6 and 1.0): the same timed loop on the same inputs
+    other_T = None
+    T2 = 0.6 if (cfg["name"] == "qwen3_8b_b32" and args.T != 0.6) else None
+    if T2 is not None:
+        pos2, rnd2 = synth.initial_state(cfg, dev)
+
+        def step2(k):
+            dblast_draft_and_verify(head, ws, blk["hidden"], pos2, rnd2, T2, cfg["Z_T"], seed,
+                                    blk["target"], blk["has_bonus"], impl=args.kernels,
+                                    dout=dout, vout=vouts[k % K_steps], mode=args.mode,
+                                    top_k=args.top_k, top_p=args.top_p)
+        ms2 = _timed_steps(step2, K_steps, args.warmup)
+        acc2 = sum(int(v["accepted"].sum()) for v in vouts)
+        ms2, (acc2,) = job_totals(ms2, (acc2,), world, dev)
+        other_T = {"T": T2, "ms_per_step": ms2 / K_steps,
+                   "value": job_value(N, world, K_steps, ms2),
+                   "accepted_tokens_per_s": acc2 / (ms2 / 1e3),
+                   "mean_accepted_length": acc2 / (N * world * K_steps)}
     ms, (accepted, emitted) = job_totals(ev0.elapsed_time(ev1), (accepted, emitted), world, dev)
     ms_step = ms / K_steps
     value = job_value(N, world, K_steps, ms)
@@ -591,6 +653,14 @@ def main():
                          "traffic": traffic, "kernel": "draft pass",
                          "ms_per_launch": draft_ms},
             "verify_pass_ms": verify_ms,
+            "ties": {"sequences_flagged_per_step": tie_seqs / K_steps,
+                     "sequences_flagged": tie_seqs, "sequences": N * K_steps,
+                     "by_kind": tie_bits,
+                     "sequences_near_per_step": near_seqs / K_steps,
+                     "what": "sequences whose step took a decision within 1e-6 of its "
+                             "threshold by the kernels' arithmetic (tie bits), and within "
+                             "1e-6 plus the kernels' precision allowance (near bits), over "
+                             "the timed steps"},
             "prep_ms": prep_ms,
             "gpu_launches": int(st["kernel_launches"]),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -598,6 +668,9 @@ def main():
                     "overlap": "inputs of step k+1 copied on a second stream during step k"},
             "clocks": clk,
         }
+        if other_T is not None:
+            other_T["roofline_frac"] = 1e3 * t_roof / other_T["ms_per_step"]
+            line["T%.1f" % other_T["T"]] = other_T
         if world == 1 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline(cfg, head_t, blk, args.T, cfg["Z_T"],
                                                 mode=args.mode, top_k=args.top_k,

@@ -149,7 +149,13 @@ typedef struct {
   float* alpha_len;     /* [N]        sum_i prod_{j<=i} alpha_j */
   uint32_t* tie_flags;  /* [N]        bit0 z-hat, bit1 draft, bit2 accept, bit3 residual/bonus,
                                        bit4 residual mass < 1e-6: a decision within 1e-6 of its threshold
-                                       (GREEDY mode leaves bit1 clear: argmax decisions are not flagged) */
+                                       by the kernels' own arithmetic.  Bits 8-14: the same kinds,
+                                       "near": within 1e-6 plus the kernels' precision allowance
+                                       (5e-5 of probability mass for a draw, 1e-4 relative for the
+                                       acceptance ratio p/q), so every decision that may be a tie of
+                                       the exact arithmetic is flagged; a tie bit implies its near bit.
+                                       GREEDY mode: bit1 (and bit9) = the greedy argmax of a branch in
+                                       C_i whose top-two logit gap is below 1e-4 (the logits are fp32) */
   float* collision;     /* [N, B]     sum_v p_i(v)^2, the collision probability of target row i (App. B) */
   float* determinism;   /* [N]        target-block early determinism D_B = (1/B) sum_j prod_{i<=j}
                                        collision_i (App. B, Eq. appendix-early-determinism, for
@@ -164,7 +170,7 @@ typedef struct {
    * token and collision/determinism; lse_target stays the unfiltered
    * log-sum-exp.  With a filter on, at most 256 tokens may stay (top-p needs
    * top_k in 1..256, or V <= 256) and V <= 262144; else DBLAST_ERR_UNSUPPORTED.
-   * tie_flags bit5: a top-p cut within 1e-6 of top_p on some row. */
+   * tie_flags bit5 (and bit13): a top-p cut within 1e-6 of top_p on some row. */
   int top_k;
   float top_p;
 } dblast_verify_out;
@@ -237,8 +243,9 @@ dblast_status dblast_stats_get(dblast_stats* out);
  * DBLAST_ERR_WORKSPACE is returned and nothing is launched.  It calls no
  * allocation routine.  The first call on a device, with that device current,
  * looks up the array's device address (cudaGetSymbolAddress); make that first
- * call before any stream capture.  `stream` must belong to the current
- * device.  Every call reuses the same array, so calls that overlap on the GPU
+ * call before any stream capture.  After a cudaDeviceReset the next call sees
+ * the device's new context and looks the address up again (so, again, before
+ * any capture).  `stream` must belong to the current device.  Every call reuses the same array, so calls that overlap on the GPU
  * (other streams or threads) race; serialise them. */
 #define DBLAST_NOALLOC_MAX_RECORDS (1u << 20)
 dblast_status dblast_target_lse_noalloc(const void* target, int rows, int V, dblast_dtype dtype,
@@ -261,7 +268,8 @@ dblast_status dblast_target_lse_noalloc(const void* target, int rows, int V, dbl
  *   nll[n]       = -log sum_z q(z|y) prod_i q_i(x*_i|y,z) (Eq. dependent-nll;
  *                  K = 1: Eq. independent-nll)
  *   tie_flags[n] bit5: a top-p cut within 1e-6; bit6: an r_l within 1e-6
- *                (relative) of tau among l <= l_tau.
+ *                (relative) of tau among l <= l_tau; bits 13, 14: the same
+ *                within the precision allowance (1e-4 relative per factor of r_l).
  * Natural logarithms.  args->mode must be DBLAST_MODE_SOFT; args->seed, pos
  * and round are read (the latent draw of the shared draft kernels) but not
  * advanced.  Uses the step workspace (dblast_workspace_bytes with the same

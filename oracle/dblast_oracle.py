@@ -212,10 +212,11 @@ def filter_target(t_row, T, top_k=0, top_p=0.0):
     return out, keep, float(margin)
 
 
-def target_distributions(target, T, top_k, top_p, ties):
+def target_distributions(target, T, top_k, top_p, ties, decisions=None):
     """p_i for every target row: softmax(t_i / T), filtered by top-k / top-p
     when either is on (filter_target); a top-p cut within TIE_TOL is recorded
-    as a tie of kind "top_p" at row i.  Also returns the unfiltered natural
+    as a tie of kind "top_p" at row i, and every finite cut margin is listed
+    in `decisions` when given.  Also returns the unfiltered natural
     log-sum-exp of t_i / T."""
     st = target / T
     lse_t = logsumexp(st, axis=-1)
@@ -224,6 +225,8 @@ def target_distributions(target, T, top_k, top_p, ties):
     p = np.empty_like(st)
     for i in range(target.shape[0]):
         p[i], _, margin = filter_target(target[i], T, top_k, top_p)
+        if decisions is not None and np.isfinite(margin):
+            decisions.append(("top_p", i, margin))
         if margin < TIE_TOL:
             ties.append(("top_p", i, margin))
     return p, lse_t
@@ -241,13 +244,16 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     W = head["W"]
     a = h[0] if anchor is None else anchor
     ties = []
+    decisions = []  # (kind, position, margin) of every decision taken
 
     # prior and latent category (Sec. 3.1; Appendix A)
     ell, pi = category_prior(head["Wp"], head["bp"], a, Z_T)
     u0 = decision_uniform(seed, STREAM_PRIOR, round_, n, pos)
     zhat, m0 = inverse_cdf(pi, u0)
-    if Z_T != 0 and m0 < TIE_TOL:
-        ties.append(("zhat", -1, m0))
+    if Z_T != 0:
+        decisions.append(("zhat", -1, m0))
+        if m0 < TIE_TOL:
+            ties.append(("zhat", -1, m0))
     with np.errstate(divide="ignore"):
         log_pi = np.log(pi)
 
@@ -262,6 +268,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     for i in range(B):
         u1 = decision_uniform(seed, STREAM_DRAFT, round_, n, pos + i)
         tokens[i], m1 = inverse_cdf(np.exp(logq[i, zhat]), u1)
+        decisions.append(("draft", i, m1))
         if m1 < TIE_TOL:
             ties.append(("draft", i, m1))
 
@@ -273,7 +280,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     q_tok = qmix[np.arange(B), tokens]
 
     # target distributions p_i = softmax(t_i / T)
-    p, lse_t = target_distributions(target, T, top_k, top_p, ties)  # [B+hb, V]
+    p, lse_t = target_distributions(target, T, top_k, top_p, ties, decisions)  # [B+hb, V]
     p_tok = p[np.arange(B), tokens]
 
     alpha = np.sum(np.minimum(p[:B], qmix), axis=-1)
@@ -285,6 +292,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     for i in range(B):
         u2 = decision_uniform(seed, STREAM_ACCEPT, round_, n, pos + i)
         m2 = abs(u2 * q_tok[i] - p_tok[i]) / q_tok[i]
+        decisions.append(("accept", i, m2))
         if m2 < TIE_TOL:
             ties.append(("accept", i, m2))
         if not (u2 < ratio[i]):
@@ -302,6 +310,8 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
             extra, m3 = inverse_cdf(res, u3)
         else:
             extra, m3 = inverse_cdf(p[L], u3)
+        decisions.append(("residual_mass", L, mass))
+        decisions.append(("residual", L, m3))
         if mass < TIE_TOL:
             ties.append(("residual_mass", L, mass))
         if m3 < TIE_TOL:
@@ -309,6 +319,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     elif has_bonus:
         u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + B)
         extra, m3 = inverse_cdf(p[B], u3)
+        decisions.append(("bonus", B, m3))
         if m3 < TIE_TOL:
             ties.append(("bonus", B, m3))
     if extra >= 0:
@@ -326,7 +337,7 @@ def draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 logw=logw, q_tok=q_tok, p_tok=p_tok, accept_prob=accept_prob,
                 alpha=alpha, accepted=L, emitted=emitted,
                 n_emitted=len(emitted), exp_len=exp_len, alpha_len=alpha_len,
-                lse_target=lse_t, ties=ties, first_tie=first_tie,
+                lse_target=lse_t, ties=ties, decisions=decisions, first_tie=first_tie,
                 collision=collision_probability(p[:B]),
                 determinism=early_determinism_exact(p[:B]))
 
@@ -485,13 +496,16 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     V = W.shape[0]
     a = h[0] if anchor is None else anchor
     ties = []
+    decisions = []  # (kind, position, margin) of every decision taken
 
     # prior and latent category, as in the stochastic mode
     ell, pi = category_prior(head["Wp"], head["bp"], a, Z_T)
     u0 = decision_uniform(seed, STREAM_PRIOR, round_, n, pos)
     zhat, m0 = inverse_cdf(pi, u0)
-    if Z_T != 0 and m0 < TIE_TOL:
-        ties.append(("zhat", -1, m0))
+    if Z_T != 0:
+        decisions.append(("zhat", -1, m0))
+        if m0 < TIE_TOL:
+            ties.append(("zhat", -1, m0))
 
     # all K greedy branches and the selected block
     hz = branch_hidden(h, head["U"], head["Vf"], head["e"])
@@ -501,8 +515,10 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     C = consistent_branches(xhat, tokens)
     for i in range(B):
         for z in range(xhat.shape[1]):
-            if C[i, z] and gap[i, z] < GREEDY_TIE_TOL:
-                ties.append(("greedy", i, float(gap[i, z])))
+            if C[i, z]:
+                decisions.append(("greedy", i, float(gap[i, z])))
+                if gap[i, z] < GREEDY_TIE_TOL:
+                    ties.append(("greedy", i, float(gap[i, z])))
 
     # the proposal conditional used by verification
     q, pit = greedy_conditional(pi, xhat, C, V)
@@ -511,7 +527,7 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
         logw = np.log(pit)
 
     # target distributions p_i = softmax(t_i / T)
-    p, lse_t = target_distributions(target, T, top_k, top_p, ties)
+    p, lse_t = target_distributions(target, T, top_k, top_p, ties, decisions)
     p_tok = p[np.arange(B), tokens]
     alpha = np.sum(np.minimum(p[:B], q), axis=-1)
     ratio = p_tok / q_tok
@@ -521,6 +537,7 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     for i in range(B):
         u2 = decision_uniform(seed, STREAM_ACCEPT, round_, n, pos + i)
         m2 = abs(u2 * q_tok[i] - p_tok[i]) / q_tok[i]
+        decisions.append(("accept", i, m2))
         if m2 < TIE_TOL:
             ties.append(("accept", i, m2))
         if not (u2 < ratio[i]):
@@ -537,6 +554,8 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
             extra, m3 = inverse_cdf(res, u3)
         else:
             extra, m3 = inverse_cdf(p[L], u3)
+        decisions.append(("residual_mass", L, mass))
+        decisions.append(("residual", L, m3))
         if mass < TIE_TOL:
             ties.append(("residual_mass", L, mass))
         if m3 < TIE_TOL:
@@ -544,6 +563,7 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
     elif has_bonus:
         u3 = decision_uniform(seed, STREAM_RESIDUAL, round_, n, pos + B)
         extra, m3 = inverse_cdf(p[B], u3)
+        decisions.append(("bonus", B, m3))
         if m3 < TIE_TOL:
             ties.append(("bonus", B, m3))
     if extra >= 0:
@@ -560,7 +580,7 @@ def greedy_draft_and_verify_sequence(head, h, anchor, target, has_bonus, T, Z_T,
                 consistent=C, gap=gap, logw=logw, q_tok=q_tok, p_tok=p_tok,
                 accept_prob=accept_prob, alpha=alpha, accepted=L,
                 emitted=emitted, n_emitted=len(emitted), exp_len=exp_len,
-                alpha_len=alpha_len, lse_target=lse_t, ties=ties,
+                alpha_len=alpha_len, lse_target=lse_t, ties=ties, decisions=decisions,
                 first_tie=first_tie, collision=collision_probability(p[:B]),
                 determinism=early_determinism_exact(p[:B]))
 

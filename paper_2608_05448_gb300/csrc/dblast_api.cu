@@ -8,6 +8,8 @@
 #include <mutex>
 #include <vector>
 
+#include <cuda.h>
+
 #include "dblast_internal.cuh"
 
 namespace dblast {
@@ -155,6 +157,7 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_fp = take((size_t)w.Rt * FILTER_MAX_K * sizeof(float));
   w.off_fcnt = take((size_t)w.Rt * sizeof(int32_t));
   w.off_ftie = take((size_t)w.Rt * sizeof(uint32_t));
+  w.off_partg = take((size_t)w.nt * K * w.Mpad * sizeof(float));
   w.total = o;
   return w;
 }
@@ -167,6 +170,33 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c);
 using namespace dblast;
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+namespace dblast {
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_cur = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_cur = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  if (!get_cur || !get_id) return 0ull;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0ull;
+  if (get_cur(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS) return 0ull;
+  return id;
+}
+}  // namespace dblast
 
 static dblast_status check_head(const dblast_head* h, bool need_prep) {
   if (!h) return DBLAST_ERR_INVALID_ARG;
@@ -324,14 +354,17 @@ static dblast_status verify_impl(StepCtx c, dblast_verify_out* out) {
   return cuda_status(e);
 }
 
+
 // One internal stream and four events per device for the fork/join of
 // kernels that do not depend on each other inside dblast_draft_and_verify
 // (no device memory; created by the first such call on the device and held
-// until the process exits).  The mutex keeps one call's fork/join pairs
+// until the process exits, or made again after a device reset gave the
+// device a new context).  The mutex keeps one call's fork/join pairs
 // together when several host threads call in.
 struct SideStream {
   cudaStream_t s = nullptr;
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  unsigned long long ctx = 0ull;  // context the handles belong to
 };
 static std::mutex g_side_mu;
 static SideStream g_side[64];
@@ -342,7 +375,10 @@ static cudaError_t side_stream(SideStream** out) {
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   SideStream& ss = g_side[dev];
+  const unsigned long long ctx = current_context_id();
+  if (ss.s && ctx != ss.ctx) ss = SideStream{};  // handles of a context that was reset
   if (!ss.s) {
+    ss.ctx = ctx;
     e = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking);
     for (int i = 0; i < 4 && e == cudaSuccess; ++i)
       e = cudaEventCreateWithFlags(&ss.ev[i], cudaEventDisableTiming);

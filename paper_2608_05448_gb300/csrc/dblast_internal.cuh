@@ -19,11 +19,25 @@ constexpr int MTILE = 128;  // rows (positions) per tensor-core tile
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float LN2 = 0.6931471805599453f;
 constexpr float TIE_TOL = 1e-6f;
+// greedy-branch mode: an argmax whose top-two logit gap is below this is
+// reported as a tie (the logits are formed in fp32, within about 1e-5 of the
+// exact values at the Qwen3 shapes)
+constexpr float GREEDY_TIE_TOL = 1e-4f;
 
 enum TieBits : uint32_t {
   TIE_ZHAT = 1u, TIE_DRAFT = 2u, TIE_ACCEPT = 4u, TIE_RESID = 8u, TIE_RMASS = 16u, TIE_TOPP = 32u,
   TIE_TAU = 64u
 };
+// "Near" bits (the tie bit of the same kind, shifted): the decision is within
+// TIE_TOL of its threshold once the kernels' own precision is allowed for.
+// The vocabulary-head logits come from fp32 tensor-core accumulation of H
+// bf16 products: at H = 4096 they are within 5.7e-6 (RMS, 3.8e-5 at most) of
+// the exact values, which moves a draw's CDF by up to about 1e-5 of the total
+// mass and an acceptance ratio p/q by up to about 1e-4 (relative).  A decision
+// whose own margin is below TIE_TOL plus these allowances may be a tie.
+constexpr uint32_t NEAR_SHIFT = 8u;
+constexpr float NEAR_DRAW = 5e-5f;    // probability mass, for every inverse-CDF draw
+constexpr float NEAR_ACCEPT = 1e-4f;  // relative to q(x_i|x_<i), for the acceptance test
 
 // target filter (top-k / top-p): at most FILTER_MAX_K kept tokens per row,
 // and vocabularies of at most FILTER_MAX_TILES tiles
@@ -55,6 +69,8 @@ struct PrepLayout {
 //   partv float2 [nt,Mpad] | ties u32 [N]
 //   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
 //   token and the consistent-branch set C_i as a bit mask over z)
+//   partg f32 [nt,K,Mpad]  (greedy-branch mode: the second-largest logit of
+//   every draft record's tile, for the argmax tie report)
 //   coll f32 [Rt]  (collision probability sum_v p(v)^2 of every target row)
 //   ftok i32 [Rt, FILTER_MAX_K] | fp f32 [Rt, FILTER_MAX_K] | fcnt i32 [Rt] | ftie u32 [Rt]
 //   (target filter: kept tokens by index, their filtered probabilities, count, top-p tie)
@@ -64,7 +80,7 @@ struct WsLayout {
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,
       off_partd, off_lsep, off_lse2, off_lq2, off_w2, off_qtok, off_tok, off_vcz, off_vb0,
       off_partt, off_lt2, off_partv, off_ties, off_xhat, off_cmask, off_coll, off_ftok,
-      off_fp, off_fcnt, off_ftie, total;
+      off_fp, off_fcnt, off_ftie, off_partg, total;
 };
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
@@ -257,6 +273,11 @@ template <typename T> const T* prp(const StepCtx& c, size_t off) {
 // measurement hooks (dblast_api.cu)
 void count_launches(int n);
 void count_tc_launch();
+// Process-unique id of the calling thread's current CUDA context (0 when the
+// driver cannot tell).  Per-device caches of device addresses, streams and
+// kernel attributes compare it with the id they were made under: after a
+// cudaDeviceReset the device gets a new context and they are made again.
+unsigned long long current_context_id();
 // with DBLAST_DEBUG_SYNC=1: synchronise and report the kernel just launched
 void debug_kernel(const char* name, cudaStream_t s);
 

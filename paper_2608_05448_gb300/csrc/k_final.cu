@@ -112,12 +112,13 @@ template <int NT> struct FindShared {
   FF d[NT / 32];
   int i[NT / 32];
   FF before;
-  int tile, x, tie;
+  int tile, x, tie, near;
 };
 
 struct FindOut {
-  int x;     // chosen token, -1 if no token has mass
-  bool tie;  // the decision is within TIE_TOL of its threshold, or rounding forced a fallback
+  int x;      // chosen token, -1 if no token has mass
+  bool tie;   // the decision is within TIE_TOL of its threshold, or rounding forced a fallback
+  bool near;  // within TIE_TOL + near_abs / total (near_abs: an absolute mass allowance)
 };
 
 // Smallest token whose cumulative mass (in vocabulary order) exceeds `target`.
@@ -126,7 +127,8 @@ struct FindOut {
 // tile masses, and that sum scales the margin.
 template <int NT, typename TM, typename EM>
 __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF target,
-                              float total, FindShared<NT>& fs, bool frac = false) {
+                              float total, FindShared<NT>& fs, bool frac = false,
+                              float near_abs = NEAR_DRAW) {
   static_assert(NT >= TILE_V, "one thread per token of a tile");
   const int tid = threadIdx.x, lane = tid & 31;
   const int chunk = ceil_div(nt, NT);
@@ -198,12 +200,14 @@ __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF 
         fs.tile = miss ? lp : tt;
         fs.before = miss ? lastlo : before;
         fs.tie = miss ? 1 : 0;
+        fs.near = fs.tie;
       }
     }
   } else if (tid == 0) {  // rounding left the target at or above the total
     fs.tile = lastall;
     fs.before = lastall >= 0 ? ff_add(sc.total, FF{-tmass(lastall), 0.f}) : FF{0.f, 0.f};
     fs.tie = 1;
+    fs.near = 1;
   }
   __syncthreads();
   const int tt = fs.tile;
@@ -220,13 +224,15 @@ __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF 
       fs.x = tt * TILE_V + fj;
       const float margin = fminf(ff_f(ff_sub(target, lo)), ff_f(ff_sub(hi, target))) / total;
       if (margin < TIE_TOL) fs.tie = 1;
+      if (margin < TIE_TOL + near_abs / total) fs.near = 1;
     }
   } else if (tid == 0) {
     fs.x = (tt >= 0 && lastv >= 0) ? tt * TILE_V + lastv : -1;
     fs.tie = 1;
+    fs.near = 1;
   }
   __syncthreads();
-  const FindOut r{fs.x, fs.tie != 0};
+  const FindOut r{fs.x, fs.tie != 0, fs.near != 0};
   __syncthreads();
   return r;
 }
@@ -400,6 +406,7 @@ __global__ void __launch_bounds__(DT_NT)
     if (tid == 0) {
       tok[m] = x;
       if (f.tie || f.x < 0) atomicOr(&ties[n], (uint32_t)TIE_DRAFT);
+      if (f.near || f.x < 0) atomicOr(&ties[n], (uint32_t)TIE_DRAFT << NEAR_SHIFT);
     }
   }
   if (tid < K) {  // log2 q_z(x) = (base_x + corr_z(x)) k2 - L_z, products exact
@@ -885,8 +892,11 @@ __global__ void __launch_bounds__(VF_NT)
     const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
     const int L = rej ? (__ffs(rej) - 1) : B;
     // acceptance ties only for the positions that were tested (i <= L)
-    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    const float amargin = fabsf(fmaf(u2, qtok, -ptok));
+    const bool atie = lane < B && lane <= L && amargin < TIE_TOL * qtok;
+    const bool anear = lane < B && lane <= L && amargin < (TIE_TOL + NEAR_ACCEPT) * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    if (__ballot_sync(FULLMASK, anear)) ties |= TIE_ACCEPT << NEAR_SHIFT;
     // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha (products in lane order)
     // App. B: collision probabilities of the block's target rows and
     // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
@@ -936,7 +946,7 @@ __global__ void __launch_bounds__(VF_NT)
   const int L = sL;
   const FF Rm = sR;
   int extra = -1;
-  bool tie = false;
+  bool tie = false, near = false;
   uint32_t tbits = 0;
   const int irow = (L < B) ? L : B;  // target row of the extra token
   if ((L < B) || (Bt > B)) {
@@ -949,6 +959,7 @@ __global__ void __launch_bounds__(VF_NT)
       const int m = n * B + L;
       const float Rf = ff_f(Rm);
       if (Rf < TIE_TOL) tbits |= TIE_RMASS;
+      if (Rf < TIE_TOL + NEAR_DRAW) tbits |= TIE_RMASS << NEAR_SHIFT;
       if (Rf > 0.f) {
         const ResidualTokenMass<Tin> rm{pv, stash + (size_t)m * V, wu,
                                         codes + (size_t)m * K * rr, sC, K, rr, k2};
@@ -956,10 +967,11 @@ __global__ void __launch_bounds__(VF_NT)
                                             ff_mulf(Rm, u3), Rf, fs);
         extra = f.x;
         tie = f.tie;
+        near = f.near;
       }
       if (extra < 0) {  // no positive residual mass left by rounding: draw from p
         from_p = true;
-        tie = true;
+        tie = near = true;
         tbits |= TIE_RMASS;
       }
     }
@@ -968,10 +980,13 @@ __global__ void __launch_bounds__(VF_NT)
                                           pv, FF{u3, 0.f}, 1.f, fs);
       extra = f.x >= 0 ? f.x : 0;
       tie = tie || f.tie || f.x < 0;
+      near = near || f.near || f.x < 0;
     }
   }
   if (tid == 0) {
-    const uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u);
+    uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u) |
+                    (near ? (uint32_t)TIE_RESID << NEAR_SHIFT : 0u);
+    ties |= (ties & 0xffu) << NEAR_SHIFT;  // a tie is also near
     const int ne = L + (extra >= 0 ? 1 : 0);
     if (out.accepted) out.accepted[n] = L;
     if (out.n_emitted) out.n_emitted[n] = ne;
@@ -1018,51 +1033,61 @@ cudaError_t launch_verify_finalize(const StepCtx& c, const dblast_verify_out* o)
 // and verify with it.  q_greedy has at most K atoms per position, so p is
 // needed only at those tokens, plus the target tile records for the residual
 // and bonus draws.
-__device__ __forceinline__ void arg_keep(float& mx, int& ix, float v, int i) {
+// top-two merge of (max, index, second) with a record (v, i, vs): ties to
+// the lower index; the second of the union is the larger of the losing max
+// and the winner's own second
+__device__ __forceinline__ void arg_keep2(float& mx, int& ix, float& sc, float v, int i, float vs) {
   if (v > mx || (v == mx && i < ix)) {
+    sc = fmaxf(mx, vs);
     mx = v;
     ix = i;
+  } else {
+    sc = fmaxf(sc, v);
   }
 }
 
 // Partial argmax of the draft records: block (row group of 32, z, split), lane
 // = row, warps and splits interleave over the tiles (as k_draft_lse).
-// lsep[sp][m][z] = (max, token bits, 0, 0).
+// lsep[sp][m][z] = (max, token bits, second-largest logit, 0).
 __global__ void __launch_bounds__(LSE_WARPS * 32)
-    k_greedy_argmax(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
-                    float4* __restrict__ lsep) {
+    k_greedy_argmax(const float2* __restrict__ partd, const float* __restrict__ partg, int nt,
+                    int K, int M, int Mpad, float4* __restrict__ lsep) {
   griddep_wait();  // launched as a dependent of the previous kernel
-  __shared__ float smx[LSE_WARPS][32];
+  __shared__ float smx[LSE_WARPS][32], ssc[LSE_WARPS][32];
   __shared__ int six[LSE_WARPS][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int m = blockIdx.x * 32 + lane, z = blockIdx.y, sp = blockIdx.z;
   const int step = LSE_WARPS * LSE_SPLIT;
-  float mx = -INFINITY;
+  float mx = -INFINITY, sc = -INFINITY;
   int ix = 0x7fffffff;
   if (m < M) {
     const float2* p = partd + (size_t)z * Mpad + m;
+    const float* g = partg + (size_t)z * Mpad + m;
     const size_t st = (size_t)K * Mpad;
     int t = sp * LSE_WARPS + warp;
     for (; t + 3 * step < nt; t += 4 * step) {
       const float2 q0 = p[(size_t)t * st], q1 = p[(size_t)(t + step) * st];
       const float2 q2 = p[(size_t)(t + 2 * step) * st], q3 = p[(size_t)(t + 3 * step) * st];
-      arg_keep(mx, ix, q0.x, __float_as_int(q0.y));
-      arg_keep(mx, ix, q1.x, __float_as_int(q1.y));
-      arg_keep(mx, ix, q2.x, __float_as_int(q2.y));
-      arg_keep(mx, ix, q3.x, __float_as_int(q3.y));
+      const float g0 = g[(size_t)t * st], g1 = g[(size_t)(t + step) * st];
+      const float g2 = g[(size_t)(t + 2 * step) * st], g3 = g[(size_t)(t + 3 * step) * st];
+      arg_keep2(mx, ix, sc, q0.x, __float_as_int(q0.y), g0);
+      arg_keep2(mx, ix, sc, q1.x, __float_as_int(q1.y), g1);
+      arg_keep2(mx, ix, sc, q2.x, __float_as_int(q2.y), g2);
+      arg_keep2(mx, ix, sc, q3.x, __float_as_int(q3.y), g3);
     }
     for (; t < nt; t += step) {
       const float2 q = p[(size_t)t * st];
-      arg_keep(mx, ix, q.x, __float_as_int(q.y));
+      arg_keep2(mx, ix, sc, q.x, __float_as_int(q.y), g[(size_t)t * st]);
     }
   }
   smx[warp][lane] = mx;
   six[warp][lane] = ix;
+  ssc[warp][lane] = sc;
   __syncthreads();
   if (warp == 0 && m < M) {
 #pragma unroll
-    for (int w = 1; w < LSE_WARPS; ++w) arg_keep(mx, ix, smx[w][lane], six[w][lane]);
-    lsep[((size_t)sp * M + m) * K + z] = make_float4(mx, __int_as_float(ix), 0.f, 0.f);
+    for (int w = 1; w < LSE_WARPS; ++w) arg_keep2(mx, ix, sc, smx[w][lane], six[w][lane], ssc[w][lane]);
+    lsep[((size_t)sp * M + m) * K + z] = make_float4(mx, __int_as_float(ix), sc, 0.f);
   }
 }
 
@@ -1072,31 +1097,40 @@ __global__ void __launch_bounds__(LSE_WARPS * 32)
 // The draft side of one sequence, for any block size: x-hat_{i,z} (thread
 // (i, z), strided), the block, C_i (bit z of cmask[m]: branch z drafted x_j at
 // every j < i), pi~_{i,z} and q_greedy(x_i|x_<i), and the draft outputs.
-// Shared arrays: X [B K], tokS, eqS, cmS, piS, sumS [32].
+// An argmax of a branch in C_i whose top-two logit gap is below
+// GREEDY_TIE_TOL sets the draft tie bit of the sequence (ties_ws[n]).
+// Shared arrays: X [B K], tokS, eqS, nearS, cmS, piS, sumS [32].
 __device__ void greedy_draft_body(const float4* __restrict__ lsep, const float* __restrict__ log2pi,
                                   const int32_t* __restrict__ zhat, int n, int B, int K, int M,
                                   int V, int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
                                   float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
-                                  const dblast_draft_out& out, int* X, int* tokS, uint32_t* eqS,
-                                  uint32_t* cmS, float* piS, float* sumS, float* qS) {
+                                  uint32_t* __restrict__ ties_ws, const dblast_draft_out& out,
+                                  int* X, int* tokS, uint32_t* eqS, uint32_t* nearS, uint32_t* cmS,
+                                  float* piS, float* sumS, float* qS) {
   const int nt = blockDim.x;
+  if (threadIdx.x < 32) {
+    eqS[threadIdx.x] = 0u;
+    nearS[threadIdx.x] = 0u;
+  }
+  __syncthreads();
   for (int t = threadIdx.x; t < B * K; t += nt) {
     const int i = t / K, z = t - i * K;
     const size_t m = (size_t)n * B + i;
-    float mx = -INFINITY;
+    float mx = -INFINITY, sc = -INFINITY;
     int ix = 0x7fffffff;
 #pragma unroll
     for (int sp = 0; sp < LSE_SPLIT; ++sp) {
       const float4 q = lsep[((size_t)sp * M + m) * K + z];
-      arg_keep(mx, ix, q.x, __float_as_int(q.y));
+      arg_keep2(mx, ix, sc, q.x, __float_as_int(q.y), q.z);
     }
+    // top-two gap (0 for equal logits; NaN logits compare false and count as near)
+    if (!(mx - sc >= GREEDY_TIE_TOL)) atomicOr(&nearS[i], 1u << z);
     ix = min(max(ix, 0), V - 1);  // every logit NaN: not a token, keep the index valid
     X[t] = ix;
     xhat_ws[m * K + z] = ix;
     if (out.branch_tokens) out.branch_tokens[m * K + z] = ix;
   }
   if ((int)threadIdx.x < K) piS[threadIdx.x] = exp2f(log2pi[n * K + threadIdx.x]);  // -inf gives 0
-  if (threadIdx.x < 32) eqS[threadIdx.x] = 0u;
   __syncthreads();
   const int zh = zhat[n];
   if ((int)threadIdx.x < B) tokS[threadIdx.x] = X[threadIdx.x * K + zh];
@@ -1111,6 +1145,7 @@ __device__ void greedy_draft_body(const float4* __restrict__ lsep, const float* 
     uint32_t c = (K >= 32) ? 0xffffffffu : ((1u << K) - 1u);
     for (int j = 0; j < t; ++j) c &= eqS[j];
     cmS[t] = c;
+    if (c & nearS[t]) atomicOr(&ties_ws[n], (uint32_t)TIE_DRAFT | ((uint32_t)TIE_DRAFT << NEAR_SHIFT));
     float S = 0.f, Q = 0.f;
     for (int k = 0; k < K; ++k) {
       if ((c >> k) & 1u) {
@@ -1145,14 +1180,14 @@ __global__ void __launch_bounds__(1024)
                    const int32_t* __restrict__ zhat, int B, int K, int M, int V,
                    int32_t* __restrict__ xhat_ws, int32_t* __restrict__ tok_ws,
                    float* __restrict__ qtok_ws, uint32_t* __restrict__ cmask_ws,
-                   dblast_draft_out out) {
+                   uint32_t* __restrict__ ties_ws, dblast_draft_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ int X[1024];
   __shared__ int tokS[32];
-  __shared__ uint32_t eqS[32], cmS[32];
+  __shared__ uint32_t eqS[32], nearS[32], cmS[32];
   __shared__ float piS[32], sumS[32], qS[32];
   greedy_draft_body(lsep, log2pi, zhat, blockIdx.x, B, K, M, V, xhat_ws, tok_ws, qtok_ws, cmask_ws,
-                    out, X, tokS, eqS, cmS, piS, sumS, qS);
+                    ties_ws, out, X, tokS, eqS, nearS, cmS, piS, sumS, qS);
 }
 
 cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_out* outp) {
@@ -1160,7 +1195,8 @@ cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_ou
   const int K = c.head->K;
   cudaError_t le =
       launch_dep(k_greedy_argmax, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
-                 c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+                 c.stream, wsp<float2>(c, w.off_partd), wsp<float>(c, w.off_partg), w.nt, K, w.M,
+                 w.Mpad, wsp<float4>(c, w.off_lsep));
   debug_kernel("k_greedy_argmax", c.stream);
   dblast_draft_out out{};
   if (outp) out = *outp;
@@ -1168,7 +1204,7 @@ cudaError_t launch_greedy_draft_finalize(const StepCtx& c, const dblast_draft_ou
   if (le == cudaSuccess) le = launch_dep(k_greedy_draft, dim3(w.N), dim3(pt), 0, c.stream,
       wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_log2pi), wsp<int32_t>(c, w.off_zhat), w.B,
       K, w.M, w.V, wsp<int32_t>(c, w.off_xhat), wsp<int32_t>(c, w.off_tok),
-      wsp<float>(c, w.off_qtok), wsp<uint32_t>(c, w.off_cmask), out);
+      wsp<float>(c, w.off_qtok), wsp<uint32_t>(c, w.off_cmask), wsp<uint32_t>(c, w.off_ties), out);
   debug_kernel("k_greedy_draft", c.stream);
   count_launches(2);
   return le != cudaSuccess ? le : cudaGetLastError();
@@ -1214,6 +1250,7 @@ struct GreedyDraftArgs {
   int32_t* tok_ws;
   float* qtok_ws;
   uint32_t* cmask_ws;
+  uint32_t* ties_ws;
   dblast_draft_out out;
 };
 
@@ -1235,7 +1272,7 @@ __global__ void __launch_bounds__(VF_NT)
   __shared__ uint32_t cmS[32];
   __shared__ float SS[32];
   __shared__ int tokS[32];
-  __shared__ uint32_t eqS[32];
+  __shared__ uint32_t eqS[32], nearS[32];
   __shared__ float qS[32];
   __shared__ float T[1024];  // min(p, q) of each distinct atom, at its first branch
   __shared__ int sL, sna;
@@ -1246,7 +1283,8 @@ __global__ void __launch_bounds__(VF_NT)
   const uint32_t rd = rnd[n];
   if constexpr (WITH_DRAFT) {
     greedy_draft_body(gd.lsep, log2pi, gd.zhat, n, B, K, gd.M, V, gd.xhat_ws, gd.tok_ws,
-                      gd.qtok_ws, gd.cmask_ws, gd.out, X, tokS, eqS, cmS, piS, SS, qS);
+                      gd.qtok_ws, gd.cmask_ws, gd.ties_ws, gd.out, X, tokS, eqS, nearS, cmS, piS,
+                      SS, qS);
     __syncthreads();
   } else {
     for (int j = tid; j < B * K; j += VF_NT) X[j] = xhat[(size_t)n * B * K + j];
@@ -1319,8 +1357,11 @@ __global__ void __launch_bounds__(VF_NT)
     const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
     const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
     const int L = rej ? (__ffs(rej) - 1) : B;
-    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    const float amargin = fabsf(fmaf(u2, qtok, -ptok));
+    const bool atie = lane < B && lane <= L && amargin < TIE_TOL * qtok;
+    const bool anear = lane < B && lane <= L && amargin < (TIE_TOL + NEAR_ACCEPT) * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    if (__ballot_sync(FULLMASK, anear)) ties |= TIE_ACCEPT << NEAR_SHIFT;
     // App. B: collision probabilities of the block's target rows and
     // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
     float cC = 1.f;
@@ -1383,7 +1424,7 @@ __global__ void __launch_bounds__(VF_NT)
   __syncthreads();
   const int L = sL;
   int extra = -1;
-  bool tie = false;
+  bool tie = false, near = false;
   uint32_t tbits = 0;
   const int irow = (L < B) ? L : B;  // target row of the extra token
   if ((L < B) || (Bt > B)) {
@@ -1410,13 +1451,15 @@ __global__ void __launch_bounds__(VF_NT)
       }
       __syncthreads();
       if (sR < TIE_TOL) tbits |= TIE_RMASS;
+      if (sR < TIE_TOL + NEAR_DRAW) tbits |= TIE_RMASS << NEAR_SHIFT;
       const FindOut f = block_find<VF_NT>(nt, V, GreedyResidTileMass{ptm, atile, amass, na}, rm,
                                           FF{u3, 0.f}, 1.f, fs, true);
       extra = f.x;
       tie = f.tie;
+      near = f.near;
       if (extra < 0) {  // no positive residual mass left by rounding: draw from p
         from_p = true;
-        tie = true;
+        tie = near = true;
         tbits |= TIE_RMASS;
       }
     }
@@ -1424,10 +1467,13 @@ __global__ void __launch_bounds__(VF_NT)
       const FindOut f = block_find<VF_NT>(nt, V, ptm, pv, FF{u3, 0.f}, 1.f, fs);
       extra = f.x >= 0 ? f.x : 0;
       tie = tie || f.tie || f.x < 0;
+      near = near || f.near || f.x < 0;
     }
   }
   if (tid == 0) {
-    const uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u);
+    uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u) |
+                    (near ? (uint32_t)TIE_RESID << NEAR_SHIFT : 0u);
+    ties |= (ties & 0xffu) << NEAR_SHIFT;  // a tie is also near
     const int ne = L + (extra >= 0 ? 1 : 0);
     if (out.accepted) out.accepted[n] = L;
     if (out.n_emitted) out.n_emitted[n] = ne;
@@ -1458,6 +1504,7 @@ static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out
     gd.tok_ws = wsp<int32_t>(c, w.off_tok);
     gd.qtok_ws = wsp<float>(c, w.off_qtok);
     gd.cmask_ws = wsp<uint32_t>(c, w.off_cmask);
+    gd.ties_ws = wsp<uint32_t>(c, w.off_ties);
     if (dout) gd.out = *dout;
   }
   cudaError_t le = launch_dep(k_greedy_verify<Tin, WITH_DRAFT>, dim3(w.N), dim3(VF_NT), 0, c.stream,
@@ -1484,7 +1531,8 @@ cudaError_t launch_greedy_step_finalize(const StepCtx& c, const dblast_draft_out
   const int K = c.head->K;
   cudaError_t le =
       launch_dep(k_greedy_argmax, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
-                 c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
+                 c.stream, wsp<float2>(c, w.off_partd), wsp<float>(c, w.off_partg), w.nt, K, w.M,
+                 w.Mpad, wsp<float4>(c, w.off_lsep));
   debug_kernel("k_greedy_argmax", c.stream);
   count_launches(1);
   if (le != cudaSuccess) return le;
@@ -2156,8 +2204,11 @@ __global__ void __launch_bounds__(VF_NT)
     const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
     const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
     const int L = rej ? (__ffs(rej) - 1) : B;
-    const bool atie = lane < B && lane <= L && fabsf(fmaf(u2, qtok, -ptok)) < TIE_TOL * qtok;
+    const float amargin = fabsf(fmaf(u2, qtok, -ptok));
+    const bool atie = lane < B && lane <= L && amargin < TIE_TOL * qtok;
+    const bool anear = lane < B && lane <= L && amargin < (TIE_TOL + NEAR_ACCEPT) * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
+    if (__ballot_sync(FULLMASK, anear)) ties |= TIE_ACCEPT << NEAR_SHIFT;
     float cC = 1.f;
     if (lane < B) {
       cC = coll[(size_t)n * (B + 1) + lane];
@@ -2198,6 +2249,7 @@ __global__ void __launch_bounds__(VF_NT)
         j = warp_inverse_cdf(cnt, [&](int jj) { return fmaxf(pk[jj] - qS[L * kf + jj], 0.f); },
                              u3, &margin, &total);
         if (total < TIE_TOL) ties |= TIE_RMASS;
+        if (total < TIE_TOL + NEAR_DRAW) ties |= TIE_RMASS << NEAR_SHIFT;
         if (j < 0) {
           from_p = true;
           ties |= TIE_RMASS;
@@ -2205,6 +2257,7 @@ __global__ void __launch_bounds__(VF_NT)
       }
       if (from_p) j = warp_inverse_cdf(cnt, [&](int jj) { return pk[jj]; }, u3, &margin, &total);
       if (margin < TIE_TOL) ties |= TIE_RESID;
+      if (!(total > 0.f) || margin < TIE_TOL + NEAR_DRAW / total) ties |= TIE_RESID << NEAR_SHIFT;
       extra = j >= 0 ? tk[j] : (cnt > 0 ? tk[0] : 0);
     }
     if (lane == 0) {
@@ -2222,7 +2275,7 @@ __global__ void __launch_bounds__(VF_NT)
     const int ne = L + (extra >= 0 ? 1 : 0);
     if (out.accepted) out.accepted[n] = L;
     if (out.n_emitted) out.n_emitted[n] = ne;
-    if (out.tie_flags) out.tie_flags[n] = sties;
+    if (out.tie_flags) out.tie_flags[n] = sties | ((sties & 0xffu) << NEAR_SHIFT);
     pos[n] = p0 + ne;
     rnd[n] = rd + 1u;
   }
@@ -2339,6 +2392,10 @@ __global__ void __launch_bounds__(32)
   const bool in = lane < l_tau;
   if (__ballot_sync(FULLMASK, in && tau > 0.f && fabsf(lrf - l2tau) * LN2 < TIE_TOL))
     ties |= TIE_TAU;
+  // r_l multiplies l + 1 ratios, each within NEAR_ACCEPT (relative)
+  if (__ballot_sync(FULLMASK, in && tau > 0.f &&
+                                  fabsf(lrf - l2tau) * LN2 < TIE_TOL + NEAR_ACCEPT * (lane + 1)))
+    ties |= TIE_TAU << NEAR_SHIFT;
   FF jt{in ? lrf + ff_f(ff_log2(S)) : 0.f, 0.f};
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) jt = ff_add(jt, ff_shfl_xor(jt, o));
@@ -2367,7 +2424,7 @@ __global__ void __launch_bounds__(32)
     if (al.j_al) al.j_al[n] = ff_f(jt) * LN2;
     if (al.l_tau) al.l_tau[n] = l_tau;
     if (al.nll) al.nll[n] = (mx == -INFINITY) ? INFINITY : -(mx + log2f(e)) * LN2;
-    if (al.tie_flags) al.tie_flags[n] = ties;
+    if (al.tie_flags) al.tie_flags[n] = ties | ((ties & 0xffu) << NEAR_SHIFT);
   }
 }
 

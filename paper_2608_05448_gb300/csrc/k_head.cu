@@ -11,21 +11,31 @@ constexpr int RB = 16;  // rows (positions) per CTA of the CUDA-core passes
 // ---------------------------------------------------------------------------
 // draft pass on CUDA cores: stash = W h + b; partd per (tile, z, row).
 // Greedy-branch mode: no stash, and the records hold (max logit, its token)
-// with ties to the lowest index (the token's bits stored in the float).
-__device__ __forceinline__ float2 arg_merge2(float2 a, float2 b) {
+// with ties to the lowest index (the token's bits stored in the float), plus
+// the tile's second-largest logit in partg.
+// (max, token) merge, ties to the lower token, carrying the second-largest
+// values sa, sb of both sides
+__device__ __forceinline__ void arg_merge2s(float2& a, float& sa, float2 b, float sb) {
   const int ia = __float_as_int(a.y), ib = __float_as_int(b.y);
-  return (b.x > a.x || (b.x == a.x && ib < ia)) ? b : a;
+  if (b.x > a.x || (b.x == a.x && ib < ia)) {
+    sa = fmaxf(a.x, sb);
+    a = b;
+  } else {
+    sa = fmaxf(sa, b.x);
+  }
 }
 template <typename Tin>
 __global__ void __launch_bounds__(TILE_V)
     k_draft_simt(const Tin* __restrict__ W, const Tin* __restrict__ hid,
                  const float* __restrict__ vbias, const float* __restrict__ wu,
                  const float* __restrict__ codes, int V, int H, int K, int rr, int M, int Mpad,
-                 float k2, bool greedy, float* __restrict__ stash, float2* __restrict__ partd) {
+                 float k2, bool greedy, float* __restrict__ stash, float2* __restrict__ partd,
+                 float* __restrict__ partg) {
   extern __shared__ float smem[];
   float* hs = smem;                    // [RB][64]
   float* cs = smem + RB * 64;          // [K*rr]
   float2* red = reinterpret_cast<float2*>(cs + 32 * 65);  // [RB*K][4] (8-byte aligned offset)
+  float* redg = reinterpret_cast<float*>(red + RB * 32 * 4);  // [RB*K][4] greedy seconds
   const int t = blockIdx.x, m0 = blockIdx.y * RB, tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
   const int v = t * TILE_V + tid;
@@ -60,6 +70,7 @@ __global__ void __launch_bounds__(TILE_V)
     for (int z = 0; z < K; ++z) {
       float2 p = greedy ? make_float2(-INFINITY, __int_as_float(0x7fffffff))
                         : make_float2(-INFINITY, 0.f);
+      float sg = -INFINITY;  // greedy: second-largest logit of the merged lanes
       if (vok) {
         float corr = 0.f;
         const float* wr = wu + ((size_t)v * K + z) * rr;
@@ -71,12 +82,16 @@ __global__ void __launch_bounds__(TILE_V)
         for (int o = 16; o > 0; o >>= 1) {
           const float2 q = make_float2(__shfl_xor_sync(0xffffffffu, p.x, o),
                                        __shfl_xor_sync(0xffffffffu, p.y, o));
-          p = arg_merge2(p, q);
+          const float qs = __shfl_xor_sync(0xffffffffu, sg, o);
+          arg_merge2s(p, sg, q, qs);
         }
       } else {
         p = warp_lse_merge(p);
       }
-      if (lane == 0) red[(r * K + z) * 4 + warp] = p;
+      if (lane == 0) {
+        red[(r * K + z) * 4 + warp] = p;
+        redg[(r * K + z) * 4 + warp] = sg;
+      }
     }
     __syncthreads();
   }
@@ -84,8 +99,13 @@ __global__ void __launch_bounds__(TILE_V)
     const int r = idx / K, z = idx - r * K, m = m0 + r;
     if (m >= M) continue;
     float2 p = red[idx * 4];
-    for (int j = 1; j < 4; ++j) p = greedy ? arg_merge2(p, red[idx * 4 + j]) : lse_merge(p, red[idx * 4 + j]);
+    float sg = redg[idx * 4];
+    for (int j = 1; j < 4; ++j) {
+      if (greedy) arg_merge2s(p, sg, red[idx * 4 + j], redg[idx * 4 + j]);
+      else p = lse_merge(p, red[idx * 4 + j]);
+    }
     partd[((size_t)t * K + z) * Mpad + m] = p;
+    if (greedy) partg[((size_t)t * K + z) * Mpad + m] = sg;
   }
 }
 
@@ -93,11 +113,13 @@ template <typename Tin> static cudaError_t draft_simt_typed(const StepCtx& c) {
   const dblast_head* h = c.head;
   const WsLayout& w = c.wl;
   dim3 grid(w.nt, ceil_div(w.M, RB));
-  const size_t smem = (RB * 64 + 32 * 65) * sizeof(float) + RB * 32 * 4 * sizeof(float2);
+  const size_t smem = (RB * 64 + 32 * 65) * sizeof(float) + RB * 32 * 4 * sizeof(float2) +
+                      RB * 32 * 4 * sizeof(float);
   k_draft_simt<Tin><<<grid, TILE_V, smem, c.stream>>>(
       static_cast<const Tin*>(h->W), static_cast<const Tin*>(c.args->hidden), h->vbias,
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), h->V, h->H, h->K, w.rr, w.M,
-      w.Mpad, c.k2, c.greedy, wsp<float>(c, w.off_stash), wsp<float2>(c, w.off_partd));
+      w.Mpad, c.k2, c.greedy, wsp<float>(c, w.off_stash), wsp<float2>(c, w.off_partd),
+      wsp<float>(c, w.off_partg));
   debug_kernel("k_draft_simt", c.stream);
   count_launches(1);
   return cudaGetLastError();

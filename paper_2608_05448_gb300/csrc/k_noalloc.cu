@@ -68,21 +68,26 @@ __global__ void k_noalloc_merge(const float2* __restrict__ rec, int rows, int nt
 }
 
 // Device address of the static scratch, looked up once per device with that
-// device current (the first call on each device does it).
+// device current (the first call on each device does it), and again when the
+// device's context has changed since (a cudaDeviceReset loads the library's
+// device code anew, at an address that may differ).
 static std::mutex g_noalloc_mu;
 static float2* g_noalloc_addr[128] = {};
+static unsigned long long g_noalloc_ctx[128] = {};
 
 static cudaError_t noalloc_scratch(float2** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 128) return cudaErrorInvalidDevice;
+  const unsigned long long ctx = current_context_id();
   std::lock_guard<std::mutex> lk(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
+  if (!g_noalloc_addr[dev] || g_noalloc_ctx[dev] != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
     g_noalloc_addr[dev] = static_cast<float2*>(p);
+    g_noalloc_ctx[dev] = ctx;
   }
   *out = g_noalloc_addr[dev];
   return cudaSuccess;

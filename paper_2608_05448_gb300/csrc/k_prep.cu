@@ -241,6 +241,7 @@ __global__ void __launch_bounds__(256)
   }
   if (lane == 0) {
     if (zt != 0.f && margin < TIE_TOL) atomicOr(&ties[n], TIE_ZHAT);
+    if (zt != 0.f && margin < TIE_TOL + NEAR_DRAW) atomicOr(&ties[n], TIE_ZHAT << NEAR_SHIFT);
     zhat_ws[n] = zh;
   }
   if (on) log2pi_ws[n * K + lane] = pz > 0.f ? log2f(pz) : -INFINITY;

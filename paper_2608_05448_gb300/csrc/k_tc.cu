@@ -146,18 +146,6 @@ __device__ __forceinline__ void tma_load_3d_once(void* dst, const CUtensorMap* m
       : "memory");
 }
 
-// the same copy written to the same shared-memory offset of every CTA in
-// cta_mask (this GPU's own memory only); each destination's mbarrier at the
-// same offset receives the complete_tx bytes
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                               int x, int y, uint16_t cta_mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster "
-      "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(cta_mask)
-      : "memory");
-}
-
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -218,15 +206,6 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
-      : "memory");
-}
-
-// arrive on the mbarrier at this offset in every CTA of cta_mask once the
-// MMAs issued so far have completed
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t cta_mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
-      "[%0], %1;" ::"r"(smem_u32(bar)), "h"(cta_mask)
       : "memory");
 }
 
@@ -370,7 +349,7 @@ static_assert(DCfg<true>::SMEM <= 227 * 1024 && DCfg<false>::SMEM <= 227 * 1024,
 
 struct Params {
   int mode;
-  int cs;                    // CTAs per cluster: M tiles sharing one vocabulary tile (1, 2 or 4)
+  int cs;                    // CTAs per cluster: 2 for the CTA pair, else 1
   int n_mt, n_vt, n_tiles;   // M tiles, vocabulary tiles, cluster tiles (x ksplit in prep mode)
   int nb;                    // base stages per tile
   int K, rp, zps;            // components, padded rank, components per 64-wide block
@@ -381,6 +360,7 @@ struct Params {
   const float* sw;           // [K]
   float* stash;              // [M, V]
   float2* partd;             // [nt, K, Mpad]
+  float* partg;              // [nt, K, Mpad] greedy mode: second-largest logit of the record
   float* wu;                 // prep output [ksplit][V, prep_rows]
   int prep_rows;             // valid A rows in prep mode
   size_t split_stride;       // elements between the split-K partial outputs
@@ -397,10 +377,10 @@ struct Params {
   float* t_lse;              // [t_rows] natural log-sum-exp, or null
 };
 
-// Tile `slot` of this CTA.  The CTAs of one cluster (cs of them) share a
-// vocabulary tile and take consecutive M tiles; cluster tiles are numbered
-// split-major (prep mode), then vocabulary-major, so concurrently running
-// clusters also share B tiles through L2.
+// Tile `slot` of this CTA.  The two CTAs of a pair share a vocabulary tile
+// and take consecutive M tiles; cluster tiles are numbered split-major (prep
+// mode), then vocabulary-major, so concurrently running clusters also share
+// B tiles through L2.
 struct Sched {
   int cid, ncl, rank;  // cluster index, cluster count, rank in the cluster
 };
@@ -448,13 +428,9 @@ __device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
                                                unsigned char* stages, uint64_t* full,
                                                uint64_t* empty, const Ctl& ctl, int my_tiles) {
   using C = DCfg<PAIR>;
-  // with cs > 1 (single form) every CTA loads its own A tile and a 1/cs slice
-  // of the shared B tile, multicast to the whole cluster (the B maps then
-  // have DBN/cs rows); a pair CTA loads its own A tile and its half of B
+  // a pair CTA loads its own A tile and its half of the B tile (the B maps
+  // then have DBN/2 rows)
   const int bq = DBN / P.cs;
-  const bool mc = !PAIR && P.cs > 1;
-  const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
-  const uint32_t boff = (uint32_t)(S.rank * bq * BK * 2);
   const bool lead = !PAIR || S.rank == 0;
   const uint32_t full_cl = PAIR ? cluster_addr(full, 0) : 0u;  // the even CTA's full barriers
   int stage = 0;
@@ -474,8 +450,7 @@ __device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
       tma_load_2d_pair(sa + DSTAGE_A, mb, fcl, xk, y1);
     } else {
       tma_load_2d(sa, ma, fb, xk, y0);
-      if (!mc) tma_load_2d(sa + DSTAGE_A, mb, fb, xk, y1);
-      else tma_load_2d_mc(sa + DSTAGE_A + boff, mb, fb, xk, y1, mask);
+      tma_load_2d(sa + DSTAGE_A, mb, fb, xk, y1);
     }
     issued_mask |= 1u << stage;
     issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -530,8 +505,6 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
   constexpr int MM = PAIR ? 2 * BM : BM;
   const uint32_t id_base = idesc_f16(true, DBN, MM);
   const uint32_t id_corr = idesc_f16(false, DBN, MM);
-  const uint16_t mask = (uint16_t)((1u << P.cs) - 1u);
-  const bool mc = !PAIR && P.cs > 1;
   // shared-memory descriptors: the start-address field holds addr >> 4, so a
   // byte offset off inside the 1024-aligned stages moves it by off >> 4
   const uint64_t d0 = sdesc(smem_u32(stages));
@@ -543,7 +516,6 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
   // on the barrier at the same offset in both CTAs
   auto commit_all = [&](uint64_t* bar) {
     if constexpr (PAIR) umma_commit_pair(bar);
-    else if (mc) umma_commit_mc(bar, mask);
     else umma_commit(bar);
   };
   auto commit_acc = [&](uint64_t* bar) {
@@ -678,55 +650,44 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Two fp32 lanes per instruction (fma/add/sub/mul .rn.f32x2): each lane is
-// rounded exactly as the scalar instruction, with half the issue slots.
-struct F2 {
-  uint64_t v;
-};
-__device__ __forceinline__ F2 f2(float lo, float hi) {
-  F2 r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r.v) : "f"(lo), "f"(hi));
-  return r;
+// 2^x on the special-function unit, as a plain (reorderable) instruction
+__device__ __forceinline__ float ex2n(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
+
+// Two fp32 lanes per instruction (the compiler's packed fma/add/mul, round to
+// nearest): each lane is rounded exactly as the scalar instruction, with half
+// the issue slots.  a - b is fma(b, -1, a), exact up to the one rounding.
+typedef float2 F2;
+__device__ __forceinline__ F2 f2(float lo, float hi) { return make_float2(lo, hi); }
 __device__ __forceinline__ void f2_get(F2 a, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(a.v));
+  lo = a.x;
+  hi = a.y;
 }
-__device__ __forceinline__ F2 f2_fma(F2 a, F2 b, F2 c) {
-  F2 r;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r.v) : "l"(a.v), "l"(b.v), "l"(c.v));
-  return r;
-}
-__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
-  F2 r;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
-  return r;
-}
-__device__ __forceinline__ F2 f2_sub(F2 a, F2 b) {
-  F2 r;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
-  return r;
-}
-__device__ __forceinline__ F2 f2_mul(F2 a, F2 b) {
-  F2 r;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r.v) : "l"(a.v), "l"(b.v));
-  return r;
-}
-__device__ __forceinline__ F2 f2_ex2(F2 a) {
-  float lo, hi;
-  f2_get(a, lo, hi);
-  return f2(ex2(lo), ex2(hi));
-}
+__device__ __forceinline__ F2 f2_fma(F2 a, F2 b, F2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ F2 f2_sub(F2 a, F2 b) { return __ffma2_rn(b, make_float2(-1.f, -1.f), a); }
+__device__ __forceinline__ F2 f2_mul(F2 a, F2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ F2 f2_ex2(F2 a) { return make_float2(ex2n(a.x), ex2n(a.y)); }
 
 // Greedy-branch epilogue of one tile (Sec. 3.1, "Drafter sampling during
 // inference"): for every component z, the largest logit
 // l_v = base_v + b_v + D_z / (cscale sw) of this thread's 128 columns and its
 // token (lowest index on ties) become the record (max, index) of the half
-// tile; no stash and no exponentials.  Four interleaved chains keep the
-// compare-and-select sequences independent.
-__device__ __forceinline__ void arg_keep(float& mx, int& ix, float v, int i) {
+// tile, and the second-largest logit its tie record; no stash and no
+// exponentials.  Four interleaved chains keep the compare-and-select
+// sequences independent.
+// top-two merge of (max, index, second): the second of the union is the
+// larger of the losing max and the winner's own second
+__device__ __forceinline__ void arg_keep2(float& mx, int& ix, float& sc, float v, int i, float vs) {
   if (v > mx || (v == mx && i < ix)) {
+    sc = fmaxf(mx, vs);
     mx = v;
     ix = i;
+  } else {
+    sc = fmaxf(sc, v);
   }
 }
 template <bool PAIR>
@@ -745,6 +706,7 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
     tc_fence_after();
     const float a = az[z * D_EPI + et];
     float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
+    float s0 = -INFINITY, s1 = -INFINITY, s2 = -INFINITY, s3 = -INFINITY;
     int i0 = 0, i1 = 1, i2 = 2, i3 = 3;
     const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
     uint32_t ra[32], rb[32];
@@ -762,7 +724,12 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
         const float x1 = fmaf(__uint_as_float(cur[j + 1]), a, bk[c + 1]);
         const float x2 = fmaf(__uint_as_float(cur[j + 2]), a, bk[c + 2]);
         const float x3 = fmaf(__uint_as_float(cur[j + 3]), a, bk[c + 3]);
-        // each chain sees increasing columns, so a strict compare keeps the lowest
+        // each chain sees increasing columns, so a strict compare keeps the
+        // lowest; the chain's second is max(second, min(x, max)) before the update
+        s0 = fmaxf(s0, fminf(x0, m0));
+        s1 = fmaxf(s1, fminf(x1, m1));
+        s2 = fmaxf(s2, fminf(x2, m2));
+        s3 = fmaxf(s3, fminf(x3, m3));
         if (x0 > m0) { m0 = x0; i0 = c; }
         if (x1 > m1) { m1 = x1; i1 = c + 1; }
         if (x2 > m2) { m2 = x2; i2 = c + 2; }
@@ -776,10 +743,14 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
       if constexpr (PAIR) mbar_arrive_taken_cluster(cluster_addr(&cempty[rg], 0));
       else mbar_arrive_taken(&cempty[rg]);
     }
-    arg_keep(m0, i0, m1, i1);
-    arg_keep(m2, i2, m3, i3);
-    arg_keep(m0, i0, m2, i2);
-    if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(m0, __int_as_float(v0 + i0));
+    arg_keep2(m0, i0, s0, m1, i1, s1);
+    arg_keep2(m2, i2, s2, m3, i3, s3);
+    arg_keep2(m0, i0, s0, m2, i2, s2);
+    if (live) {
+      const size_t ro = ((size_t)rec * P.K + z) * P.Mpad + m;
+      P.partd[ro] = make_float2(m0, __int_as_float(v0 + i0));
+      P.partg[ro] = s0;
+    }
   }
   return true;
 }
@@ -1124,9 +1095,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
-      // one MMA commit from every CTA of a multicast cluster; a pair's MMAs
-      // are issued (and committed) by the even CTA alone
-      mbar_init(&empty[s], PAIR ? 1 : P.cs);
+      // a pair's MMAs are issued (and committed) by the even CTA alone
+      mbar_init(&empty[s], 1);
     }
     for (int g = 0; g < 2; ++g) {
       mbar_init(&bfull[g], 1);
@@ -1157,8 +1127,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // every CTA's barriers exist before any multicast copy or commit reaches them
-  if (PAIR || P.cs > 1) cluster_sync_all();
+  // both CTAs' barriers exist before the peer's copies or commits reach them
+  if (PAIR) cluster_sync_all();
   const uint32_t tmem = *tmem_slot;
   griddep_wait();  // the set-up above overlaps the end of the previous kernel
 
@@ -1192,8 +1162,8 @@ __global__ void __launch_bounds__(D_THREADS, 1)
       asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                    "r"(TMEM_COLS));
   }
-  // no CTA leaves while a peer may still multicast into it or arrive on it
-  if (PAIR || P.cs > 1) cluster_sync_all();
+  // no CTA leaves while its peer may still arrive on its barriers
+  if (PAIR) cluster_sync_all();
 }
 
 // ------------------------------------------------------------ verify pass
@@ -1632,6 +1602,10 @@ static int num_sms() {
 template <bool PAIR, bool GREEDY, bool TS>
 static cudaError_t pass_kernel_ready() {
   static int state = -1;
+  static unsigned long long ctx = 0ull;  // the attribute is set again in a new context
+  const unsigned long long cur = current_context_id();
+  if (cur != ctx) state = -1;
+  ctx = cur;
   if (state < 0) {
     cudaFuncAttributes fa;
     cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_pass<PAIR, GREEDY, TS>);
@@ -1686,7 +1660,7 @@ static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUte
   cudaError_t e = pass_kernel_ready<PAIR, GREEDY, TS>();
   if (e != cudaSuccess) return e;
   if (P.n_tiles <= 0) return cudaSuccess;
-  if (!PAIR && P.cs == 1) {
+  if (!PAIR) {
     const int grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
     e = launch_dep(k_tc_pass<false, GREEDY, TS>, dim3(grid), dim3(D_THREADS), DCfg<false>::SMEM, s, a,
                    b, ca, cb, P);
@@ -1704,19 +1678,6 @@ static cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUte
   count_launches(1);
   count_tc_launch();
   return cudaGetLastError();
-}
-
-// CTAs per cluster of the single-SM draft schedule: the M tiles that share a
-// vocabulary tile.  One by default: multicasting the shared B tile halves L2
-// reads but not the shared-memory traffic per SM, and the lockstep it imposes
-// measured slower on this GPU.  DBLAST_DRAFT_CLUSTER=2|4 selects the
-// multicast schedule (tests cover every size).
-static int draft_cluster_size(int n_mt) {
-  int cs = 1;
-  const char* env = getenv("DBLAST_DRAFT_CLUSTER");
-  if (env && (env[0] == '1' || env[0] == '2' || env[0] == '4') && env[1] == 0) cs = env[0] - '0';
-  while (cs > 1 && (n_mt % cs) != 0) cs >>= 1;
-  return cs;
 }
 
 // The CTA-pair schedule (the default) needs an even number of M tiles: a
@@ -1842,8 +1803,8 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   const WsLayout& w = c.wl;
   const int n_mt = w.Mpad / tc::BM;
   const bool pair = tc::draft_pair(n_mt);
-  const int cs = pair ? 2 : tc::draft_cluster_size(n_mt);
-  const uint32_t bq = tc::DBN / cs;  // B rows each CTA of a cluster loads
+  const int cs = pair ? 2 : 1;
+  const uint32_t bq = tc::DBN / cs;  // B rows each CTA loads
   CUtensorMap ma, mb, mca, mcb;
   const unsigned char* prep = c.prep;
   if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true, tc::BM) ||
@@ -1870,6 +1831,7 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   P.sw = prp<float>(c, c.pl.off_sw);
   P.stash = wsp<float>(c, w.off_stash);
   P.partd = wsp<float2>(c, w.off_partd);
+  P.partg = wsp<float>(c, w.off_partg);
   P.status = wsp<DevStatus>(c, w.off_status);
   P.spin_limit = wait_limit();
   if (c.fuse_tstats) {
@@ -1945,6 +1907,10 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
   P.spin_limit = wait_limit();
   // the register split (setmaxnreg) assumes exactly VREG registers per thread
   static int state = -1;
+  static unsigned long long ctx = 0ull;  // the attribute is set again in a new context
+  const unsigned long long cur = current_context_id();
+  if (cur != ctx) state = -1;
+  ctx = cur;
   if (state < 0) {
     cudaFuncAttributes fa;
     cudaError_t e = cudaFuncGetAttributes(&fa, tc::k_tc_verify);

@@ -141,12 +141,48 @@ def test_qwen3_4b_single_sequence_full(impl):
     _case(cfg, 1.0, 1.0, seed=0, impl=impl)
 
 
-@pytest.mark.parametrize("impl", IMPLS)
 @pytest.mark.parametrize("T", [1.0, 0.6])
-def test_qwen3_8b_batched_sampled(impl, T):
+def test_qwen3_8b_batched_all_sequences(T):
+    """The headline workload in the launch configuration the bench times
+    (tensor-core passes, N=32, B=16, K=8, r=16, H=4096, V=151936): every one
+    of the 32 sequences against the oracle, at both temperatures."""
     cfg = synth.config("qwen3_8b_b32")
+    st = _case(cfg, T, 1.0, seed=0, impl="auto")
+    assert st["sequences"] == 32 and st["emitted_checked"] >= 28
+
+
+def test_qwen3_8b_batched_simt_sampled():
+    """The CUDA-core passes on the headline shapes, two sequences."""
+    cfg = synth.config("qwen3_8b_b32")
+    _case(cfg, 1.0, 1.0, seed=0, impl="simt", seqs=[0, 31])
+
+
+@pytest.mark.parametrize("impl", IMPLS)
+@pytest.mark.parametrize("bonus,top_k,top_p", [(True, 0, 0.0), (False, 0, 0.0), (True, 20, 0.95),
+                                              (False, 20, 0.8)])
+def test_soft_split_calls_match_oracle(impl, bonus, top_k, top_p):
+    """dblast_draft_block, then dblast_verify_block on the workspace it left
+    (Sec. 3.1 drafting, then Algorithm 1's verification), against the oracle
+    element by element, with and without a bonus row and a target filter;
+    and the fused call on the same inputs gives the same decisions."""
+    cfg = synth.config("qwen3_8b_b32", V=6000, H=256, K=8, r=16, B=16, N=16, bonus=bonus)
     _skip_unsupported(cfg, impl)
-    _case(cfg, T, 1.0, seed=0, impl=impl, seqs=[0, 31])
+    head = synth.make_head(cfg, "cuda")
+    blk = synth.make_block(cfg, head, 0, "cuda")
+    seqs = list(range(cfg["N"]))
+    pos, rnd = synth.initial_state(cfg, "cuda")
+    pos0, rnd0 = pos.clone(), rnd.clone()
+    gpu = parity.run_gpu_split(head, blk, 0.9, 1.0, 12, pos, rnd, impl=impl, top_k=top_k,
+                               top_p=top_p)
+    orc = parity.run_oracle(head, blk, 0.9, 1.0, 12, pos0, rnd0, seqs, top_k=top_k, top_p=top_p)
+    parity.compare(gpu, orc, seqs)
+    assert torch.equal(pos.cpu(), pos0.cpu() + gpu["n_emitted"].long())
+    assert torch.equal(rnd.cpu(), rnd0.cpu() + 1)
+    posf, rndf = pos0.clone(), rnd0.clone()
+    fused = parity.run_gpu(head, blk, 0.9, 1.0, 12, posf, rndf, impl=impl, top_k=top_k,
+                           top_p=top_p)
+    for k in ("z_hat", "tokens", "accepted", "emitted", "n_emitted", "tie_flags"):
+        assert torch.equal(gpu[k], fused[k]), k
 
 
 @pytest.mark.parametrize("T,sigma", [(0.7, 0.3), (1.5, 1.0)])

@@ -40,30 +40,6 @@ def test_tc_prep_matches_cuda_core_prep(over, monkeypatch):
                           atol=1e-5 * float(ref.abs().max()))
 
 
-@pytest.mark.parametrize("cs", ["2", "4"])
-def test_draft_pass_cluster_multicast_matches_single_cta(cs, monkeypatch):
-    """The draft pass shares each vocabulary tile of the head between the CTAs
-    of a cluster (one M tile each, the tile multicast by slices).  Cluster
-    sizes only change who loads the operands, so every output must be
-    bit-identical to the one-CTA schedule; the oracle checks a few sequences."""
-    from tests import parity
-    cfg = synth.config("qwen3_8b_b32", V=20000, H=512, K=8, r=16, B=16, N=32)  # 4 M tiles
-    head = synth.make_head(cfg, "cuda")
-    blk = synth.make_block(cfg, head, 0, "cuda")
-    runs = {}
-    monkeypatch.setenv("DBLAST_DRAFT_PAIR", "0")  # the multicast schedule is a one-SM form
-    for c in ("1", cs):
-        monkeypatch.setenv("DBLAST_DRAFT_CLUSTER", c)
-        pos, rnd = synth.initial_state(cfg, "cuda")
-        runs[c] = parity.run_gpu(head, blk, 0.8, 1.0, 7, pos, rnd, impl="tcgen05")
-    for k, v in runs["1"].items():
-        assert torch.equal(v, runs[cs][k]), k
-    pos0, rnd0 = synth.initial_state(cfg, "cuda")
-    seqs = [0, 13, 31]
-    orc = parity.run_oracle(head, blk, 0.8, 1.0, 7, pos0, rnd0, seqs)
-    parity.compare(runs[cs], orc, seqs)
-
-
 @pytest.mark.parametrize("over", [dict(V=20000, H=512, K=8, r=16, B=16, N=32),   # 4 M tiles
                                   dict(V=3001, H=256, K=3, r=4, B=5, N=40,        # 2 M tiles
                                        expander_bias=True)])
