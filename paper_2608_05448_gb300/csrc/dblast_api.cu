@@ -149,7 +149,7 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_partt = take((size_t)w.nt * w.Rt * sizeof(float2));
   w.off_lt2 = take((size_t)w.Rt * sizeof(float2));
   w.off_partv = take((size_t)w.nt * w.Mpad * sizeof(float2));
-  w.off_ties = take((size_t)N * sizeof(uint32_t));
+  w.off_ties = take((size_t)2 * N * sizeof(uint32_t));  // tie flags, then per-sequence counters
   w.off_xhat = take((size_t)w.M * K * sizeof(int32_t));
   w.off_cmask = take((size_t)w.M * sizeof(uint32_t));
   w.off_coll = take((size_t)w.Rt * sizeof(float));
@@ -307,7 +307,7 @@ dblast_status dblast_head_prepare(const dblast_head* h, dblast_stream_t stream) 
 
 static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   g_calls.fetch_add(1, std::memory_order_relaxed);
-  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t),
+  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
                                   c.stream);
   if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
   if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
@@ -388,9 +388,10 @@ static cudaError_t side_stream(SideStream** out) {
   return cudaSuccess;
 }
 
-// draft and verify of one block with two forks: the category prior runs
-// beside the codes GEMM, and the target statistics beside the draft
-// finalize kernels (both pairs are independent and latency-bound).
+// draft and verify of one block.  The category prior runs beside the codes
+// GEMM on the library's second stream; the target statistics run inside the
+// draft pass (bf16 targets with 16-byte rows), else on the second stream
+// beside the draft finalize kernels, where the target filter also runs.
 static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_out* vout) {
   if (debug_sync()) {  // serial order, so a failing launcher is named
     dblast_status st = draft_impl(c, dout);
@@ -399,14 +400,12 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   c.target = vout->target;
   c.Bt = c.args->B + (vout->has_bonus ? 1 : 0);
   // bf16 targets with 16-byte rows: the draft pass's idle warps compute the
-  // target statistics while its tensor cores run.  It pays where the second
-  // stream's work after the draft pass (target statistics, filter) outlasts
-  // the draft finalize kernels: the greedy mode and the target filter.  In
-  // the plain stochastic step the two are about equal, and the extra memory
-  // traffic would slow the draft pass by more than it saves.
+  // target statistics while its tensor cores run.  The pass takes about 4%
+  // longer, but the latency-bound draft finalize kernels after it then run
+  // alone: beside a stand-alone statistics kernel, which fills HBM and the
+  // SMs, they took twice as long as on their own.
   c.fuse_tstats = c.tc && c.head->dtype == DBLAST_BF16 && (c.head->V % 8) == 0 &&
-                  aligned16(vout->target) && (c.greedy || filter_on(c.head, vout)) &&
-                  fuse_tstats_enabled();
+                  aligned16(vout->target) && fuse_tstats_enabled();
   c.lse_target = vout->lse_target;
   g_calls.fetch_add(2, std::memory_order_relaxed);
   std::lock_guard<std::mutex> lk(g_side_mu);
@@ -415,7 +414,7 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   StepCtx side = c;
   if (e == cudaSuccess) side.stream = ss->s;
   if (e == cudaSuccess)
-    e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t), c.stream);
+    e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t), c.stream);
   // fork 1: prior | codes
   if (e == cudaSuccess) e = cudaEventRecord(ss->ev[0], c.stream);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[0], 0);
@@ -570,7 +569,7 @@ dblast_status dblast_al_objective(const dblast_head* h, const dblast_block_args*
   c.target = al->target;
   c.Bt = a->B + vo.has_bonus;
   g_calls.fetch_add(1, std::memory_order_relaxed);
-  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)c.wl.N * sizeof(uint32_t),
+  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
                                   c.stream);
   if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
   if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);

@@ -66,7 +66,8 @@ struct PrepLayout {
 //   zhat i32 [N] | log2pi f32 [N,K] | stash f32 [M,V] | partd float2 [nt,K,Mpad]
 //   lsep float4 [LSE_SPLIT,M,K] | lse2, lq2, w2 ff [M,K] | qtok f32 [M] | tok i32 [M]
 //   vcz float2 [M,K] | vb0 f32 [M] | partt float2 [nt,Rt] | lt2 ff [Rt]
-//   partv float2 [nt,Mpad] | ties u32 [N]
+//   partv float2 [nt,Mpad] | ties u32 [N] then done u32 [N] (rows of a sequence
+//   with their draft token: the last one runs the posterior; zeroed per step)
 //   xhat i32 [M,K] | cmask u32 [M]   (greedy-branch mode: every branch's greedy
 //   token and the consistent-branch set C_i as a bit mask over z)
 //   partg f32 [nt,K,Mpad]  (greedy-branch mode: the second-largest logit of

@@ -121,6 +121,11 @@ struct FindOut {
   bool near;  // within TIE_TOL + near_abs / total (near_abs: an absolute mass allowance)
 };
 
+// A token-mass functor may stage the chosen tile first, with every thread of
+// the block (an overload of em_prepare for its type); the others read their
+// tokens directly.
+template <typename EM> __device__ __forceinline__ void em_prepare(const EM&, int) {}
+
 // Smallest token whose cumulative mass (in vocabulary order) exceeds `target`.
 // tmass(t): mass of tile t; emass(v): mass of token v (floats); `total` scales
 // the decision margin.  With `frac`, target.hi is a fraction u of the summed
@@ -212,6 +217,7 @@ __device__ FindOut block_find(int nt, int V, const TM tmass, const EM emass, FF 
   __syncthreads();
   const int tt = fs.tile;
   const FF before = fs.before;
+  em_prepare(emass, tt);
   float e = 0.f;
   const int v = tt * TILE_V + tid;
   if (tt >= 0 && tid < TILE_V && v < V) e = emass(v);
@@ -279,25 +285,48 @@ template <typename Tin> struct TargetTokenProb {  // p_i(v) = 2^{t_v k2 - Lt}
   FF Lt;
   __device__ float operator()(int v) const { return exp2_rel(ldf(trow + v), k2, Lt); }
 };
-template <typename Tin> struct ResidualTokenMass {  // [p(v) - q(v|x_<i)]_+
+// [p(v) - q(v|x_<i)]_+ of the tokens of one tile, computed by the whole
+// block once the tile is known (prepare): thread j takes token j % 128 and
+// the components z = g, g + G, ... with g = j / 128 and G = NT / 128, so
+// a token's K correction loads are spread over G threads; the partial sums
+// are then added in the order g = 0 .. G-1.
+template <typename Tin> struct ResidualTokenMass {
   TargetTokenProb<Tin> p;
   const float* srow;
   const float* wu;
   const float* cm;  // codes of row m, [K, rr]
   const FF* C;      // [K] in shared memory: L_z - log2 w_z (+inf if w_z = 0)
-  int K, rr;
+  float* qpart;     // [G * TILE_V] shared: partial q sums
+  float* pbuf;      // [TILE_V] shared: p(v) of the tile's tokens
+  int K, rr, V, G;
   float k2;
-  __device__ float operator()(int v) const {
+  __device__ void prepare(int tt) const {  // every thread of the block
+    const int tk = threadIdx.x % TILE_V, g = threadIdx.x / TILE_V;
+    const int v = tt * TILE_V + tk;
     float q = 0.f;
-    const float base = srow[v];
-    for (int z = 0; z < K; ++z) {
-      const FF c = C[z];
-      if (c.hi == INFINITY) continue;
-      q += exp2_rel2(base, corr_at(wu, cm + z * rr, v, z, K, rr), k2, c);
+    if (tt >= 0 && v < V && g < G) {
+      if (g == 0) pbuf[tk] = p(v);
+      const float base = srow[v];
+      for (int z = g; z < K; z += G) {
+        const FF c = C[z];
+        if (c.hi == INFINITY) continue;
+        q += exp2_rel2(base, corr_at(wu, cm + z * rr, v, z, K, rr), k2, c);
+      }
     }
-    return fmaxf(p(v) - q, 0.f);
+    if (g < G) qpart[threadIdx.x] = q;
+    __syncthreads();
+  }
+  __device__ float operator()(int v) const {  // thread v % TILE_V, after prepare
+    const int tk = threadIdx.x;
+    float q = 0.f;
+    for (int g = 0; g < G; ++g) q += qpart[g * TILE_V + tk];
+    return fmaxf(pbuf[tk] - q, 0.f);
   }
 };
+template <typename Tin>
+__device__ __forceinline__ void em_prepare(const ResidualTokenMass<Tin>& e, int tt) {
+  e.prepare(tt);
+}
 
 // ---------------------------------------------------------------- draft side
 // Partial log-sum-exps of the draft records: block (row group of 32, z, split);
@@ -353,9 +382,96 @@ __global__ void __launch_bounds__(LSE_WARPS * 32)
   }
 }
 
+// The category posterior of one sequence n (Eq. category-posterior) and
+// q(x_i|x_<i) (Eq. dep-next-token), run by one block of NT threads once every
+// row of the sequence has its token: log2 w_{i,z} from the prefix sums over
+// i of log2 q_z(x_j) (one thread per branch, positions in order), the
+// per-row constants of the tensor-core verify pass and the user-visible
+// draft outputs.  Rows of other blocks are read past L1 (ld.global.cg).
+struct PostShared {
+  FF A[32 * 32];   // log2 pi_z + sum_{j<i} log2 q_z(x_j), [B][K]
+  FF Lq[32 * 32];  // log2 q_z(x_i)
+  FF Lz[32 * 32];  // lse2 of every (i, z)
+  float E[32 * 32];
+  FF rowv[32];
+  float rowb[32];
+};
+__device__ __forceinline__ FF ff_ldcg(const float2* p) {
+  const float2 v = __ldcg(p);
+  return FF{v.x, v.y};
+}
+template <int NT>
+__device__ void posterior_seq(int n, const float2* __restrict__ lq2, const float2* __restrict__ lse2,
+                              const float* __restrict__ log2pi, const int32_t* __restrict__ zhat,
+                              const int32_t* __restrict__ tok, const float* __restrict__ cscale,
+                              const float* __restrict__ sw, float k2, int B, int K,
+                              float2* __restrict__ w2, float* __restrict__ qtok,
+                              float2* __restrict__ vcz, float* __restrict__ vb0,
+                              const dblast_draft_out& out, PostShared& ps) {
+  const int t = threadIdx.x, BK = B * K;
+  const size_t mb = (size_t)n * B;
+  for (int e = t; e < BK; e += NT) {
+    ps.Lq[e] = ff_ldcg(lq2 + mb * K + e);
+    ps.Lz[e] = ff_ldcg(lse2 + mb * K + e);
+  }
+  __syncthreads();
+  if (t < K) {  // exclusive prefix over positions, branch t
+    const float lp = log2pi[n * K + t];
+    FF run{0.f, 0.f};
+    for (int i = 0; i < B; ++i) {
+      ps.A[i * K + t] = (lp == -INFINITY || run.hi == -INFINITY) ? FF{-INFINITY, 0.f}
+                                                                : ff_addf(run, lp);
+      run = ff_add(run, ps.Lq[i * K + t]);
+    }
+  }
+  __syncthreads();
+  for (int i = t; i < B; i += NT) {  // log2 sum_z of row i, and B0 of the verify pass
+    float mx = -INFINITY, lmx = -INFINITY;
+    for (int k = 0; k < K; ++k) {
+      mx = fmaxf(mx, ps.A[i * K + k].hi);
+      lmx = fmaxf(lmx, ps.Lz[i * K + k].hi);
+    }
+    FF S{0.f, 0.f};
+    if (mx != -INFINITY)
+      for (int k = 0; k < K; ++k)
+        if (ps.A[i * K + k].hi != -INFINITY) S = ff_addf(S, ff_exp2(ff_addf(ps.A[i * K + k], -mx)));
+    ps.rowv[i] = (mx == -INFINITY) ? FF{-INFINITY, 0.f} : ff_add(FF{mx, 0.f}, ff_log2(S));
+    ps.rowb[i] = floorf(lmx);  // keeps the verify pass's two factors in range
+  }
+  __syncthreads();
+  for (int e = t; e < BK; e += NT) {
+    const int i = e / K, z = e - i * K;
+    const size_t m = mb + i;
+    const FF acc = ps.A[e], lz = ps.rowv[i], lq = ps.Lq[e];
+    const bool wdead = acc.hi == -INFINITY || lz.hi == -INFINITY;
+    const FF wz = wdead ? FF{-INFINITY, 0.f} : ff_sub(acc, lz);
+    ps.E[e] = (wdead || lq.hi == -INFINITY) ? 0.f : ff_exp2(ff_add(wz, lq));
+    const FF Lz = ps.Lz[e];
+    w2[m * K + z] = ff_st(wz);
+    vcz[m * K + z] = make_float2(k2 / (cscale[m * K + z] * sw[z]),
+                                 wdead ? -INFINITY : ff_f(ff_addf(ff_sub(wz, Lz), ps.rowb[i])));
+    if (out.logw) out.logw[m * K + z] = wdead ? -INFINITY : ff_f(wz) * LN2;
+    if (out.lse) out.lse[m * K + z] = ff_f(Lz) * LN2;
+  }
+  __syncthreads();
+  for (int i = t; i < B; i += NT) {
+    const size_t m = mb + i;
+    FF qt{0.f, 0.f};
+    for (int k = 0; k < K; ++k) qt = ff_addf(qt, ps.E[i * K + k]);
+    qtok[m] = ff_f(qt);
+    vb0[m] = ps.rowb[i];
+    if (out.q_tok) out.q_tok[m] = ff_f(qt);
+    if (out.tokens) out.tokens[m] = __ldcg(tok + m);
+  }
+  if (t < K && out.pi) out.pi[n * K + t] = exp2f(log2pi[n * K + t]);
+  if (t == 0 && out.z_hat) out.z_hat[n] = zhat[n];
+}
+
 // One block per row m = (n, i): lse2 of every branch, the draft token
-// x_i ~ q_i(.|z-hat) (stream 1), and log2 q_z(x_i) for every branch.
-constexpr int DT_NT = 128;
+// x_i ~ q_i(.|z-hat) (stream 1), and log2 q_z(x_i) for every branch; the
+// last block of a sequence to finish (a per-sequence counter, zeroed before
+// the step) then runs that sequence's posterior.
+constexpr int DT_NT = 256;
 __global__ void __launch_bounds__(DT_NT)
     k_draft_token(const float2* __restrict__ partd, const float4* __restrict__ lsep,
                   const float* __restrict__ stash, const float* __restrict__ wu,
@@ -364,10 +480,16 @@ __global__ void __launch_bounds__(DT_NT)
                   const int64_t* __restrict__ pos, const uint32_t* __restrict__ rnd,
                   const int32_t* __restrict__ given, float2* __restrict__ lse2,
                   int32_t* __restrict__ tok, float2* __restrict__ lq2,
-                  uint32_t* __restrict__ ties) {
+                  uint32_t* __restrict__ ties, uint32_t* __restrict__ done,
+                  const float* __restrict__ log2pi, const float* __restrict__ cscale,
+                  const float* __restrict__ sw, float2* __restrict__ w2,
+                  float* __restrict__ qtok, float2* __restrict__ vcz, float* __restrict__ vb0,
+                  dblast_draft_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<DT_NT> fs;
   __shared__ FF sL[32];
+  __shared__ int s_last;
+  __shared__ PostShared ps;
   const int m = blockIdx.x, tid = threadIdx.x;
   const int n = m / B, i = m - n * B;
   // the sampled branch and the draw's uniform do not depend on the merge below
@@ -413,84 +535,16 @@ __global__ void __launch_bounds__(DT_NT)
     const FF s = ff_add(ff_prod(srow[x], k2), ff_prod(corr_at(wu, cm + tid * rr, x, tid, K, rr), k2));
     lq2[(size_t)m * K + tid] = ff_st(ff_sub(s, sL[tid]));
   }
-}
-
-// One block per sequence, thread t = (i, z) with i = t / K: the category
-// posterior log2 w_{i,z} (Eq. category-posterior) from prefix sums over i of
-// log2 q_z(x_j), q(x_i|x_<i) (Eq. dep-next-token), the per-row constants of
-// the tensor-core verify pass, and the user-visible draft outputs.
-__global__ void __launch_bounds__(1024)
-    k_posterior(const float2* __restrict__ lq2, const float2* __restrict__ lse2,
-                const float* __restrict__ log2pi, const int32_t* __restrict__ zhat,
-                const int32_t* __restrict__ tok, const float* __restrict__ cscale,
-                const float* __restrict__ sw, float k2, int B, int K, float2* __restrict__ w2,
-                float* __restrict__ qtok, float2* __restrict__ vcz, float* __restrict__ vb0,
-                dblast_draft_out out) {
-  griddep_wait();  // launched as a dependent of the previous kernel
-  __shared__ FF A[1024];
-  __shared__ FF rowv[32];
-  __shared__ float rowb[32];
-  __shared__ float E[1024];
-  const int n = blockIdx.x, t = threadIdx.x;
-  const int i = t / K, z = t - i * K;
-  const bool ok = i < B;
-  const size_t m = (size_t)n * B + (ok ? i : 0);
-  const FF lq = ok ? ff_ld(lq2 + m * K + z) : FF{0.f, 0.f};
-  // exclusive prefix over positions: A[i][z] = sum_{j<i} log2 q_z(x_j)
-  A[t] = (ok && i > 0) ? ff_ld(lq2 + (m - 1) * K + z) : FF{0.f, 0.f};
+  // this row's results are written: count it, and the sequence's last row
+  // block runs the posterior
+  __threadfence();
   __syncthreads();
-  for (int o = 1; o < B; o <<= 1) {
-    const FF v = (ok && i >= o) ? A[t - o * K] : FF{0.f, 0.f};
-    __syncthreads();
-    if (ok) A[t] = ff_add(v, A[t]);
-    __syncthreads();
-  }
-  const float lp = ok ? log2pi[n * K + z] : -INFINITY;
-  const FF acc = (lp == -INFINITY || A[t].hi == -INFINITY) ? FF{-INFINITY, 0.f}
-                                                           : ff_addf(A[t], lp);
+  if (tid == 0) s_last = atomicAdd(&done[n], 1u) == (uint32_t)(B - 1);
   __syncthreads();
-  A[t] = acc;
-  __syncthreads();
-  if (ok && z == 0) {
-    float mx = -INFINITY, lmx = -INFINITY;
-    for (int k = 0; k < K; ++k) {
-      mx = fmaxf(mx, A[t + k].hi);
-      lmx = fmaxf(lmx, lse2[m * K + k].x);
-    }
-    FF S{0.f, 0.f};
-    if (mx != -INFINITY)
-      for (int k = 0; k < K; ++k)
-        if (A[t + k].hi != -INFINITY) S = ff_addf(S, ff_exp2(ff_addf(A[t + k], -mx)));
-    rowv[i] = (mx == -INFINITY) ? FF{-INFINITY, 0.f} : ff_add(FF{mx, 0.f}, ff_log2(S));
-    rowb[i] = floorf(lmx);  // B0 of the verify pass: keeps its two factors in range
-  }
-  __syncthreads();
-  const FF lz = ok ? rowv[i] : FF{-INFINITY, 0.f};
-  const bool wdead = acc.hi == -INFINITY || lz.hi == -INFINITY;
-  const FF wz = wdead ? FF{-INFINITY, 0.f} : ff_sub(acc, lz);
-  E[t] = (wdead || lq.hi == -INFINITY) ? 0.f : ff_exp2(ff_add(wz, lq));
-  __syncthreads();
-  if (ok) {
-    const FF Lz = ff_ld(lse2 + m * K + z);
-    w2[m * K + z] = ff_st(wz);
-    const float b0 = rowb[i];
-    vcz[m * K + z] = make_float2(k2 / (cscale[m * K + z] * sw[z]),
-                                 wdead ? -INFINITY : ff_f(ff_addf(ff_sub(wz, Lz), b0)));
-    if (out.logw) out.logw[m * K + z] = wdead ? -INFINITY : ff_f(wz) * LN2;
-    if (out.lse) out.lse[m * K + z] = ff_f(Lz) * LN2;
-    if (z == 0) {
-      FF qt{0.f, 0.f};
-      for (int k = 0; k < K; ++k) qt = ff_addf(qt, E[t + k]);
-      qtok[m] = ff_f(qt);
-      vb0[m] = b0;
-      if (out.q_tok) out.q_tok[m] = ff_f(qt);
-      if (out.tokens) out.tokens[m] = tok[m];
-    }
-  }
-  if (t < K) {
-    if (out.pi) out.pi[n * K + t] = exp2f(log2pi[n * K + t]);
-    if (out.z_hat && t == 0) out.z_hat[n] = zhat[n];
-  }
+  if (!s_last) return;
+  __threadfence();
+  posterior_seq<DT_NT>(n, lq2, lse2, log2pi, zhat, tok, cscale, sw, k2, B, K, w2, qtok, vcz, vb0,
+                       out, ps);
 }
 
 cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp,
@@ -502,23 +556,19 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
       launch_dep(k_draft_lse, dim3(ceil_div(w.M, 32), K, LSE_SPLIT), dim3(LSE_WARPS * 32), 0,
                  c.stream, wsp<float2>(c, w.off_partd), w.nt, K, w.M, w.Mpad, wsp<float4>(c, w.off_lsep));
   debug_kernel("k_draft_lse", c.stream);
+  dblast_draft_out out{};
+  if (outp) out = *outp;
   if (le == cudaSuccess) le = launch_dep(k_draft_token, dim3(w.M), dim3(DT_NT), 0, c.stream,
       wsp<float2>(c, w.off_partd), wsp<float4>(c, w.off_lsep), wsp<float>(c, w.off_stash),
       prp<float>(c, c.pl.off_wu), wsp<float>(c, w.off_codes), wsp<int32_t>(c, w.off_zhat), w.nt,
       w.V, K, w.rr, w.B, w.M, w.Mpad, c.k2, a->seed, a->pos, a->round, given,
       wsp<float2>(c, w.off_lse2),
-      wsp<int32_t>(c, w.off_tok), wsp<float2>(c, w.off_lq2), wsp<uint32_t>(c, w.off_ties));
-  debug_kernel("k_draft_token", c.stream);
-  dblast_draft_out out{};
-  if (outp) out = *outp;
-  const int pt = ceil_div(w.B * K, 32) * 32;
-  if (le == cudaSuccess) le = launch_dep(k_posterior, dim3(w.N), dim3(pt), 0, c.stream,
-      wsp<float2>(c, w.off_lq2), wsp<float2>(c, w.off_lse2), wsp<float>(c, w.off_log2pi),
-      wsp<int32_t>(c, w.off_zhat), wsp<int32_t>(c, w.off_tok), wsp<float>(c, w.off_cscale),
-      prp<float>(c, c.pl.off_sw), c.k2, w.B, K, wsp<float2>(c, w.off_w2),
+      wsp<int32_t>(c, w.off_tok), wsp<float2>(c, w.off_lq2), wsp<uint32_t>(c, w.off_ties),
+      wsp<uint32_t>(c, w.off_ties) + w.N, wsp<float>(c, w.off_log2pi),
+      wsp<float>(c, w.off_cscale), prp<float>(c, c.pl.off_sw), wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_vcz), wsp<float>(c, w.off_vb0), out);
-  debug_kernel("k_posterior", c.stream);
-  count_launches(3);
+  debug_kernel("k_draft_token", c.stream);
+  count_launches(2);
   return le != cudaSuccess ? le : cudaGetLastError();
 }
 
@@ -804,12 +854,16 @@ cudaError_t launch_target_stats(const StepCtx& c, const dblast_verify_out* o) {
 
 // ---------------------------------------------------------------- verify side
 // One block per sequence: the per-row sums of the verify records (alpha_i and
-// the residual mass, thread (s, i) over tiles s, s + S, ... with consecutive
-// threads on consecutive rows of a tile), acceptance (stream 2), residual or
-// bonus draw (stream 3), expected lengths, emitted tokens, state update.
-constexpr int VF_NT = 256;
+// the residual mass), acceptance (stream 2), residual or bonus draw (stream
+// 3), expected lengths, emitted tokens, state update.  Warp 0 loads what the
+// acceptance test needs (tokens, p and q at them, the uniforms, collision
+// probabilities, the rows' branch normalisers) while warps 1.. add the
+// records: thread (s, i) takes tiles s, s + S, ... of row i, consecutive
+// threads on consecutive rows of a tile.
+constexpr int VF_NT = 256;   // threads of the per-sequence kernels of the other modes
+constexpr int VFS_NT = 512;  // threads of the stochastic-mode verify-final kernel
 template <typename Tin>
-__global__ void __launch_bounds__(VF_NT)
+__global__ void __launch_bounds__(VFS_NT, 1)
     k_verify_final(const Tin* __restrict__ target, const float* __restrict__ stash,
                    const float* __restrict__ wu, const float* __restrict__ codes,
                    const float2* __restrict__ lse2, const float2* __restrict__ w2,
@@ -822,21 +876,50 @@ __global__ void __launch_bounds__(VF_NT)
                    int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
                    dblast_verify_out out) {
   griddep_wait();  // launched as a dependent of the previous kernel
-  __shared__ FindShared<VF_NT> fs;
+  constexpr int G = VFS_NT / TILE_V;
+  __shared__ FindShared<VFS_NT> fs;
   __shared__ FF sC[32];
   __shared__ int sL;
   __shared__ uint32_t sties;
   __shared__ FF sR;
-  __shared__ FF pa[VF_NT], pr[VF_NT];
+  __shared__ FF pa[VFS_NT], pr[VFS_NT];
   __shared__ FF rowA[32], rowR[32];
+  __shared__ FF sCall[32 * 32];  // L_z - log2 w_z of every (i, z), +inf if w_z = 0
+  __shared__ float qpart[G * TILE_V], pbuf[TILE_V];
+  __shared__ float sacc[4][32];  // p(x_i), q(x_i|x_<i), u_i, coll_i
   const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
   const int64_t p0 = pos[n];
   const uint32_t rd = rnd[n];
-  {
-    const int S = VF_NT / B;  // tile strides per row (B <= 32)
+  if (tid < 32) {
+    // lane i: p(x_i) and q(x_i|x_<i), the acceptance uniform, coll_i, kept in
+    // shared memory so that the loads complete while warps 1.. add records
+    float ptok = 0.f, qtok = 1.f, u2 = 0.f, cC = 1.f;
+    if (lane < B) {
+      const int m = n * B + lane;
+      const int x = min(max(tok[m], 0), V - 1);
+      const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
+      const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
+      qtok = qtok_ws[m];
+      cC = coll[(size_t)n * (B + 1) + lane];
+      u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
+      ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
+    }
+    sacc[0][lane] = ptok;
+    sacc[1][lane] = qtok;
+    sacc[2][lane] = u2;
+    sacc[3][lane] = cC;
+    if (lane == 0) sties = ties_draft[n];
+    for (int j = lane; j < B * K; j += 32) {
+      const size_t mz = (size_t)n * B * K + j;
+      const FF wz = ff_ld(w2 + mz);
+      sCall[j] = (wz.hi == -INFINITY) ? FF{INFINITY, 0.f} : ff_sub(ff_ld(lse2 + mz), wz);
+    }
+  } else {
+    const int S = (VFS_NT - 32) / B;  // tile strides per row (B <= 32)
+    const int t32 = tid - 32;
     FF a{0.f, 0.f}, r{0.f, 0.f};
-    if (tid < S * B) {
-      const int i = tid % B, s0 = tid / B;
+    if (t32 < S * B) {
+      const int i = t32 % B, s0 = t32 / B;
       const float2* pv = partv + (size_t)n * B + i;
       // eight records in flight per thread
       for (int t = s0; t < nt; t += 8 * S) {
@@ -855,38 +938,36 @@ __global__ void __launch_bounds__(VF_NT)
     }
     pa[tid] = a;
     pr[tid] = r;
-    __syncthreads();
-    if (tid < B) {
-      FF A{0.f, 0.f}, R{0.f, 0.f};
-      for (int s0 = 0; s0 < S; ++s0) {
-        A = ff_add(A, pa[s0 * B + tid]);
-        R = ff_add(R, pr[s0 * B + tid]);
-      }
-      rowA[tid] = A;
-      rowR[tid] = R;
-    }
-    __syncthreads();
   }
+  __syncthreads();
+  if (tid < B) {
+    const int S = (VFS_NT - 32) / B;
+    FF A{0.f, 0.f}, R{0.f, 0.f};
+    for (int s0 = 0; s0 < S; ++s0) {
+      A = ff_add(A, pa[32 + s0 * B + tid]);
+      R = ff_add(R, pr[32 + s0 * B + tid]);
+    }
+    rowA[tid] = A;
+    rowR[tid] = R;
+  }
+  __syncthreads();
   if (tid < 32) {
-    // lane i: p(x_i), q(x_i|x_<i), acceptance
-    uint32_t ties = ties_draft[n];
-    float A = 0.f, alpha = 0.f, ptok = 0.f, qtok = 1.f, u2 = 0.f;
+    // lane i: acceptance u < p/q
+    const float ptok = sacc[0][lane], qtok = sacc[1][lane], u2 = sacc[2][lane];
+    float cC = sacc[3][lane];
+    uint32_t ties = sties;
+    float A = 0.f, alpha = 0.f;
     bool acc_ok = false;
     if (lane < B) {
       const int m = n * B + lane;
-      const int x = min(max(tok[m], 0), V - 1);
-      const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
-      const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
-      ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
-      qtok = qtok_ws[m];
       const float ratio = ptok / qtok;
       A = fminf(1.f, ratio);
       alpha = ff_f(rowA[lane]);
-      u2 = decision_uniform(seed, 2u, rd, (uint32_t)n, (uint32_t)(p0 + lane));
       acc_ok = u2 < ratio;
       if (out.p_tok) out.p_tok[m] = ptok;
       if (out.accept_prob) out.accept_prob[m] = A;
       if (out.alpha) out.alpha[m] = alpha;
+      if (out.collision) out.collision[n * B + lane] = cC;
     }
     const unsigned acc_mask = __ballot_sync(FULLMASK, acc_ok);
     const unsigned rej = ~acc_mask & ((B >= 32) ? FULLMASK : ((1u << B) - 1u));
@@ -900,12 +981,8 @@ __global__ void __launch_bounds__(VF_NT)
     // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha (products in lane order)
     // App. B: collision probabilities of the block's target rows and
     // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
-    float cC = 1.f;
-    if (lane < B) {
-      cC = coll[(size_t)n * (B + 1) + lane];
-      if (out.collision) out.collision[n * B + lane] = cC;
-    }
     float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
+    if (lane >= B) cC = 1.f;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const float ta = __shfl_up_sync(FULLMASK, cA, o);
@@ -928,11 +1005,7 @@ __global__ void __launch_bounds__(VF_NT)
       ea = ff_add(ea, ff_shfl_xor(ea, o));
       ed = ff_add(ed, ff_shfl_xor(ed, o));
     }
-    if (L < B && lane < K) {  // normalisers of the rejected row: L_z - log2 w_z
-      const size_t mz = (size_t)(n * B + L) * K + lane;
-      const FF wz = ff_ld(w2 + mz);
-      sC[lane] = (wz.hi == -INFINITY) ? FF{INFINITY, 0.f} : ff_sub(ff_ld(lse2 + mz), wz);
-    }
+    if (L < B && lane < K) sC[lane] = sCall[L * K + lane];  // normalisers of the rejected row
     if (lane == 0) {
       if (out.exp_len) out.exp_len[n] = ff_f(el);
       if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
@@ -961,10 +1034,10 @@ __global__ void __launch_bounds__(VF_NT)
       if (Rf < TIE_TOL) tbits |= TIE_RMASS;
       if (Rf < TIE_TOL + NEAR_DRAW) tbits |= TIE_RMASS << NEAR_SHIFT;
       if (Rf > 0.f) {
-        const ResidualTokenMass<Tin> rm{pv, stash + (size_t)m * V, wu,
-                                        codes + (size_t)m * K * rr, sC, K, rr, k2};
-        const FindOut f = block_find<VF_NT>(nt, V, ResidTileMass{partv + m, (size_t)Mpad}, rm,
-                                            ff_mulf(Rm, u3), Rf, fs);
+        const ResidualTokenMass<Tin> rm{pv, stash + (size_t)m * V, wu, codes + (size_t)m * K * rr,
+                                        sC, qpart, pbuf, K, rr, V, G, k2};
+        const FindOut f = block_find<VFS_NT>(nt, V, ResidTileMass{partv + m, (size_t)Mpad}, rm,
+                                             ff_mulf(Rm, u3), Rf, fs);
         extra = f.x;
         tie = f.tie;
         near = f.near;
@@ -976,26 +1049,26 @@ __global__ void __launch_bounds__(VF_NT)
       }
     }
     if (from_p) {
-      const FindOut f = block_find<VF_NT>(nt, V, TargetTileMass{partt + rl, (size_t)Rt, k2, Lt},
-                                          pv, FF{u3, 0.f}, 1.f, fs);
+      const FindOut f = block_find<VFS_NT>(nt, V, TargetTileMass{partt + rl, (size_t)Rt, k2, Lt},
+                                           pv, FF{u3, 0.f}, 1.f, fs);
       extra = f.x >= 0 ? f.x : 0;
       tie = tie || f.tie || f.x < 0;
       near = near || f.near || f.x < 0;
     }
   }
   if (tid == 0) {
-    uint32_t ties = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u) |
-                    (near ? (uint32_t)TIE_RESID << NEAR_SHIFT : 0u);
-    ties |= (ties & 0xffu) << NEAR_SHIFT;  // a tie is also near
+    uint32_t tf = sties | tbits | (tie ? (uint32_t)TIE_RESID : 0u) |
+                  (near ? (uint32_t)TIE_RESID << NEAR_SHIFT : 0u);
+    tf |= (tf & 0xffu) << NEAR_SHIFT;  // a tie is also near
     const int ne = L + (extra >= 0 ? 1 : 0);
     if (out.accepted) out.accepted[n] = L;
     if (out.n_emitted) out.n_emitted[n] = ne;
-    if (out.tie_flags) out.tie_flags[n] = ties;
+    if (out.tie_flags) out.tie_flags[n] = tf;
     pos[n] = p0 + ne;
     rnd[n] = rd + 1u;
   }
   if (out.emitted) {
-    for (int j = tid; j < B + 1; j += VF_NT) {
+    for (int j = tid; j < B + 1; j += VFS_NT) {
       int val = -1;
       if (j < L) val = tok[n * B + j];
       else if (j == L && extra >= 0) val = extra;
@@ -1008,7 +1081,7 @@ template <typename Tin>
 static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out* o) {
   const int Bt = c.Bt;
   const WsLayout& w = c.wl;
-  cudaError_t le = launch_dep(k_verify_final<Tin>, dim3(w.N), dim3(VF_NT), 0, c.stream,
+  cudaError_t le = launch_dep(k_verify_final<Tin>, dim3(w.N), dim3(VFS_NT), 0, c.stream,
       static_cast<const Tin*>(o->target), wsp<float>(c, w.off_stash), prp<float>(c, c.pl.off_wu),
       wsp<float>(c, w.off_codes), wsp<float2>(c, w.off_lse2), wsp<float2>(c, w.off_w2),
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
