@@ -27,6 +27,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "draft+verify blocks/sec and accepted tokens/sec at 1 GB300; % of roofline"
+PASS_TIMING_PERIOD = 4
 UNIT = "blocks/s"
 
 
@@ -504,7 +505,10 @@ def main():
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    dblast_stats_reset(True)
+    # CUDA events around the passes of every PASS_TIMING_PERIOD-th timed step
+    # only: an event between two kernels keeps the later one from starting
+    # early, so timing every step would slow the step it measures
+    dblast_stats_reset(PASS_TIMING_PERIOD)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record()
     for k in range(K_steps):
@@ -651,7 +655,9 @@ def main():
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"],
                          "unit": "TFLOP/s", "frac": achieved / peaks["bf16"],
                          "traffic": traffic, "kernel": "draft pass",
-                         "ms_per_launch": draft_ms},
+                         "ms_per_launch": draft_ms, "timed_launches": int(st["timed_draft"]),
+                         "timing": "CUDA events on the launching stream around the draft "
+                                   "pass of every %dth timed step" % PASS_TIMING_PERIOD},
             "verify_pass_ms": verify_ms,
             "ties": {"sequences_flagged_per_step": tie_seqs / K_steps,
                      "sequences_flagged": tie_seqs, "sequences": N * K_steps,

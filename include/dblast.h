@@ -211,13 +211,17 @@ dblast_status dblast_device_status(void* workspace, dblast_stream_t stream);
  * waits of later calls (0 = default).  A limit of 1 makes waits give up. */
 void dblast_set_wait_limit(uint32_t spins);
 
-/* Measurement counters of this process.  dblast_stats_reset() zeroes them and
- * turns per-pass timing on or off: while on, every call records CUDA events
- * on its stream around its draft pass (the vocabulary-head contraction with
- * its fused softmax epilogue) and its verify pass (the fused target-streaming
- * kernel).  dblast_stats_get() waits for the recorded events and returns the
- * summed pass times (ms), the number of timed calls and the number of kernel
- * launches issued by the library since the reset. */
+/* Measurement counters of this process.  dblast_stats_reset(n) zeroes them
+ * and sets per-pass timing: with n > 0, CUDA events are recorded on the
+ * caller's stream around every n-th draft pass (the vocabulary-head
+ * contraction with its fused softmax epilogue) and every n-th verify pass
+ * (the fused target-streaming kernel) from the reset on; n = 0 turns it off.
+ * An event between two kernels keeps the later one from starting while the
+ * earlier one drains, so a timed call runs a little slower than an untimed
+ * one; n > 1 leaves the other calls as they are.  dblast_stats_get() waits
+ * for the recorded events and returns the summed pass times (ms), the number
+ * of timed passes and the number of kernel launches issued by the library
+ * since the reset. */
 typedef struct {
   uint64_t calls;            /* draft/verify entry-point calls */
   uint64_t kernel_launches;  /* kernels launched by the library */

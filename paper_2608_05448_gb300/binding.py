@@ -344,7 +344,9 @@ def dblast_set_wait_limit(spins):
 
 
 def dblast_stats_reset(enable_pass_timing=True):
-    lib().dblast_stats_reset(int(bool(enable_pass_timing)))
+    """Zero the counters; time every n-th pass with CUDA events (True = 1,
+    False = 0 = off)."""
+    lib().dblast_stats_reset(int(enable_pass_timing))
 
 
 def dblast_stats_get():

@@ -20,10 +20,16 @@ uint32_t wait_limit() { return g_wait_limit; }
 // ------------------------------------------------------------ measurement
 static std::mutex g_stats_mu;
 static std::atomic<uint64_t> g_launches{0}, g_calls{0}, g_tc_launches{0};
-static bool g_timing = false;
+// Per-pass timing: CUDA events around every g_period-th draft pass and
+// verify pass (0: off).  An event between two kernels keeps the later one
+// from being scheduled while the earlier one finishes, so a period above 1
+// leaves most passes undisturbed.
+static int g_period = 0;
 constexpr int kMaxTimed = 4096;
 static std::vector<cudaEvent_t> g_ev[2];  // pairs (begin, end) per timed call
 static int g_n_ev[2] = {0, 0};
+static uint64_t g_seen[2] = {0, 0};       // passes seen since the reset
+static bool g_open[2] = {false, false};   // a begin event awaits its end
 
 void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 void count_tc_launch() { g_tc_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -71,19 +77,19 @@ static cudaEvent_t pool_event(int which, int idx) {
 
 void pass_event_begin(int which, cudaStream_t s) {
   std::lock_guard<std::mutex> lk(g_stats_mu);
-  if (!g_timing || g_n_ev[which] >= kMaxTimed) return;
+  g_open[which] = false;
+  if (g_period <= 0 || g_n_ev[which] >= kMaxTimed) return;
+  if (g_seen[which]++ % (uint64_t)g_period != 0) return;
   cudaEvent_t e = pool_event(which, 2 * g_n_ev[which]);
-  if (e) cudaEventRecord(e, s);
+  g_open[which] = e && cudaEventRecord(e, s) == cudaSuccess;
 }
 
 void pass_event_end(int which, cudaStream_t s) {
   std::lock_guard<std::mutex> lk(g_stats_mu);
-  if (!g_timing || g_n_ev[which] >= kMaxTimed) return;
+  if (!g_open[which]) return;
+  g_open[which] = false;
   cudaEvent_t e = pool_event(which, 2 * g_n_ev[which] + 1);
-  if (e) {
-    cudaEventRecord(e, s);
-    ++g_n_ev[which];
-  }
+  if (e && cudaEventRecord(e, s) == cudaSuccess) ++g_n_ev[which];
 }
 
 PrepLayout prep_layout(int V, int H, int K, int r, bool has_e) {
@@ -521,7 +527,9 @@ void dblast_stats_reset(int enable_pass_timing) {
   g_calls = 0;
   g_tc_launches = 0;
   g_n_ev[0] = g_n_ev[1] = 0;
-  g_timing = enable_pass_timing != 0;
+  g_seen[0] = g_seen[1] = 0;
+  g_open[0] = g_open[1] = false;
+  g_period = enable_pass_timing > 0 ? enable_pass_timing : 0;
 }
 
 dblast_status dblast_stats_get(dblast_stats* out) {

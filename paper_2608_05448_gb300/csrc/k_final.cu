@@ -60,8 +60,7 @@ template <int NT> __device__ BlockScan block_scan_ff(FF v, FF* sh) {
 }
 
 template <int NT> __device__ int block_min_i(int v, int* sh) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(FULLMASK, v, o));
+  v = __reduce_min_sync(FULLMASK, v);
   if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
   __syncthreads();
   int r = sh[0];
@@ -978,41 +977,32 @@ __global__ void __launch_bounds__(VFS_NT, 1)
     const bool anear = lane < B && lane <= L && amargin < (TIE_TOL + NEAR_ACCEPT) * qtok;
     if (__ballot_sync(FULLMASK, atie)) ties |= TIE_ACCEPT;
     if (__ballot_sync(FULLMASK, anear)) ties |= TIE_ACCEPT << NEAR_SHIFT;
-    // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha (products in lane order)
-    // App. B: collision probabilities of the block's target rows and
-    // D_B = (1/B) sum_j prod_{i<=j} coll_i (rows independent of the prefix)
-    float cA = (lane < B) ? A : 1.f, cAl = (lane < B) ? alpha : 1.f;
-    if (lane >= B) cC = 1.f;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float ta = __shfl_up_sync(FULLMASK, cA, o);
-      const float tl = __shfl_up_sync(FULLMASK, cAl, o);
-      const float tc = __shfl_up_sync(FULLMASK, cC, o);
-      if (lane >= o) {
-        cA *= ta;
-        cAl *= tl;
-        cC *= tc;
-      }
-    }
-    FF el{lane < B ? cA : 0.f, 0.f}, ea{lane < B ? cAl : 0.f, 0.f};
-    FF ed{lane < B ? cC : 0.f, 0.f};
-    FF R{0.f, 0.f};
-    if (L < B && lane == 0) R = rowR[L];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      R = ff_add(R, ff_shfl_xor(R, o));
-      el = ff_add(el, ff_shfl_xor(el, o));
-      ea = ff_add(ea, ff_shfl_xor(ea, o));
-      ed = ff_add(ed, ff_shfl_xor(ed, o));
-    }
+    // E[L|x] = sum_i prod_{j<=i} A_j and the same over alpha; App. B: the
+    // collision probabilities of the block's target rows and D_B = (1/B)
+    // sum_j prod_{i<=j} coll_i (rows independent of the prefix).  Lane 0
+    // forms the products and sums in position order from shared memory:
+    // here that is much faster than shuffle scans of float pairs.
+    sacc[0][lane] = A;
+    sacc[1][lane] = alpha;
     if (L < B && lane < K) sC[lane] = sCall[L * K + lane];  // normalisers of the rejected row
+    __syncwarp();
     if (lane == 0) {
+      float pA = 1.f, pAl = 1.f, pC = 1.f;
+      FF el{0.f, 0.f}, ea{0.f, 0.f}, ed{0.f, 0.f};
+      for (int i = 0; i < B; ++i) {
+        pA *= sacc[0][i];
+        pAl *= sacc[1][i];
+        pC *= sacc[3][i];
+        el = ff_addf(el, pA);
+        ea = ff_addf(ea, pAl);
+        ed = ff_addf(ed, pC);
+      }
       if (out.exp_len) out.exp_len[n] = ff_f(el);
       if (out.alpha_len) out.alpha_len[n] = ff_f(ea);
       if (out.determinism) out.determinism[n] = ff_f(ed) / (float)B;
       sL = L;
       sties = ties;
-      sR = R;
+      sR = (L < B) ? rowR[L] : FF{0.f, 0.f};
     }
   }
   __syncthreads();
