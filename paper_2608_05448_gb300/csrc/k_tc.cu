@@ -331,7 +331,8 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
 // component has been taken before starting tile t+1.  12 warps: warp 0 issues TMA, warp
 // 1 issues MMAs and owns TMEM, warps 4-11 are the epilogue (two per TMEM lane
 // quarter, 128 columns each).  Warpgroup 0 gives registers to the epilogue
-// warpgroups with setmaxnreg (56 + 2 x 224 = 3 x 168 per thread).
+// warpgroups with setmaxnreg (56 + 2 x 224 = 3 x 168 per thread; 64 + 2 x 216
+// when warps 2-3 also run the target statistics).
 //
 // The pair form (PAIR = true) runs the same roles on a cluster of two CTAs
 // with cta_group::2 MMAs of 256 x 256: each SM stages its own 128 rows of A
@@ -346,6 +347,10 @@ constexpr int DCOLS = DBN / 2;               // columns per epilogue thread
 constexpr int D_THREADS = 384;
 constexpr int DREG = 168, DREG_LO = 56, DREG_HI = 224;
 static_assert(4 * DREG_LO + 8 * DREG_HI == 12 * DREG, "register split must equal the launch pool");
+// with the target statistics on warps 2-3 the first warpgroup needs 64
+// registers (56 spilled in its stage loops); the epilogue fits in 216
+constexpr int DREG_LO_TS = 64, DREG_HI_TS = 216;
+static_assert(4 * DREG_LO_TS + 8 * DREG_HI_TS <= 12 * DREG, "register split must fit the launch pool");
 constexpr int D_EPI = 256;                   // epilogue threads
 constexpr int DAZ_BYTES = KMAX * D_EPI * 4;  // per-thread branch scales
 constexpr int DVB_BYTES = 2 * DBN * 4;       // vocabulary bias of two tiles
@@ -1147,11 +1152,11 @@ __global__ void __launch_bounds__(D_THREADS, 1)
   griddep_wait();  // the set-up above overlaps the end of the previous kernel
 
   if (warp >= 4) {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(DREG_HI));
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(TS ? DREG_HI_TS : DREG_HI));
     draft_epilogue<PAIR, GREEDY>(P, tmem, warp, lane, az, vbs, vbar, bfull, bempty, cfull, cempty, ctl,
                          my_tiles);
   } else {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(DREG_LO));
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(TS ? DREG_LO_TS : DREG_LO));
     if (warp == 0 && lane == 0)
       draft_producer<PAIR>(P, S, &tm_a, &tm_b, &tm_ca, &tm_cb, stages, full, empty, ctl, my_tiles);
     else if (warp == 1 && lane == 0 && (!PAIR || S.rank == 0))
