@@ -315,7 +315,6 @@ static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   g_calls.fetch_add(1, std::memory_order_relaxed);
   cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
                                   c.stream);
-  if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
   if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
@@ -394,10 +393,10 @@ static cudaError_t side_stream(SideStream** out) {
   return cudaSuccess;
 }
 
-// draft and verify of one block.  The category prior runs beside the codes
-// GEMM on the library's second stream; the target statistics run inside the
-// draft pass (bf16 targets with 16-byte rows), else on the second stream
-// beside the draft finalize kernels, where the target filter also runs.
+// draft and verify of one block.  The category prior runs in the launch that
+// reduces the codes; the target statistics run inside the draft pass (bf16
+// targets with 16-byte rows), else on the library's second stream beside the
+// draft finalize kernels, where the target filter also runs.
 static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_out* vout) {
   if (debug_sync()) {  // serial order, so a failing launcher is named
     dblast_status st = draft_impl(c, dout);
@@ -421,20 +420,16 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   if (e == cudaSuccess) side.stream = ss->s;
   if (e == cudaSuccess)
     e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t), c.stream);
-  // fork 1: prior | codes
-  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[0], c.stream);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(side.stream, ss->ev[0], 0);
-  if (e == cudaSuccess) e = launch_prior(side);
-  if (e == cudaSuccess) e = cudaEventRecord(ss->ev[1], side.stream);
+  // the codes GEMM, then the codes reduction and the category prior in one
+  // launch, then the draft pass
   if (e == cudaSuccess) e = launch_codes(c);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
     e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
     pass_event_end(0, c.stream);
   }
-  // join 1, fork 2: target statistics (unless the draft pass took them) and
-  // the target filter | draft finalize
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, ss->ev[1], 0);
+  // fork: target statistics (unless the draft pass took them) and the target
+  // filter | draft finalize
   const bool side_work = !c.fuse_tstats || filter_on(c.head, vout);
   if (side_work) {
     if (e == cudaSuccess) e = cudaEventRecord(ss->ev[2], c.stream);
@@ -455,7 +450,7 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   }
   if (e == cudaSuccess)
     e = c.greedy ? launch_greedy_draft_finalize(c, dout) : launch_draft_finalize(c, dout);
-  // join 2
+  // join
   if (e == cudaSuccess && side_work) e = cudaStreamWaitEvent(c.stream, ss->ev[3], 0);
   if (e == cudaSuccess) e = verify_passes(c, vout);
   return cuda_status(e);
@@ -579,7 +574,6 @@ dblast_status dblast_al_objective(const dblast_head* h, const dblast_block_args*
   g_calls.fetch_add(1, std::memory_order_relaxed);
   cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
                                   c.stream);
-  if (e == cudaSuccess) e = dbg(launch_prior(c), "prior", c.stream);
   if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
   if (e == cudaSuccess)
     e = dbg(c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c), "draft_pass", c.stream);

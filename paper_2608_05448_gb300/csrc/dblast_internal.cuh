@@ -312,7 +312,6 @@ cudaError_t launch_prep(const dblast_head* head, const PrepLayout& pl, cudaStrea
 cudaError_t launch_prep_tc(const dblast_head* head, const PrepLayout& pl, cudaStream_t s);
 cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit);
 bool tc_supported(const dblast_head* h);
-cudaError_t launch_prior(const StepCtx& c);
 cudaError_t launch_codes(const StepCtx& c);
 cudaError_t launch_draft_pass_simt(const StepCtx& c);
 cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* out,

@@ -165,19 +165,23 @@ cudaError_t launch_prep(const dblast_head* h, const PrepLayout& pl, cudaStream_t
   return h->dtype == DBLAST_F32 ? prep_typed<float>(h, pl, s) : prep_typed<__nv_bfloat16>(h, pl, s);
 }
 
-// ------------------------------------------------------------- prior
-// One CTA per sequence: l = Wp a + bp (a warp per category, 16-byte loads),
-// then warp 0 with lane z: pi = softmax(l / Z_T) (Z_T = 0: one-hot argmax,
-// lowest index on ties) and z-hat by an inverse-CDF draw (stream 0).
+// ------------------------------------------------------------- prior and codes
+// Prior of sequence n, run by one block of 256 threads: l = Wp a + bp (a warp
+// per category, 16-byte loads), then warp 0 with lane z: pi = softmax(l / Z_T)
+// (Z_T = 0: one-hot argmax, lowest index on ties) and z-hat by an inverse-CDF
+// draw (stream 0).
 template <typename Tin>
-__global__ void __launch_bounds__(256)
-    k_prior(const Tin* __restrict__ Wp, const float* __restrict__ bp,
-            const Tin* __restrict__ anchor, const Tin* __restrict__ hidden, int H, int K, int B,
-            float zt, uint64_t seed, const int64_t* __restrict__ pos,
-            const uint32_t* __restrict__ rnd, int32_t* __restrict__ zhat_ws,
-            float* __restrict__ log2pi_ws, uint32_t* __restrict__ ties) {
-  __shared__ float ell[32];
-  const int n = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+__device__ __forceinline__ void prior_body(int n, const Tin* __restrict__ Wp,
+                                           const float* __restrict__ bp,
+                                           const Tin* __restrict__ anchor,
+                                           const Tin* __restrict__ hidden, int H, int K, int B,
+                                           float zt, uint64_t seed,
+                                           const int64_t* __restrict__ pos,
+                                           const uint32_t* __restrict__ rnd,
+                                           int32_t* __restrict__ zhat_ws,
+                                           float* __restrict__ log2pi_ws,
+                                           uint32_t* __restrict__ ties, float* ell) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const Tin* a = anchor ? anchor + (size_t)n * H : hidden + (size_t)n * B * H;
   for (int z = warp; z < K; z += blockDim.x >> 5) {
     const Tin* w = Wp + (size_t)z * H;
@@ -247,13 +251,15 @@ __global__ void __launch_bounds__(256)
   if (on) log2pi_ws[n * K + lane] = pz > 0.f ? log2f(pz) : -INFINITY;
 }
 
-// Deterministic split-K reduction of the codes, the constant code for e, the
-// per-(m, z) power-of-two scale and the split-fp16 operand rows.  One warp per (m, z).
-__global__ void k_codes_finish(const float* __restrict__ part, int nsplit, int M, int Mpad, int K,
-                               int r, int rr, int rp, bool has_e, float* __restrict__ codes,
-                               float* __restrict__ cscale, __half* __restrict__ cop) {
-  griddep_wait();  // launched as a dependent of the codes GEMM
-  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+// Deterministic split-K reduction of the codes of one (m, z) by one warp, the
+// constant code for e, the per-(m, z) power-of-two scale and the split-fp16
+// operand rows.
+__device__ __forceinline__ void codes_finish_warp(int gw, int lane, const float* __restrict__ part,
+                                                  int nsplit, int M, int Mpad, int K, int r,
+                                                  int rr, int rp, bool has_e,
+                                                  float* __restrict__ codes,
+                                                  float* __restrict__ cscale,
+                                                  __half* __restrict__ cop) {
   if (gw >= Mpad * K) return;
   const int m = gw / K, z = gw - m * K;
   const int Nb = K * rr;
@@ -290,19 +296,41 @@ __global__ void k_codes_finish(const float* __restrict__ part, int nsplit, int M
   }
 }
 
-template <typename Tin> static cudaError_t prior_typed(const StepCtx& c) {
-  const dblast_head* h = c.head;
-  const dblast_block_args* a = c.args;
-  const WsLayout& w = c.wl;
-  cudaStream_t s = c.stream;
-  k_prior<Tin><<<a->N, 256, 0, s>>>(
-      static_cast<const Tin*>(h->Wp), h->bp, static_cast<const Tin*>(a->anchor),
-      static_cast<const Tin*>(a->hidden), h->H, h->K, a->B, a->z_temperature, a->seed, a->pos,
-      a->round, wsp<int32_t>(c, w.off_zhat), wsp<float>(c, w.off_log2pi),
-      wsp<uint32_t>(c, w.off_ties));
-  debug_kernel("k_prior", s);
-  count_launches(1);
-  return cudaGetLastError();
+// One launch after the codes GEMM: blocks [0, nfin) reduce the codes (a warp
+// per (m, z)), blocks nfin + n compute the prior of sequence n.  The prior
+// reads the positions and round counters that the previous step's
+// verify-final kernel wrote, so it too waits for the preceding grids.
+struct PriorArgs {
+  const void* Wp;
+  const float* bp;
+  const void* anchor;
+  const void* hidden;
+  int H, K, B;
+  float zt;
+  uint64_t seed;
+  const int64_t* pos;
+  const uint32_t* rnd;
+  int32_t* zhat;
+  float* log2pi;
+  uint32_t* ties;
+};
+template <typename Tin>
+__global__ void __launch_bounds__(256)
+    k_codes_prior(const float* __restrict__ part, int nsplit, int M, int Mpad, int K, int r,
+                  int rr, int rp, bool has_e, float* __restrict__ codes,
+                  float* __restrict__ cscale, __half* __restrict__ cop, int nfin,
+                  const PriorArgs pa) {
+  griddep_wait();  // launched as a dependent of the codes GEMM
+  __shared__ float ell[32];
+  if ((int)blockIdx.x < nfin) {
+    const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    codes_finish_warp(gw, threadIdx.x & 31, part, nsplit, M, Mpad, K, r, rr, rp, has_e, codes,
+                      cscale, cop);
+    return;
+  }
+  prior_body<Tin>((int)blockIdx.x - nfin, static_cast<const Tin*>(pa.Wp), pa.bp,
+                  static_cast<const Tin*>(pa.anchor), static_cast<const Tin*>(pa.hidden), pa.H,
+                  pa.K, pa.B, pa.zt, pa.seed, pa.pos, pa.rnd, pa.zhat, pa.log2pi, pa.ties, ell);
 }
 
 template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
@@ -330,17 +358,17 @@ template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
     nsplit = (int)grid.z;
   }
   const int warps = w.Mpad * h->K;
+  const int nfin = ceil_div(warps * 32, 256);
+  const PriorArgs pa{h->Wp, h->bp, a->anchor, a->hidden, h->H, h->K, a->B, a->z_temperature,
+                     a->seed, a->pos, a->round, wsp<int32_t>(c, w.off_zhat),
+                     wsp<float>(c, w.off_log2pi), wsp<uint32_t>(c, w.off_ties)};
   cudaError_t le = launch_dep(
-      k_codes_finish, dim3(ceil_div(warps * 32, 256)), dim3(256), 0, s, part, nsplit, w.M, w.Mpad,
-      h->K, h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes), wsp<float>(c, w.off_cscale),
-      wsp<__half>(c, w.off_cop));
-  debug_kernel("k_codes_finish", s);
+      k_codes_prior<Tin>, dim3(nfin + a->N), dim3(256), 0, s, part, nsplit, w.M, w.Mpad, h->K,
+      h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes), wsp<float>(c, w.off_cscale),
+      wsp<__half>(c, w.off_cop), nfin, pa);
+  debug_kernel("k_codes_prior", s);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
-}
-
-cudaError_t launch_prior(const StepCtx& c) {
-  return c.head->dtype == DBLAST_F32 ? prior_typed<float>(c) : prior_typed<__nv_bfloat16>(c);
 }
 
 cudaError_t launch_codes(const StepCtx& c) {
