@@ -332,6 +332,7 @@ __device__ __forceinline__ void em_prepare(const ResidualTokenMass<Tin>& e, int 
 // lane = row, warps and splits interleave over the tiles.
 // lsep[sp][m][z] = (max, sum.hi, sum.lo, 0) with sum * 2^max the partial mass.
 constexpr int LSE_WARPS = 16;
+constexpr int LSE_BATCH = 20;  // records in flight per thread (1187 tiles: one batch)
 __global__ void __launch_bounds__(LSE_WARPS * 32)
     k_draft_lse(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
                 float4* __restrict__ lsep) {
@@ -343,28 +344,31 @@ __global__ void __launch_bounds__(LSE_WARPS * 32)
   const int step = LSE_WARPS * LSE_SPLIT;
   float mx = -INFINITY;
   FF s{0.f, 0.f};
-  auto merge = [&](float2 q) {
-    if (q.y > 0.f) {
-      if (q.x > mx) {
-        s = ff_mulf(s, exp2f(mx - q.x));
-        mx = q.x;
-      }
-      s = ff_addf(s, q.y * exp2f(q.x - mx));
-    }
-  };
   if (m < M) {
+    // batches of LSE_BATCH records, all loaded before any is used (one
+    // memory round trip per batch); the batch's maximum, then its sum
+    // against the running maximum
     const float2* p = partd + (size_t)z * Mpad + m;
     const size_t st = (size_t)K * Mpad;
-    int t = sp * LSE_WARPS + warp;
-    for (; t + 3 * step < nt; t += 4 * step) {
-      const float2 q0 = p[(size_t)t * st], q1 = p[(size_t)(t + step) * st];
-      const float2 q2 = p[(size_t)(t + 2 * step) * st], q3 = p[(size_t)(t + 3 * step) * st];
-      merge(q0);
-      merge(q1);
-      merge(q2);
-      merge(q3);
+    for (int t0 = sp * LSE_WARPS + warp; t0 < nt; t0 += LSE_BATCH * step) {
+      float2 q[LSE_BATCH];
+#pragma unroll
+      for (int j = 0; j < LSE_BATCH; ++j) {
+        const int t = t0 + j * step;
+        q[j] = t < nt ? p[(size_t)t * st] : make_float2(-INFINITY, 0.f);
+      }
+      float bm = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < LSE_BATCH; ++j)
+        if (q[j].y > 0.f) bm = fmaxf(bm, q[j].x);
+      if (bm > mx) {
+        if (mx != -INFINITY) s = ff_mulf(s, exp2f(mx - bm));
+        mx = bm;
+      }
+#pragma unroll
+      for (int j = 0; j < LSE_BATCH; ++j)
+        if (q[j].y > 0.f) s = ff_addf(s, q[j].y * exp2f(q[j].x - mx));
     }
-    for (; t < nt; t += step) merge(p[(size_t)t * st]);
   }
   smx[warp][lane] = mx;
   ssum[warp][lane] = s;
@@ -920,16 +924,16 @@ __global__ void __launch_bounds__(VFS_NT, 1)
     if (t32 < S * B) {
       const int i = t32 % B, s0 = t32 / B;
       const float2* pv = partv + (size_t)n * B + i;
-      // eight records in flight per thread
-      for (int t = s0; t < nt; t += 8 * S) {
-        float2 q[8];
+      // 24 records in flight per thread
+      for (int t = s0; t < nt; t += 24 * S) {
+        float2 q[24];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 24; ++j) {
           const int tj = t + j * S;
           q[j] = tj < nt ? pv[(size_t)tj * Mpad] : make_float2(0.f, 0.f);
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 24; ++j) {
           a = ff_addf(a, q[j].x);
           r = ff_addf(r, q[j].y);
         }

@@ -124,19 +124,6 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
 }
 
 // copies of data read once (evict-first L2 policy)
-// An fp32 pair stored with the L2 evict-last policy: per-tile records that
-// the finalize kernels read right after the pass, kept in L2 while the pass
-// streams the head (and the stash) through it.
-__device__ __forceinline__ uint64_t l2_evict_last() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-__device__ __forceinline__ void st_keep(float2* p, float2 v, uint64_t pol) {
-  asm volatile("st.global.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p), "f"(v.x), "f"(v.y),
-               "l"(pol)
-               : "memory");
-}
 __device__ __forceinline__ uint64_t l2_evict_first() {
   uint64_t pol;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
@@ -888,7 +875,6 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     for (int j = 0; j < DCOLS; ++j) bk[j] = (v0 + j < P.V) ? fmaf(bk[j], P.k2, -ref) : -INFINITY;
 
     const int rec = vt * 2 + half;
-    const uint64_t keep = l2_evict_last();
     bool ok = true;
     for (int z = 0; z < P.K; ++z) {
       if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6)) {
@@ -952,7 +938,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
         if constexpr (PAIR) mbar_arrive_taken_cluster(cluster_addr(&cempty[rg], 0));
         else mbar_arrive_taken(&cempty[rg]);
       }
-      if (live) st_keep(P.partd + ((size_t)rec * P.K + z) * P.Mpad + m, make_float2(rz, sum), keep);
+      if (live) P.partd[((size_t)rec * P.K + z) * P.Mpad + m] = make_float2(rz, sum);
     }
     if (!ok) break;
   }
@@ -1427,9 +1413,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 16)) break;
       if (cq == 0) {
         const float2 o1 = red[BM + row], o2 = red[2 * BM + row], o3 = red[3 * BM + row];
-        st_keep(P.partv + (size_t)vt * P.Mpad + m,
-                make_float2((As + o1.x) + (o2.x + o3.x), (Rs + o1.y) + (o2.y + o3.y)),
-                l2_evict_last());
+        P.partv[(size_t)vt * P.Mpad + m] =
+            make_float2((As + o1.x) + (o2.x + o3.x), (Rs + o1.y) + (o2.y + o3.y));
       }
       mbar_arrive(redm);
     }
