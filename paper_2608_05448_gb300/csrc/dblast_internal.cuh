@@ -75,7 +75,7 @@ struct PrepLayout {
 //   coll f32 [Rt]  (collision probability sum_v p(v)^2 of every target row)
 //   ftok i32 [Rt, FILTER_MAX_K] | fp f32 [Rt, FILTER_MAX_K] | fcnt i32 [Rt] | ftie u32 [Rt]
 //   (target filter: kept tokens by index, their filtered probabilities, count, top-p tie)
-constexpr int LSE_SPLIT = 4;  // partial merges of the draft records per (m, z)
+constexpr int LSE_SPLIT = 2;  // partial merges of the draft records per (m, z) (one wave of blocks)
 struct WsLayout {
   int N, B, M, Mpad, K, rr, rp, KC, V, nt, Rt;
   size_t off_status, off_codes, off_cscale, off_cop, off_zhat, off_log2pi, off_stash,

@@ -332,7 +332,7 @@ __device__ __forceinline__ void em_prepare(const ResidualTokenMass<Tin>& e, int 
 // lane = row, warps and splits interleave over the tiles.
 // lsep[sp][m][z] = (max, sum.hi, sum.lo, 0) with sum * 2^max the partial mass.
 constexpr int LSE_WARPS = 16;
-constexpr int LSE_BATCH = 20;  // records in flight per thread (1187 tiles: one batch)
+constexpr int LSE_BATCH = 19;  // records in flight per thread (1187 tiles: two batches)
 __global__ void __launch_bounds__(LSE_WARPS * 32)
     k_draft_lse(const float2* __restrict__ partd, int nt, int K, int M, int Mpad,
                 float4* __restrict__ lsep) {
