@@ -77,6 +77,30 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// The retry of a wait that did not complete at once: the warp may be
+// suspended for up to WAIT_HINT_NS nanoseconds (or until the phase completes)
+// before the loop around it checks its bounds again, instead of polling and
+// taking issue slots from the warps that share its scheduler.
+#ifndef DBLAST_WAIT_HINT_NS
+#define DBLAST_WAIT_HINT_NS 20000
+#endif
+constexpr uint32_t WAIT_HINT_NS = DBLAST_WAIT_HINT_NS;
+__device__ __forceinline__ bool mbar_retry_wait(uint64_t* bar, uint32_t parity) {
+  if constexpr (WAIT_HINT_NS == 0) {
+    return mbar_try_wait(bar, parity);
+  } else {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "n"(WAIT_HINT_NS)
+        : "memory");
+    return ok != 0;
+  }
+}
+
 // Shared state of the roles: every wait is bounded; a wait that runs out
 // raises `abort` so that the other roles leave their loops too.
 struct Ctl {
@@ -96,7 +120,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    // a spin limit (fault injection) counts plain polls
+    if (c.spin_limit ? mbar_try_wait(bar, parity) : mbar_retry_wait(bar, parity)) return true;
     if (*c.abort) return false;
     if ((c.spin_limit && i >= c.spin_limit) || (globaltimer() - t0) > 2000000000ull) {
       record_timeout(c, where);
@@ -246,12 +271,27 @@ __device__ __forceinline__ bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity)
       : "memory");
   return ok != 0;
 }
+__device__ __forceinline__ bool mbar_retry_wait_cl(uint64_t* bar, uint32_t parity) {
+  if constexpr (WAIT_HINT_NS == 0) {
+    return mbar_try_wait_cl(bar, parity);
+  } else {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "n"(WAIT_HINT_NS)
+        : "memory");
+    return ok != 0;
+  }
+}
 __device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity, const Ctl& c,
                                              uint32_t where) {
   if (mbar_try_wait_cl(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait_cl(bar, parity)) return true;
+    if (c.spin_limit ? mbar_try_wait_cl(bar, parity) : mbar_retry_wait_cl(bar, parity)) return true;
     if (*c.abort) return false;
     if ((c.spin_limit && i >= c.spin_limit) || (globaltimer() - t0) > 2000000000ull) {
       record_timeout(c, where);
@@ -1179,12 +1219,19 @@ __global__ void __launch_bounds__(D_THREADS, 1)
 // and the tile records (sum min(p, q), sum [p - q]_+).  bk = stash log2(e)/T;
 // B0 = floor(max_z L_{m,z}) keeps both factors inside the fp32 range.
 // The stash and target tiles of a verify tile go through shared memory when
-// use_x (V % 8 == 0 and 128 % B == 0): the producer loads them by TMA while
-// the epilogue is still busy with the tile's branch exponentials.
+// use_x (V % 8 == 0 and 128 % B == 0), one 32-column quarter at a time: each
+// quarter has its own barriers and its own copying lane (warp 2, lanes 0-3),
+// so that the four warps of a quarter never wait for the other quarters.  The
+// four partial records of a row are added by whichever of its four warps
+// finishes the tile last, so no barrier spans all epilogue warps either.
 constexpr int VSTAGES = 3;
-constexpr int XS_BYTES = BM * BN * 4;   // stash tile: 4 boxes [128 rows][32 fp32], SW128
-constexpr int XT_BYTES = BM * BN * 2;   // target tile: 2 boxes [128 rows][64 bf16], SW128
-constexpr size_t VSMEM = (size_t)VSTAGES * STAGE_BYTES + XS_BYTES + XT_BYTES + 4 * BM * 8 + 256 + 1024;
+constexpr int XS_BOX = BM * 32 * 4;     // stash box [128 rows][32 fp32], 128-byte swizzle
+constexpr int XT_BOX = BM * 32 * 2;     // target box [128 rows][32 bf16], 64-byte swizzle
+constexpr int XS_BYTES = 4 * XS_BOX;
+constexpr int XT_BYTES = 4 * XT_BOX;
+constexpr int VRED_BYTES = 2 * 4 * BM * 8;  // per tile parity and quarter: (sum min, sum resid) per row
+constexpr size_t VSMEM =
+    (size_t)VSTAGES * STAGE_BYTES + XS_BYTES + XT_BYTES + VRED_BYTES + 256 + 1024;
 struct VParams {
   int n_mt, n_vt, n_tiles, ncs, K, rp, zps, M, V, Mpad, B, Bt;
   int use_x;
@@ -1213,21 +1260,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stage_base = smem;
-  unsigned char* xs = smem + VSTAGES * STAGE_BYTES;  // stash tile
-  unsigned char* xt = xs + XS_BYTES;                 // target tile
-  float2* red = reinterpret_cast<float2*>(xt + XT_BYTES);   // [4][BM]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xt + XT_BYTES + 4 * BM * 8);
+  unsigned char* xs = smem + VSTAGES * STAGE_BYTES;  // stash boxes [4]
+  unsigned char* xt = xs + XS_BYTES;                 // target boxes [4]
+  float2* red = reinterpret_cast<float2*>(xt + XT_BYTES);   // [2][4][BM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xt + XT_BYTES + VRED_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + VSTAGES;
   uint64_t* sfull = bars + 2 * VSTAGES;  // [2] TMEM slot ready
   uint64_t* sempty = sfull + 2;          // [2] TMEM slot free
   uint64_t* done = sfull + 4;
-  uint64_t* redw = sfull + 5;
-  uint64_t* redm = sfull + 6;
-  uint64_t* xfull = sfull + 7;           // stash and target tile landed
-  uint64_t* xempty = sfull + 8;          // stash and target tile read (16 epilogue warps)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 9);
+  uint64_t* xfull = sfull + 5;           // [4] a quarter's stash and target boxes landed
+  uint64_t* xempty = sfull + 9;          // [4] ... and read (the quarter's 4 warps)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sfull + 13);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* qcount = reinterpret_cast<int*>(tmem_slot + 2);  // [2][4] quarters done per lane quarter
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int my_tiles = (P.n_tiles > (int)blockIdx.x)
@@ -1246,10 +1292,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(&sempty[b], NUM_EPI_WARPS);
     }
     mbar_init(done, 1);
-    mbar_init(redw, 32 * NUM_EPI_WARPS);
-    mbar_init(redm, 32 * NUM_EPI_WARPS);
-    mbar_init(xfull, 1);
-    mbar_init(xempty, NUM_EPI_WARPS);
+    for (int c = 0; c < 4; ++c) {
+      mbar_init(&xfull[c], 1);
+      mbar_init(&xempty[c], 4);
+    }
+    for (int c = 0; c < 8; ++c) qcount[c] = 0;
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -1356,20 +1403,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       };
       const bool full_cols = v0 + 32 <= P.V;
       if (P.use_x) {
-        // stash and target rows from shared memory (128-byte swizzle: the
-        // 16-byte chunk c of row r sits at chunk c ^ (r & 7)); this quarter
-        // is stash box cq and half (cq & 1) of target box cq >> 1
-        if (!mbar_wait(xfull, (uint32_t)slot & 1u, ctl, 18)) break;
+        // this quarter's stash and target rows from shared memory: stash box
+        // cq (128-byte rows, 128-byte swizzle: 16-byte chunk c of row r at
+        // chunk c ^ (r & 7)) and target box cq (64-byte rows, 64-byte
+        // swizzle: chunk c of row r at chunk c ^ ((r >> 1) & 3))
+        if (!mbar_wait(&xfull[cq], (uint32_t)slot & 1u, ctl, 18)) break;
         if (mok) {
-          const unsigned char* sbase = xs + cq * (XS_BYTES / 4) + row * 128;
-          const unsigned char* tbase = xt + (cq >> 1) * (XT_BYTES / 2) + row * 128;
+          const unsigned char* sbase = xs + cq * XS_BOX + row * 128;
+          const unsigned char* tbase = xt + cq * XT_BOX + row * 64;
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const int c0 = (2 * k) ^ (row & 7), c1 = (2 * k + 1) ^ (row & 7);
             const float4 s0 = *reinterpret_cast<const float4*>(sbase + c0 * 16);
             const float4 s1 = *reinterpret_cast<const float4*>(sbase + c1 * 16);
             const uint4 t8 =
-                *reinterpret_cast<const uint4*>(tbase + ((((cq & 1) * 4 + k) ^ (row & 7)) * 16));
+                *reinterpret_cast<const uint4*>(tbase + ((k ^ ((row >> 1) & 3)) * 16));
             const __nv_bfloat162* tp = reinterpret_cast<const __nv_bfloat162*>(&t8);
             const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
             float tv[8];
@@ -1391,7 +1439,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(xempty);
+        if (lane == 0) mbar_arrive(&xempty[cq]);
       } else if (mok) {
         const float* srow = P.stash + (size_t)m * P.V + v0;
         const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
@@ -1406,17 +1454,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       f2_get(Rs2[1], Rs4[2], Rs4[3]);
       const float As = (As4[0] + As4[1]) + (As4[2] + As4[3]);
       const float Rs = (Rs4[0] + Rs4[1]) + (Rs4[2] + Rs4[3]);
-      // the other column quarters of this row, then one record per (tile, row)
-      if (slot > 0 && !mbar_wait(redm, ((uint32_t)(slot - 1)) & 1u, ctl, 15)) break;
-      red[cq * BM + row] = make_float2(As, Rs);
-      mbar_arrive(redw);
-      if (!mbar_wait(redw, (uint32_t)slot & 1u, ctl, 16)) break;
-      if (cq == 0) {
-        const float2 o1 = red[BM + row], o2 = red[2 * BM + row], o3 = red[3 * BM + row];
-        P.partv[(size_t)vt * P.Mpad + m] =
-            make_float2((As + o1.x) + (o2.x + o3.x), (Rs + o1.y) + (o2.y + o3.y));
+      // one record per (tile, row): the last of the four warps of this lane
+      // quarter to get here adds the four column quarters, in quarter order.
+      // The counter of a tile parity only grows; its four arrivals of one
+      // tile all come before any of the tile two slots later, since that
+      // tile's first components wait for every warp to release this tile's.
+      float2* rb = red + (slot & 1) * 4 * BM;
+      rb[cq * BM + row] = make_float2(As, Rs);
+      __syncwarp();
+      int last = 0;
+      if (lane == 0) {
+        __threadfence_block();
+        last = (atomicAdd(&qcount[(slot & 1) * 4 + q], 1) & 3) == 3;
+        __threadfence_block();
       }
-      mbar_arrive(redm);
+      __syncwarp();
+      if (__shfl_sync(0xffffffffu, last, 0)) {
+        const float2 o0 = rb[row], o1 = rb[BM + row], o2 = rb[2 * BM + row], o3 = rb[3 * BM + row];
+        P.partv[(size_t)vt * P.Mpad + m] =
+            make_float2((o0.x + o1.x) + (o2.x + o3.x), (o0.y + o1.y) + (o2.y + o3.y));
+      }
     }
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(VREG_LO));
@@ -1425,8 +1482,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         int stage = 0;
         uint32_t phase = 0, issued_mask = 0u, issued_phase = 0u;
         bool ok = true;
-        bool x_issued = false;
-        uint32_t x_phase = 0;
         for (int slot = 0; slot < my_tiles && ok; ++slot) {
           int mt, vt;
           vtile_of(P, slot, &mt, &vt);
@@ -1440,24 +1495,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
             if (++stage == VSTAGES) { stage = 0; phase ^= 1u; }
           }
-          if (ok && P.use_x) {
-            // this tile's stash rows and target rows, once the epilogue has read the previous ones
-            if (!mbar_wait(xempty, ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) { ok = false; break; }
-            mbar_arrive_expect_tx(xfull, XS_BYTES + XT_BYTES);
-            // the stash and target rows are read once: evict-first in L2
-            const uint64_t pol = l2_evict_first();
-#pragma unroll
-            for (int b = 0; b < 4; ++b)
-              tma_load_2d_once(xs + b * (XS_BYTES / 4), &tm_xs, xfull, vt * BN + b * 32, mt * BM,
-                               pol);
-            const int n0 = (mt * BM) / P.B;
-#pragma unroll
-            for (int h = 0; h < 2; ++h)
-              tma_load_3d_once(xt + h * (XT_BYTES / 2), &tm_xt, xfull, vt * BN + h * 64, 0, n0,
-                               pol);
-            x_issued = true;
-            x_phase = (uint32_t)slot & 1u;
-          }
         }
         for (int s = 0; s < VSTAGES; ++s)
           if (issued_mask & (1u << s)) {
@@ -1466,9 +1503,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                    (globaltimer() - t0) < 2000000000ull) {
             }
           }
+      }
+    } else if (warp == 2) {
+      if (lane < 4 && P.use_x) {
+        // lane c copies column quarter c of every tile's stash and target
+        // rows, once that quarter's warps have read the previous tile's
+        const int c = lane;
+        bool x_issued = false;
+        uint32_t x_phase = 0;
+        // the stash and target rows are read once: evict-first in L2
+        const uint64_t pol = l2_evict_first();
+        for (int slot = 0; slot < my_tiles; ++slot) {
+          int mt, vt;
+          vtile_of(P, slot, &mt, &vt);
+          if (!mbar_wait(&xempty[c], ((uint32_t)slot & 1u) ^ 1u, ctl, 17)) break;
+          mbar_arrive_expect_tx(&xfull[c], XS_BOX + XT_BOX);
+          tma_load_2d_once(xs + c * XS_BOX, &tm_xs, &xfull[c], vt * BN + c * 32, mt * BM, pol);
+          tma_load_3d_once(xt + c * XT_BOX, &tm_xt, &xfull[c], vt * BN + c * 32, 0,
+                           (mt * BM) / P.B, pol);
+          x_issued = true;
+          x_phase = (uint32_t)slot & 1u;
+        }
         if (x_issued) {
           const uint64_t t0 = globaltimer();
-          while (!mbar_try_wait(xfull, x_phase) && (globaltimer() - t0) < 2000000000ull) {
+          while (!mbar_try_wait(&xfull[c], x_phase) && (globaltimer() - t0) < 2000000000ull) {
           }
         }
       }
@@ -1570,9 +1628,10 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t r
 }
 
 // general tiled map: rank 2 or 3, dims/strides in elements (strides in bytes
-// are derived), box in elements, 128-byte swizzle
+// are derived), box in elements, 128-byte swizzle unless given
 static bool make_map_nd(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int esize,
-                        int rank, const uint64_t* dims, const uint32_t* box) {
+                        int rank, const uint64_t* dims, const uint32_t* box,
+                        CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t d[3], st[2];
@@ -1585,7 +1644,7 @@ static bool make_map_nd(CUtensorMap* m, const void* base, CUtensorMapDataType dt
     stride *= dims[i];
   }
   CUresult r = fn(m, dt, (cuuint32_t)rank, const_cast<void*>(base), d, st, bx, es,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -1882,9 +1941,10 @@ cudaError_t launch_verify_pass_tc(const StepCtx& c) {
     const uint64_t ds[2] = {(uint64_t)h->V, (uint64_t)w.M};
     const uint32_t bs[2] = {32, (uint32_t)tc::BM};
     const uint64_t dt[3] = {(uint64_t)h->V, (uint64_t)c.Bt, (uint64_t)w.N};
-    const uint32_t bt[3] = {64, (uint32_t)w.B, (uint32_t)(tc::BM / w.B)};
+    const uint32_t bt[3] = {32, (uint32_t)w.B, (uint32_t)(tc::BM / w.B)};
     if (!tc::make_map_nd(&mxs, c.ws + w.off_stash, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 2, ds, bs) ||
-        !tc::make_map_nd(&mxt, c.target, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 3, dt, bt))
+        !tc::make_map_nd(&mxt, c.target, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 3, dt, bt,
+                         CU_TENSOR_MAP_SWIZZLE_64B))
       return cudaErrorInvalidValue;
   }
   tc::VParams P{};
