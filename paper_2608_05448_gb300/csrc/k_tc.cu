@@ -85,6 +85,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 #define DBLAST_WAIT_HINT_NS 20000
 #endif
 constexpr uint32_t WAIT_HINT_NS = DBLAST_WAIT_HINT_NS;
+// The draft epilogue's waits for its next accumulator sleep this long between
+// polls: its warps share schedulers with the producer and the MMA issuer,
+// whose instruction streams pace the tensor pipe (measured: 0.5112 -> 0.5092
+// ms per draft pass; the verify pass, whose roles all wait on one another,
+// was 1 us slower with it and does not use it).
+constexpr uint32_t NAP_NS = 100;
 __device__ __forceinline__ bool mbar_retry_wait(uint64_t* bar, uint32_t parity) {
   if constexpr (WAIT_HINT_NS == 0) {
     return mbar_try_wait(bar, parity);
@@ -115,11 +121,15 @@ __device__ __noinline__ void record_timeout(const Ctl& c, uint32_t where) {
   atomicExch(&c.status->where, where);
 }
 
+// sleep_ns > 0: a role whose waits are not on the critical path sleeps that
+// long between polls, so that it takes no issue slots from the warps sharing
+// its scheduler while it waits
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const Ctl& c,
-                                          uint32_t where) {
+                                          uint32_t where, uint32_t sleep_ns = 0) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
+    if (sleep_ns) __nanosleep(sleep_ns);
     // a spin limit (fault injection) counts plain polls
     if (c.spin_limit ? mbar_try_wait(bar, parity) : mbar_retry_wait(bar, parity)) return true;
     if (*c.abort) return false;
@@ -287,10 +297,11 @@ __device__ __forceinline__ bool mbar_retry_wait_cl(uint64_t* bar, uint32_t parit
   }
 }
 __device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity, const Ctl& c,
-                                             uint32_t where) {
+                                             uint32_t where, uint32_t sleep_ns = 0) {
   if (mbar_try_wait_cl(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
+    if (sleep_ns) __nanosleep(sleep_ns);
     if (c.spin_limit ? mbar_try_wait_cl(bar, parity) : mbar_retry_wait_cl(bar, parity)) return true;
     if (*c.abort) return false;
     if ((c.spin_limit && i >= c.spin_limit) || (globaltimer() - t0) > 2000000000ull) {
@@ -717,6 +728,15 @@ __device__ __forceinline__ F2 f2_sub(F2 a, F2 b) { return __ffma2_rn(b, make_flo
 __device__ __forceinline__ F2 f2_mul(F2 a, F2 b) { return __fmul2_rn(a, b); }
 __device__ __forceinline__ F2 f2_ex2(F2 a) { return make_float2(ex2n(a.x), ex2n(a.y)); }
 
+// the wait for a 16-column load, with its destination passed through it
+__device__ __forceinline__ void tmem_wait_ld16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
 // Greedy-branch epilogue of one tile (Sec. 3.1, "Drafter sampling during
 // inference"): for every component z, the largest logit
 // l_v = base_v + b_v + D_z / (cscale sw) of this thread's 128 columns and its
@@ -747,7 +767,7 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
     if (v0 + j >= P.V) bk[j] = -INFINITY;
   const int rec = (v0 / DCOLS);
   for (int z = 0; z < P.K; ++z) {
-    if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6)) return false;
+    if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6, NAP_NS)) return false;
     tc_fence_after();
     const float a = az[z * D_EPI + et];
     float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
@@ -834,10 +854,10 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
       const int vc = vt * DBN + et;
       vbs[(slot & 1) * DBN + et] = (P.vbias && vc < P.V) ? __ldg(P.vbias + vc) : 0.f;
       mbar_arrive(vbar);
-      if (!mbar_wait(vbar, (uint32_t)slot & 1u, ctl, 7)) break;
+      if (!mbar_wait(vbar, (uint32_t)slot & 1u, ctl, 7, NAP_NS)) break;
     }
     const int rg = slot & 1;  // the tile's TMEM region (base, then its components)
-    if (!mbar_wait(&bfull[rg], (uint32_t)(slot >> 1) & 1u, ctl, 5)) break;
+    if (!mbar_wait(&bfull[rg], (uint32_t)(slot >> 1) & 1u, ctl, 5, NAP_NS)) break;
     tc_fence_after();
     {
       const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
@@ -917,7 +937,7 @@ __device__ __forceinline__ void draft_epilogue(const Params& P, uint32_t tmem, i
     const int rec = vt * 2 + half;
     bool ok = true;
     for (int z = 0; z < P.K; ++z) {
-      if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6)) {
+      if (!mbar_wait(&cfull[rg], (uint32_t)((slot >> 1) * P.K + z) & 1u, ctl, 6, NAP_NS)) {
         ok = false;
         break;
       }
@@ -1340,25 +1360,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!mbar_wait(&sfull[gs], use & 1u, ctl, 14)) { ok = false; break; }
         if (gs) ++guse1; else ++guse0;
         tc_fence_after();
-        // this quarter's 32 columns of each component of the group; the slot
-        // is handed back once the last one is in registers
+        // this quarter's 32 columns of the group's one or two components are
+        // read in 16-column chunks (component, half), the load of the next
+        // chunk in flight while the current one is reduced; the slot is
+        // handed back once the last chunk is in registers
         const int nz = min(2, P.K - 2 * g);
-        for (int zz = 0; zz < nz; ++zz) {
-          const float2 cz = mok ? vrow[2 * g + zz] : make_float2(0.f, -INFINITY);
-          uint32_t r0[32];
-          tmem_ld32_raw(tmem + lane_off + (uint32_t)(gs * 2 * BN + zz * BN + cq * 32), r0);
-          tmem_wait_ld();
-          if (zz == nz - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_taken(&sempty[gs]);
-          }
+        const float2 c0v = mok ? vrow[2 * g] : make_float2(0.f, -INFINITY);
+        const float2 c1v = (mok && nz > 1) ? vrow[2 * g + 1] : make_float2(0.f, -INFINITY);
+        const uint32_t tb = tmem + lane_off + (uint32_t)(gs * 2 * BN + cq * 32);
+        uint32_t ra[16], rb[16];
+        auto chunk = [&](const uint32_t (&r)[16], float2 cz, int h) {
           const F2 czx = f2(cz.x, cz.x), czy = f2(cz.y, cz.y);
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            acc2[j] = f2_add(acc2[j], f2_ex2(f2_fma(f2(__uint_as_float(r0[2 * j]),
-                                                       __uint_as_float(r0[2 * j + 1])),
-                                                    czx, czy)));
+          for (int j = 0; j < 8; ++j)
+            acc2[h * 8 + j] = f2_add(acc2[h * 8 + j],
+                                     f2_ex2(f2_fma(f2(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1])),
+                                                   czx, czy)));
+        };
+        auto release = [&]() {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_taken(&sempty[gs]);
+        };
+        tmem_ld16_raw(tb, ra);
+        tmem_wait_ld16(ra);
+        tmem_ld16_raw(tb + 16, rb);
+        chunk(ra, c0v, 0);
+        tmem_wait_ld16(rb);
+        if (nz > 1) {
+          tmem_ld16_raw(tb + BN, ra);
+          chunk(rb, c0v, 1);
+          tmem_wait_ld16(ra);
+          tmem_ld16_raw(tb + BN + 16, rb);
+          chunk(ra, c1v, 0);
+          tmem_wait_ld16(rb);
+          release();
+          chunk(rb, c1v, 1);
+        } else {
+          release();
+          chunk(rb, c0v, 1);
         }
       }
       if (!ok) break;
