@@ -221,6 +221,18 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
   return d;
 }
 
+// the same for a 64-byte-swizzled operand (rows of 64 bytes, 8-row groups 512
+// bytes apart): the branch operands of one component, [hi | lo] of rank 16
+__device__ __forceinline__ uint64_t sdesc64(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(512 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;                 // 64-byte swizzle
+  return d;
+}
+
 // instruction descriptor, kind::f16: fp32 accumulate, A/B both bf16 or both
 // fp16, both K-major, M = m (128, or 256 for a CTA pair), N = n
 __host__ __device__ constexpr uint32_t idesc_f16(bool bf16, int n, int m = BM) {
@@ -399,6 +411,8 @@ struct DCfg {
   static constexpr int STAGE_B = BROWS * BK * 2;           // 16 or 32 KB
   static constexpr int STAGE = DSTAGE_A + STAGE_B;         // 32 or 48 KB
   static constexpr int TX = PAIR ? 2 * STAGE : STAGE;      // bytes completing one full barrier
+  // a branch item of rank 16: 64-byte rows of A (BM) and B (BROWS)
+  static constexpr int TX_NARROW = (PAIR ? 2 : 1) * (BM + BROWS) * 64;
   static constexpr size_t SMEM = (size_t)STAGES * STAGE + DAZ_BYTES + DVB_BYTES + 256 + 64 + 1024;
 };
 static_assert(DCfg<true>::SMEM <= 227 * 1024 && DCfg<false>::SMEM <= 227 * 1024, "shared memory");
@@ -495,11 +509,12 @@ __device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
   const int nzK = (P.mode != MODE_PREP) ? P.K : 0;
   // one stage: wait until the slot is free, arm its full barrier, copy the
   // A and B boxes
-  auto load = [&](const CUtensorMap* ma, const CUtensorMap* mb, int xk, int y0, int y1) {
+  auto load = [&](const CUtensorMap* ma, const CUtensorMap* mb, int xk, int y0, int y1,
+                  uint32_t tx) {
     if (!mbar_wait(&empty[stage], phase ^ 1u, ctl, 1)) return false;
     unsigned char* sa = stages + stage * C::STAGE;
     uint64_t* fb = &full[stage];
-    if (lead) mbar_arrive_expect_tx(fb, C::TX);
+    if (lead) mbar_arrive_expect_tx(fb, tx);
     if constexpr (PAIR) {
       const uint32_t fcl = full_cl + (uint32_t)(stage * 8);
       tma_load_2d_pair(sa, ma, fcl, xk, y0);
@@ -530,8 +545,12 @@ __device__ __forceinline__ void draft_producer(const Params& P, const Sched& S,
     for (int zd = 0; zd <= nzv && ok; ++zd) {
       const int jend = zd < nzv ? ins_point(zd, nbv, nzv) : nbv;
       for (; jb < jend; ++jb, kx += BK)
-        if (!(ok = load(tm_a, tm_b, kx, ya, yb))) break;
-      if (ok && zd < nzv) ok = load(tm_ca, tm_cb, (P.zps == 2 ? (zd >> 1) : zd) * BK, yca, ycb);
+        if (!(ok = load(tm_a, tm_b, kx, ya, yb, C::TX))) break;
+      // a branch item copies its own component: with rank 16 ([hi | lo], 32
+      // elements) a 64-byte-wide box, else the 64-wide block of the component
+      if (ok && zd < nzv)
+        ok = (P.zps == 2) ? load(tm_ca, tm_cb, zd * 32, yca, ycb, C::TX_NARROW)
+                          : load(tm_ca, tm_cb, zd * BK, yca, ycb, C::TX);
     }
   }
   // copies still in flight after an abort: wait (bounded) before leaving.  The
@@ -640,13 +659,21 @@ __device__ __forceinline__ void draft_mma(const Params& P, uint32_t tmem, unsign
       tc_fence_after();
       if (!(ok = mbar_wait(&full[stage], phase, ctl, 3))) break;
       tc_fence_after();
-      const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
-      const int o = (P.zps == 2 ? (zd & 1) : 0) * 2 * P.rp;
-      for (int kk = 0; kk < P.rp; kk += 16) {
-        const uint64_t hi = (uint64_t)((o + kk) >> 3), lo = (uint64_t)((o + P.rp + kk) >> 3);
-        mma(dcol, da + hi, db + hi, id_corr, kk > 0 ? 1u : 0u);
-        mma(dcol, da + hi, db + lo, id_corr, 1u);
-        mma(dcol, da + lo, db + hi, id_corr, 1u);
+      if (P.zps == 2) {
+        // rank 16: hi at bytes 0-31, lo at 32-63 of each 64-byte row
+        const uint32_t sa = smem_u32(stages + stage * C::STAGE);
+        const uint64_t a64 = sdesc64(sa), b64 = sdesc64(sa + DSTAGE_A);
+        mma(dcol, a64, b64, id_corr, 0u);
+        mma(dcol, a64, b64 + 2, id_corr, 1u);
+        mma(dcol, a64 + 2, b64, id_corr, 1u);
+      } else {
+        const uint64_t db = da + (uint64_t)(DSTAGE_A >> 4);
+        for (int kk = 0; kk < P.rp; kk += 16) {
+          const uint64_t hi = (uint64_t)(kk >> 3), lo = (uint64_t)((P.rp + kk) >> 3);
+          mma(dcol, da + hi, db + hi, id_corr, kk > 0 ? 1u : 0u);
+          mma(dcol, da + hi, db + lo, id_corr, 1u);
+          mma(dcol, da + lo, db + hi, id_corr, 1u);
+        }
       }
       commit_acc(&cfull[r ^ 1]);
       commit_all(&empty[stage]);
@@ -1653,16 +1680,17 @@ static EncodeTiledFn encode_fn() {
 
 // 2-D K-major tile map: rows x cols elements of 2 bytes, box box_rows x 64
 static bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, bool bf16,
-                     uint32_t box_rows) {
+                     uint32_t box_rows, bool narrow = false) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {BK, box_rows};
+  cuuint32_t box[2] = {narrow ? 32u : (cuuint32_t)BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
                   const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  narrow ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -1911,10 +1939,11 @@ cudaError_t launch_draft_pass_tc(const StepCtx& c) {
   const uint32_t bq = tc::DBN / cs;  // B rows each CTA loads
   CUtensorMap ma, mb, mca, mcb;
   const unsigned char* prep = c.prep;
+  const bool narrow = tc::BK / (2 * w.rp) == 2;  // rank 16: one component per 64-byte box
   if (!tc::make_map(&ma, c.args->hidden, h->H, w.M, true, tc::BM) ||
       !tc::make_map(&mb, h->W, h->H, h->V, true, bq) ||
-      !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM) ||
-      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, bq))
+      !tc::make_map(&mca, c.ws + w.off_cop, w.KC, w.Mpad, false, tc::BM, narrow) ||
+      !tc::make_map(&mcb, prep + c.pl.off_wuop, w.KC, h->V, false, bq, narrow))
     return cudaErrorInvalidValue;
   tc::Params P{};
   P.mode = c.greedy ? tc::MODE_GREEDY : tc::MODE_DRAFT;
