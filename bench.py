@@ -155,12 +155,59 @@ def cpu_baseline(cfg, head, blk, T, Z_T, budget_s=30.0, mode="soft", top_k=0, to
         single = {"value": n1 / el1, "unit": UNIT, "threads": 1,
                   "sample": "%d sequence(s), BLAS limited to one thread" % n1}
     except ImportError:
-        single = {"value": None, "why": "threadpoolctl not installed on this host"}
+        single = _single_thread_child(cfg, head_cpu, blk_cpu, T, Z_T, mode, top_k, top_p,
+                                      budget_s / 3)
     return {"value": n_done / el, "unit": UNIT, "cores": _cpu_threads(),
             "kind": "oracle", "nproc": os.cpu_count(), "cpu_model": _cpu_model(),
             "single_thread": single,
             "sample": "%d sequence(s) of the %s workload (one block each, %s mode), fp64 "
                       "direct form" % (n_done, cfg["name"], mode)}
+
+
+def _single_thread_child(cfg, head_cpu, blk_cpu, T, Z_T, mode, top_k, top_p, budget):
+    """The oracle on one sequence of the same inputs in a child process whose
+    BLAS and OpenMP pools are limited to one thread from the start (for hosts
+    without threadpoolctl)."""
+    import tempfile
+    import torch
+    with tempfile.TemporaryDirectory() as td:
+        path = os.path.join(td, "seq0.pt")
+        torch.save({"head": head_cpu, "hidden": blk_cpu["hidden"][:1].clone(),
+                    "target": blk_cpu["target"][:1].clone(), "has_bonus": blk_cpu["has_bonus"],
+                    "T": T, "Z_T": Z_T, "mode": mode, "top_k": top_k, "top_p": top_p,
+                    "budget": budget}, path)
+        env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1",
+                   MKL_NUM_THREADS="1")
+        try:
+            out = subprocess.run([sys.executable, os.path.abspath(__file__),
+                                  "--oracle-single-thread", path], env=env, capture_output=True,
+                                 text=True, timeout=budget * 4 + 120)
+            d = json.loads(out.stdout.strip().splitlines()[-1])
+        except (OSError, subprocess.SubprocessError, ValueError, IndexError) as e:
+            return {"value": None, "why": "single-thread child failed: %s" % type(e).__name__}
+    return {"value": d["n"] / d["s"], "unit": UNIT, "threads": 1,
+            "sample": "%d sequence(s) in a child process with OPENBLAS/OMP/MKL_NUM_THREADS=1"
+                      % d["n"]}
+
+
+def _oracle_single_thread(path):
+    """Child side of _single_thread_child: time the oracle on the saved sequence."""
+    import torch
+    torch.set_num_threads(1)
+    from oracle import dblast_oracle as orc
+    d = torch.load(path)
+    pos = torch.full((1,), 37, dtype=torch.int64).numpy()
+    rnd = torch.zeros(1, dtype=torch.int32).numpy()
+    n, t0 = 0, time.perf_counter()
+    while True:
+        orc.draft_and_verify(d["head"], d["hidden"], None, d["target"], d["has_bonus"], d["T"],
+                             d["Z_T"], 0, pos, rnd, seqs=[0], mode=d["mode"], top_k=d["top_k"],
+                             top_p=d["top_p"])
+        n += 1
+        el = time.perf_counter() - t0
+        if el > d["budget"] or n >= 1:
+            break
+    print(json.dumps({"n": n, "s": el}))
 
 
 def _cpu_model():
@@ -410,6 +457,9 @@ def run_serve(args):
 
 
 def main():
+    if len(sys.argv) == 3 and sys.argv[1] == "--oracle-single-thread":
+        _oracle_single_thread(sys.argv[2])
+        return
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
