@@ -1374,9 +1374,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int m = mt * BM + row;
       const bool mok = m < P.M;
       const int v0 = vt * BN + cq * 32;
-      // per-row constants: B0 here, (k2 / scale, log2 w - L + B0) per component below
+      // per-row constants: B0 and the target log-sum-exp here (used after the
+      // components), (k2 / scale, log2 w - L + B0) per component below
       const float B0f = mok ? P.vb0[m] : 0.f;
       const float2* vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
+      const int n = m / P.B, i = m - n * P.B;
+      const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
       F2 acc2[16];  // columns (2j, 2j+1)
 #pragma unroll
       for (int j = 0; j < 16; ++j) acc2[j] = f2(0.f, 0.f);
@@ -1384,6 +1387,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int g = 0; g < ngroups; ++g) {
         const int gs = g & 1;
         const uint32_t use = gs ? guse1 : guse0;
+        // the group's constants are loaded before the wait for its accumulators
+        const int nz = min(2, P.K - 2 * g);
+        const float2 c0v = mok ? vrow[2 * g] : make_float2(0.f, -INFINITY);
+        const float2 c1v = (mok && nz > 1) ? vrow[2 * g + 1] : make_float2(0.f, -INFINITY);
         if (!mbar_wait(&sfull[gs], use & 1u, ctl, 14)) { ok = false; break; }
         if (gs) ++guse1; else ++guse0;
         tc_fence_after();
@@ -1391,9 +1398,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // read in 16-column chunks (component, half), the load of the next
         // chunk in flight while the current one is reduced; the slot is
         // handed back once the last chunk is in registers
-        const int nz = min(2, P.K - 2 * g);
-        const float2 c0v = mok ? vrow[2 * g] : make_float2(0.f, -INFINITY);
-        const float2 c1v = (mok && nz > 1) ? vrow[2 * g + 1] : make_float2(0.f, -INFINITY);
         const uint32_t tb = tmem + lane_off + (uint32_t)(gs * 2 * BN + cq * 32);
         uint32_t ra[16], rb[16];
         auto chunk = [&](const uint32_t (&r)[16], float2 cz, int h) {
@@ -1432,8 +1436,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // four partial sums per quantity keep the add chains short: As2[h]
       // holds the sums of columns j with j & 3 == 2h and 2h + 1
       F2 As2[2] = {f2(0.f, 0.f), f2(0.f, 0.f)}, Rs2[2] = {f2(0.f, 0.f), f2(0.f, 0.f)};
-      const int n = m / P.B, i = m - n * P.B;
-      const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
       const F2 k2x = f2(P.k2, P.k2), nB0x = f2(-B0f, -B0f);
       const F2 nLtx = f2(-Lt.x, -Lt.x), Ltyx = f2(Lt.y, Lt.y);
       // columns 2jp and 2jp + 1 together
