@@ -1372,18 +1372,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint32_t guse0 = 0u, guse1 = 0u;
+    // per-row constants, loaded again only when the tile's M tile changes:
+    // B0 and the target log-sum-exp (used after the components), and the
+    // row of (k2 / scale, log2 w - L + B0) per component
+    int cur_mt = -1, m = 0;
+    bool mok = false;
+    float B0f = 0.f;
+    float2 Lt = make_float2(0.f, 0.f);
+    const float2* vrow = P.vcz;
     for (int slot = 0; slot < my_tiles; ++slot) {
       int mt, vt;
       vtile_of(P, slot, &mt, &vt);
-      const int m = mt * BM + row;
-      const bool mok = m < P.M;
+      if (mt != cur_mt) {
+        cur_mt = mt;
+        m = mt * BM + row;
+        mok = m < P.M;
+        B0f = mok ? P.vb0[m] : 0.f;
+        vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
+        const int n = m / P.B, i = m - n * P.B;
+        Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
+      }
       const int v0 = vt * BN + cq * 32;
-      // per-row constants: B0 and the target log-sum-exp here (used after the
-      // components), (k2 / scale, log2 w - L + B0) per component below
-      const float B0f = mok ? P.vb0[m] : 0.f;
-      const float2* vrow = P.vcz + (size_t)(mok ? m : 0) * P.K;
-      const int n = m / P.B, i = m - n * P.B;
-      const float2 Lt = mok ? P.lt2[(size_t)n * (P.B + 1) + i] : make_float2(0.f, 0.f);
       F2 acc2[16];  // columns (2j, 2j+1)
 #pragma unroll
       for (int j = 0; j < 16; ++j) acc2[j] = f2(0.f, 0.f);
@@ -1515,6 +1524,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (lane == 0) mbar_arrive(&xempty[cq]);
       } else if (mok) {
         const float* srow = P.stash + (size_t)m * P.V + v0;
+        const int n = m / P.B, i = m - n * P.B;
         const __nv_bfloat16* trow = P.target + ((size_t)n * P.Bt + i) * P.V + v0;
 #pragma unroll
         for (int u = 0; u < 32; ++u)
@@ -1537,9 +1547,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       int last = 0;
       if (lane == 0) {
-        __threadfence_block();
-        last = (atomicAdd(&qcount[(slot & 1) * 4 + q], 1) & 3) == 3;
-        __threadfence_block();
+        // acquire-release at CTA scope: this warp's partials (ordered by the
+        // __syncwarp above) are visible to the warp that counts 3, and that
+        // warp sees the other three
+        uint32_t old;
+        asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], 1;"
+                     : "=r"(old)
+                     : "r"(smem_u32(&qcount[(slot & 1) * 4 + q]))
+                     : "memory");
+        last = (old & 3u) == 3u;
       }
       __syncwarp();
       if (__shfl_sync(0xffffffffu, last, 0)) {
