@@ -1302,6 +1302,14 @@ __device__ __forceinline__ void vtile_of(const VParams& P, int slot, int* mt, in
   *vt = t / P.n_mt;
   *mt = t - *vt * P.n_mt;
 }
+// The next slot's tile: when the grid is a multiple of the M-tile count (the
+// usual launch) the M tile stays and the vocabulary tile advances by a
+// constant, without the integer division of vtile_of (which takes the
+// special-function unit the epilogue keeps busy).
+__device__ __forceinline__ void vtile_next(const VParams& P, int slot, int* mt, int* vt) {
+  if ((int)gridDim.x % P.n_mt == 0) *vt += (int)gridDim.x / P.n_mt;
+  else vtile_of(P, slot + 1, mt, vt);
+}
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     k_tc_verify(const __grid_constant__ CUtensorMap tm_ca, const __grid_constant__ CUtensorMap tm_cb,
@@ -1380,9 +1388,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     float B0f = 0.f;
     float2 Lt = make_float2(0.f, 0.f);
     const float2* vrow = P.vcz;
-    for (int slot = 0; slot < my_tiles; ++slot) {
-      int mt, vt;
-      vtile_of(P, slot, &mt, &vt);
+    int mt, vt;
+    vtile_of(P, 0, &mt, &vt);
+    for (int slot = 0; slot < my_tiles; vtile_next(P, slot, &mt, &vt), ++slot) {
       if (mt != cur_mt) {
         cur_mt = mt;
         m = mt * BM + row;
