@@ -71,7 +71,8 @@ typedef enum {
   DBLAST_ERR_WORKSPACE = 3,    /* prep or workspace buffer too small / misaligned */
   DBLAST_ERR_CUDA = 4,         /* a CUDA runtime call failed */
   DBLAST_ERR_TIMEOUT = 5,      /* a device-side bounded wait ran out (see dblast_device_status) */
-  DBLAST_ERR_NO_DEVICE = 6     /* no usable sm_103 device */
+  DBLAST_ERR_NO_DEVICE = 6,    /* no usable sm_103 device */
+  DBLAST_ERR_BOUNDS = 7        /* a device-side index check failed (see dblast_set_checks) */
 } dblast_status;
 
 typedef enum { DBLAST_BF16 = 0, DBLAST_F32 = 1 } dblast_dtype;
@@ -178,7 +179,10 @@ typedef struct {
 /* Bytes of the prep buffer for this head (depends on V, K, r, e != NULL). */
 size_t dblast_prep_bytes(const dblast_head* head);
 
-/* Bytes of the per-call workspace for N sequences of block B. */
+/* Bytes of the per-call workspace for N sequences of block B.  Its first 256
+ * bytes are the device status word that dblast_device_status() reads and
+ * clears: zero them once before the workspace's first call (the rest needs
+ * no initialisation). */
 size_t dblast_workspace_bytes(const dblast_head* head, int N, int B, int has_bonus);
 
 /* Once per weight set: fills head->prep with W U_z (and W e_z) in fp32 and in
@@ -204,12 +208,24 @@ dblast_status dblast_draft_and_verify(const dblast_head* head, const dblast_bloc
                                       dblast_stream_t stream);
 
 /* Synchronises `stream`, returns DBLAST_ERR_TIMEOUT if a device-side wait of
- * a previous call on this workspace ran out (and clears the record). */
+ * a previous call on this workspace ran out, else DBLAST_ERR_BOUNDS if an
+ * index check of such a call failed (checks on), and clears the record. */
 dblast_status dblast_device_status(void* workspace, dblast_stream_t stream);
 
 /* Host-side fault injection for tests: spin limit of the device-side bounded
  * waits of later calls (0 = default).  A limit of 1 makes waits give up. */
 void dblast_set_wait_limit(uint32_t spins);
+
+/* Device-side index checks of later calls (process-wide; 0 = off, the
+ * default unless the environment sets DBLAST_CHECK=1).  With checks on, every
+ * data-dependent token index a kernel reads (the given tokens of
+ * dblast_al_objective, the drafted tokens the verify kernels look up) is
+ * tested against [0, V); a value outside it is recorded in the workspace
+ * status word and reported as DBLAST_ERR_BOUNDS by dblast_device_status().
+ * There is no trap: with checks on or off the access itself uses the index
+ * clamped into [0, V), so an out-of-range value never reads outside the
+ * target or stash rows.  Not a paper operation: a debugging aid. */
+void dblast_set_checks(int enable);
 
 /* Measurement counters of this process.  dblast_stats_reset(n) zeroes them
  * and sets per-pass timing: with n > 0, CUDA events are recorded on the

@@ -14,7 +14,7 @@ from . import build as _build
 
 DBLAST_OK = 0
 STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "unsupported",
-                3: "workspace", 4: "cuda", 5: "timeout", 6: "no device"}
+                3: "workspace", 4: "cuda", 5: "timeout", 6: "no device", 7: "bounds"}
 DTYPES = {torch.bfloat16: 0, torch.float32: 1}
 IMPLS = {"auto": 0, "simt": 1, "tcgen05": 2}
 MODES = {"soft": 0, "greedy": 1}
@@ -79,7 +79,7 @@ class CVerifyOut(ctypes.Structure):
 
 EXPORTS = ["dblast_prep_bytes", "dblast_workspace_bytes", "dblast_head_prepare",
            "dblast_draft_block", "dblast_verify_block", "dblast_draft_and_verify",
-           "dblast_device_status", "dblast_set_wait_limit", "dblast_stats_reset",
+           "dblast_device_status", "dblast_set_wait_limit", "dblast_set_checks", "dblast_stats_reset",
            "dblast_stats_get", "dblast_target_lse_noalloc", "dblast_status_string",
            "dblast_version", "dblast_determinism_workspace_bytes", "dblast_target_determinism",
            "dblast_al_objective"]
@@ -115,6 +115,8 @@ def load_library(path=None, build_if_missing=True):
     lib.dblast_device_status.restype = ctypes.c_int
     lib.dblast_set_wait_limit.argtypes = [ctypes.c_uint32]
     lib.dblast_set_wait_limit.restype = None
+    lib.dblast_set_checks.argtypes = [ctypes.c_int]
+    lib.dblast_set_checks.restype = None
     lib.dblast_stats_reset.argtypes = [ctypes.c_int]
     lib.dblast_stats_reset.restype = None
     lib.dblast_stats_get.argtypes = [P(CStats)]
@@ -341,6 +343,11 @@ def dblast_device_status(ws):
 
 def dblast_set_wait_limit(spins):
     lib().dblast_set_wait_limit(int(spins))
+
+
+def dblast_set_checks(enable):
+    """Device-side index checks of later calls on (True) or off."""
+    lib().dblast_set_checks(1 if enable else 0)
 
 
 def dblast_stats_reset(enable_pass_timing=True):

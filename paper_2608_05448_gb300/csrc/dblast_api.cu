@@ -9,6 +9,7 @@
 #include <vector>
 
 #include <cuda.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "dblast_internal.cuh"
 
@@ -16,6 +17,30 @@ namespace dblast {
 
 static uint32_t g_wait_limit = 0;  // 0 = default; read by the tensor-core launchers
 uint32_t wait_limit() { return g_wait_limit; }
+
+// Device-side index checks (dblast_set_checks; DBLAST_CHECK=1 turns them on
+// from the start): data-dependent token indices are tested against [0, V)
+// and a value outside it is recorded in the workspace status word.
+static std::atomic<int> g_checks{-1};
+static bool checks_on() {
+  int v = g_checks.load(std::memory_order_relaxed);
+  if (v < 0) {
+    const char* e = getenv("DBLAST_CHECK");
+    v = (e && e[0] == '1') ? 1 : 0;
+    int expect = -1;
+    g_checks.compare_exchange_strong(expect, v);
+    v = g_checks.load(std::memory_order_relaxed);
+  }
+  return v == 1;
+}
+
+// An NVTX range around each entry point (a no-op unless a profiler is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // ------------------------------------------------------------ measurement
 static std::mutex g_stats_mu;
@@ -260,6 +285,7 @@ static dblast_status make_ctx(const dblast_head* h, const dblast_block_args* a, 
   c->Bt = a->B + (has_bonus ? 1 : 0);
   c->fuse_tstats = false;
   c->lse_target = nullptr;
+  c->chk = checks_on() ? reinterpret_cast<DevStatus*>(c->ws + c->wl.off_status) : nullptr;
   return DBLAST_OK;
 }
 
@@ -304,6 +330,7 @@ size_t dblast_workspace_bytes(const dblast_head* h, int N, int B, int has_bonus)
 }
 
 dblast_status dblast_head_prepare(const dblast_head* h, dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_head_prepare");
   dblast_status st = check_head(h, true);
   if (st != DBLAST_OK) return st;
   PrepLayout pl = prep_layout(h->V, h->H, h->K, h->r, h->e != nullptr);
@@ -459,6 +486,7 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
 dblast_status dblast_draft_block(const dblast_head* h, const dblast_block_args* a,
                                  dblast_draft_out* out, void* ws, size_t ws_bytes,
                                  dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_draft_block");
   dblast_status st = check_head(h, true);
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
@@ -471,6 +499,7 @@ dblast_status dblast_draft_block(const dblast_head* h, const dblast_block_args* 
 dblast_status dblast_verify_block(const dblast_head* h, const dblast_block_args* a,
                                   dblast_verify_out* out, void* ws, size_t ws_bytes,
                                   dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_verify_block");
   dblast_status st = check_head(h, true);
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
@@ -486,6 +515,7 @@ dblast_status dblast_verify_block(const dblast_head* h, const dblast_block_args*
 dblast_status dblast_draft_and_verify(const dblast_head* h, const dblast_block_args* a,
                                       dblast_draft_out* dout, dblast_verify_out* vout, void* ws,
                                       size_t ws_bytes, dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_draft_and_verify");
   dblast_status st = check_head(h, true);
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
@@ -505,16 +535,18 @@ dblast_status dblast_device_status(void* ws, dblast_stream_t stream) {
   cudaError_t e = cudaMemcpyAsync(&hs, ws, sizeof(hs), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_status(e);
-  if (hs.timeout) {
+  if (hs.timeout || hs.bounds) {
     e = cudaMemsetAsync(ws, 0, sizeof(DevStatus), s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_status(e);
-    return DBLAST_ERR_TIMEOUT;
+    return hs.timeout ? DBLAST_ERR_TIMEOUT : DBLAST_ERR_BOUNDS;
   }
   return DBLAST_OK;
 }
 
 void dblast_set_wait_limit(uint32_t spins) { g_wait_limit = spins; }
+
+void dblast_set_checks(int enable) { g_checks.store(enable ? 1 : 0, std::memory_order_relaxed); }
 
 void dblast_stats_reset(int enable_pass_timing) {
   std::lock_guard<std::mutex> lk(g_stats_mu);
@@ -553,6 +585,7 @@ dblast_status dblast_stats_get(dblast_stats* out) {
 dblast_status dblast_al_objective(const dblast_head* h, const dblast_block_args* a,
                                   const dblast_al_args* al, void* ws, size_t ws_bytes,
                                   dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_al_objective");
   dblast_status st = check_head(h, true);
   if (st == DBLAST_OK) st = check_args(h, a);
   if (st != DBLAST_OK) return st;
@@ -623,6 +656,7 @@ dblast_status dblast_target_determinism(const void* target, dblast_dtype dtype, 
                                         float* collision, float* d_exact, float* d_hat,
                                         int32_t* samples, void* ws, size_t ws_bytes,
                                         dblast_stream_t stream) {
+  NvtxRange nvtx("dblast_target_determinism");
   if (!target || !aligned16(target)) return DBLAST_ERR_INVALID_ARG;
   if (dtype != DBLAST_BF16 && dtype != DBLAST_F32) return DBLAST_ERR_INVALID_ARG;
   if (N < 1 || rows < 1 || V < 1 || b < 1 || b > 32 || b > rows || M < 0 || M > (1 << 24))
@@ -671,6 +705,7 @@ const char* dblast_status_string(dblast_status s) {
     case DBLAST_ERR_CUDA: return "CUDA runtime error";
     case DBLAST_ERR_TIMEOUT: return "device-side wait ran out";
     case DBLAST_ERR_NO_DEVICE: return "no usable device";
+    case DBLAST_ERR_BOUNDS: return "a device-side index check failed";
   }
   return "unknown status";
 }

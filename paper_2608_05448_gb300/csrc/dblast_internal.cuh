@@ -91,7 +91,20 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
 struct DevStatus {
   uint32_t timeout;      // set to 1 by a bounded wait that ran out
   uint32_t where;        // id of the wait that ran out
+  uint32_t bounds;       // set to 1 by a failed index check (checks on)
+  uint32_t bounds_where; // id of the check that failed
 };
+
+// A data-dependent token index, kept inside [0, V) as always; with checks
+// on (chk != nullptr) a value outside it is also recorded in the status word
+// (no trap: the access that follows uses the clamped index).
+__device__ __forceinline__ int checked_token(int x, int V, DevStatus* chk, uint32_t where) {
+  if (chk != nullptr && (x < 0 || x >= V)) {
+    atomicExch(&chk->bounds, 1u);
+    atomicExch(&chk->bounds_where, where);
+  }
+  return min(max(x, 0), V - 1);
+}
 
 // ------------------------------------------------------------- Philox
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
@@ -264,6 +277,7 @@ struct StepCtx {
   int Bt;              // target rows per sequence (B + has_bonus)
   bool fuse_tstats;    // fused step: the draft pass computes the target statistics
   float* lse_target;   // its natural log-sum-exp output (or null)
+  DevStatus* chk;      // index checks on: the workspace status word, else null
 };
 
 template <typename T> T* wsp(const StepCtx& c, size_t off) { return reinterpret_cast<T*>(c.ws + off); }

@@ -487,7 +487,7 @@ __global__ void __launch_bounds__(DT_NT)
                   const float* __restrict__ log2pi, const float* __restrict__ cscale,
                   const float* __restrict__ sw, float2* __restrict__ w2,
                   float* __restrict__ qtok, float2* __restrict__ vcz, float* __restrict__ vb0,
-                  dblast_draft_out out) {
+                  dblast_draft_out out, DevStatus* chk) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<DT_NT> fs;
   __shared__ FF sL[32];
@@ -523,7 +523,7 @@ __global__ void __launch_bounds__(DT_NT)
   const BranchTokenProb em{srow, wu, cm + z * rr, z, K, rr, k2, L};
   int x;
   if (given) {  // a given block (training-side objectives): no draw
-    x = min(max(given[m], 0), V - 1);
+    x = checked_token(given[m], V, tid == 0 ? chk : nullptr, 1u);
     if (tid == 0) tok[m] = x;
   } else {
     const FindOut f = block_find<DT_NT>(nt, V, tm, em, FF{u, 0.f}, 1.f, fs);
@@ -569,7 +569,7 @@ cudaError_t launch_draft_finalize(const StepCtx& c, const dblast_draft_out* outp
       wsp<int32_t>(c, w.off_tok), wsp<float2>(c, w.off_lq2), wsp<uint32_t>(c, w.off_ties),
       wsp<uint32_t>(c, w.off_ties) + w.N, wsp<float>(c, w.off_log2pi),
       wsp<float>(c, w.off_cscale), prp<float>(c, c.pl.off_sw), wsp<float2>(c, w.off_w2),
-      wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_vcz), wsp<float>(c, w.off_vb0), out);
+      wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_vcz), wsp<float>(c, w.off_vb0), out, c.chk);
   debug_kernel("k_draft_token", c.stream);
   count_launches(2);
   return le != cudaSuccess ? le : cudaGetLastError();
@@ -877,7 +877,7 @@ __global__ void __launch_bounds__(VFS_NT, 1)
                    int K, int rr, int B, int Bt, int nt, int M, int Mpad, int Rt, float k2,
                    uint64_t seed,
                    int64_t* __restrict__ pos, uint32_t* __restrict__ rnd,
-                   dblast_verify_out out) {
+                   dblast_verify_out out, DevStatus* chk) {
   griddep_wait();  // launched as a dependent of the previous kernel
   constexpr int G = VFS_NT / TILE_V;
   __shared__ FindShared<VFS_NT> fs;
@@ -899,7 +899,7 @@ __global__ void __launch_bounds__(VFS_NT, 1)
     float ptok = 0.f, qtok = 1.f, u2 = 0.f, cC = 1.f;
     if (lane < B) {
       const int m = n * B + lane;
-      const int x = min(max(tok[m], 0), V - 1);
+      const int x = checked_token(tok[m], V, chk, 3u);
       const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
       const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
       qtok = qtok_ws[m];
@@ -1081,7 +1081,7 @@ static cudaError_t verify_final_typed(const StepCtx& c, const dblast_verify_out*
       wsp<float>(c, w.off_qtok), wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partv),
       wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
       wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.rr, w.B, Bt,
-      w.nt, w.M, w.Mpad, w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o);
+      w.nt, w.M, w.Mpad, w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o, c.chk);
   debug_kernel("k_verify_final", c.stream);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();
@@ -1329,7 +1329,7 @@ __global__ void __launch_bounds__(VF_NT)
                     const int32_t* tok, const uint32_t* ties_draft, const float* __restrict__ coll,
                     int V, int K, int B, int Bt, int nt, int Rt, float k2, uint64_t seed,
                     int64_t* __restrict__ pos, uint32_t* __restrict__ rnd, dblast_verify_out out,
-                    GreedyDraftArgs gd) {
+                    GreedyDraftArgs gd, DevStatus* chk) {
   griddep_wait();  // launched as a dependent of the previous kernel
   __shared__ FindShared<VF_NT> fs;
   __shared__ int X[1024];
@@ -1403,7 +1403,7 @@ __global__ void __launch_bounds__(VF_NT)
     float S = 0.f;
     if (lane < B) {
       const int m = n * B + lane;
-      const int x = min(max(tokS[lane], 0), V - 1);
+      const int x = checked_token(tokS[lane], V, chk, 4u);
       const FF Lt = ff_ld(lt2 + (size_t)n * (B + 1) + lane);
       const float tx = ldf(target + ((size_t)n * Bt + lane) * V + x);
       ptok = (tx == -INFINITY) ? 0.f : ff_exp2(ff_sub(ff_prod(tx, k2), Lt));
@@ -1579,7 +1579,7 @@ static cudaError_t greedy_verify_typed(const StepCtx& c, const dblast_verify_out
       wsp<int32_t>(c, w.off_xhat), wsp<uint32_t>(c, w.off_cmask), wsp<float>(c, w.off_qtok),
       wsp<float2>(c, w.off_lt2), wsp<float2>(c, w.off_partt), wsp<int32_t>(c, w.off_tok),
       wsp<uint32_t>(c, w.off_ties), wsp<float>(c, w.off_coll), w.V, c.head->K, w.B, c.Bt, w.nt,
-      w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o, gd);
+      w.Rt, c.k2, c.args->seed, c.args->pos, c.args->round, *o, gd, c.chk);
   debug_kernel("k_greedy_verify", c.stream);
   count_launches(1);
   return le != cudaSuccess ? le : cudaGetLastError();

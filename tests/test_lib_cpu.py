@@ -99,8 +99,16 @@ def test_workspace_too_small_is_rejected():
 
 def test_status_strings():
     lib = bd.lib()
-    for s in range(7):
+    for s in range(8):
         assert lib.dblast_status_string(s)
+        assert not lib.dblast_status_string(s).startswith(b"unknown")
+    assert bd.STATUS_NAMES[7] == "bounds"
+
+
+def test_check_switch_is_host_only():
+    # toggling the device-side index checks touches no device state
+    bd.dblast_set_checks(True)
+    bd.dblast_set_checks(False)
 
 
 @pytest.mark.parametrize("kw,status", [
