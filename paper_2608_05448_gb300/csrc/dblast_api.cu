@@ -1,6 +1,7 @@
 // C ABI of libdblast: argument checks, prep/workspace layouts, launch order.
 // Every entry point is asynchronous on the caller's stream and allocates no
 // device memory.
+#include <algorithm>
 #include <atomic>
 #include <cstdio>
 #include <cstdlib>
@@ -167,7 +168,11 @@ WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus)
   w.off_cop = take((size_t)w.Mpad * w.KC * sizeof(__half));
   w.off_zhat = take((size_t)N * sizeof(int32_t));
   w.off_log2pi = take((size_t)N * K * sizeof(float));
-  w.off_stash = take((size_t)w.M * V * sizeof(float));
+  // the stash [M, V]; before the draft pass writes it, the same bytes hold
+  // the split-K partials of the codes (up to CODES_MAX_SPLIT splits of
+  // [M, K rr]), so it is never smaller than those
+  w.off_stash = take((size_t)w.M * std::max<size_t>((size_t)V, (size_t)CODES_MAX_SPLIT * K * w.rr) *
+                     sizeof(float));
   w.off_partd = take((size_t)w.nt * K * w.Mpad * sizeof(float2));
   w.off_lsep = take((size_t)LSE_SPLIT * w.M * K * sizeof(float4));
   w.off_lse2 = take((size_t)w.M * K * sizeof(float2));

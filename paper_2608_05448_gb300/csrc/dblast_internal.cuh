@@ -88,6 +88,9 @@ PrepLayout prep_layout(int V, int H, int K, int r, bool has_e);
 WsLayout ws_layout(int V, int K, int r, bool has_e, int N, int B, int has_bonus);
 
 // device status word at the start of the workspace
+// most split-K partials of the per-call codes GEMM (both kernel families)
+constexpr int CODES_MAX_SPLIT = 16;
+
 struct DevStatus {
   uint32_t timeout;      // set to 1 by a bounded wait that ran out
   uint32_t where;        // id of the wait that ran out

@@ -346,8 +346,7 @@ template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
     cudaError_t e = launch_codes_tc(c, part, &nsplit);
     if (e != cudaSuccess) return e;
   } else {
-    nsplit = max(1, min(16, h->H / 256));
-    nsplit = max(1, min(nsplit, (int)(((size_t)w.M * h->V) / ((size_t)w.M * Nb))));
+    nsplit = max(1, min(CODES_MAX_SPLIT, h->H / 256));
     const int hchunk = ceil_div(ceil_div(h->H, nsplit), 32) * 32;
     ExpanderCols<Tin> bf{static_cast<const Tin*>(h->Vf), nullptr, h->H, h->r, w.rr};
     dim3 grid(ceil_div(w.M, 64), ceil_div(Nb, 64), ceil_div(h->H, hchunk));

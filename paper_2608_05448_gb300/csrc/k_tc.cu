@@ -1936,7 +1936,7 @@ cudaError_t launch_codes_tc(const StepCtx& c, float* part, int* nsplit) {
   const int nb64 = h->H / tc::BK;
   const int base_tiles = (rows_pad / tc::BM) * ceil_div(w.M, tc::DBN);
   int ks = 1;
-  for (int d = 1; d <= 16 && d <= nb64; ++d)
+  for (int d = 1; d <= CODES_MAX_SPLIT && d <= nb64; ++d)
     if (nb64 % d == 0 && base_tiles * d <= tc::num_sms()) ks = d;
   tc::Params P{};
   P.mode = tc::MODE_PREP;

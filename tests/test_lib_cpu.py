@@ -45,6 +45,11 @@ def test_prep_and_workspace_sizes():
     assert ws >= 32 * 16 * V * 4            # fp32 stash of the base logits
     assert ws < 32 * 16 * V * 4 * 1.35      # everything else is small next to it
     assert lib.dblast_workspace_bytes(ctypes.byref(h), 32, 16, 0) == ws
+    # a small vocabulary with many components: the stash region, which first
+    # holds up to 16 split-K partials of the codes [M, K r], is sized for them
+    hs = fake_head(V=3000, H=4096, K=16, r=32)
+    M = 4 * 4
+    assert lib.dblast_workspace_bytes(ctypes.byref(hs), 4, 4, 1) >= 16 * M * 16 * 32 * 4
 
 
 def _args(N=2, B=3, T=1.0, zt=1.0):
