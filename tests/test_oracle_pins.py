@@ -273,7 +273,7 @@ def test_oracle_step_monte_carlo_matches_exact_laws():
     head, h, t = _tiny_case(2, 77, V=5, B=3)
     T = 0.7
     e_len, _, q, pi, p = _exact_expected_length(head, h, t, T)
-    n = 6000
+    n = 60000
     first = np.zeros(5)
     drafted = np.zeros(5)
     Ls = []
