@@ -800,18 +800,21 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
     float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
     float s0 = -INFINITY, s1 = -INFINITY, s2 = -INFINITY, s3 = -INFINITY;
     int i0 = 0, i1 = 1, i2 = 2, i3 = 3;
+    // 16-column chunks, the load of chunk c+1 in flight while chunk c is
+    // reduced (two 16-register buffers: with 32-column ones the epilogue,
+    // which holds the tile's 128 base logits, spilled)
     const uint32_t tb = tmem + lane_off + (uint32_t)(rg * DBN + half * DCOLS);
-    uint32_t ra[32], rb[32];
-    tmem_ld32_raw(tb, ra);
-    tmem_wait_ld(ra);
+    uint32_t ra[16], rb[16];
+    tmem_ld16_raw(tb, ra);
+    tmem_wait_ld16(ra);
 #pragma unroll
-    for (int cc = 0; cc < DCOLS / 32; ++cc) {
-      uint32_t(&cur)[32] = (cc & 1) ? rb : ra;
-      uint32_t(&nxt)[32] = (cc & 1) ? ra : rb;
-      if (cc + 1 < DCOLS / 32) tmem_ld32_raw(tb + (uint32_t)((cc + 1) * 32), nxt);
+    for (int cc = 0; cc < DCOLS / 16; ++cc) {
+      uint32_t(&cur)[16] = (cc & 1) ? rb : ra;
+      uint32_t(&nxt)[16] = (cc & 1) ? ra : rb;
+      if (cc + 1 < DCOLS / 16) tmem_ld16_raw(tb + (uint32_t)((cc + 1) * 16), nxt);
 #pragma unroll
-      for (int j = 0; j < 32; j += 4) {
-        const int c = cc * 32 + j;
+      for (int j = 0; j < 16; j += 4) {
+        const int c = cc * 16 + j;
         const float x0 = fmaf(__uint_as_float(cur[j]), a, bk[c]);
         const float x1 = fmaf(__uint_as_float(cur[j + 1]), a, bk[c + 1]);
         const float x2 = fmaf(__uint_as_float(cur[j + 2]), a, bk[c + 2]);
@@ -827,7 +830,7 @@ __device__ __forceinline__ bool greedy_components(const Params& P, uint32_t tmem
         if (x2 > m2) { m2 = x2; i2 = c + 2; }
         if (x3 > m3) { m3 = x3; i3 = c + 3; }
       }
-      if (cc + 1 < DCOLS / 32) tmem_wait_ld(nxt);
+      if (cc + 1 < DCOLS / 16) tmem_wait_ld16(nxt);
     }
     tc_fence_before();
     __syncwarp();
