@@ -345,9 +345,9 @@ dblast_status dblast_head_prepare(const dblast_head* h, dblast_stream_t stream) 
 
 static dblast_status draft_impl(const StepCtx& c, dblast_draft_out* out) {
   g_calls.fetch_add(1, std::memory_order_relaxed);
-  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
-                                  c.stream);
-  if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
+  // the tie words and draft-token counters start in the launch that computes
+  // the prior (no memset: it would end the chain of dependent launches)
+  cudaError_t e = dbg(launch_codes(c), "codes", c.stream);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
     e = c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c);
@@ -450,10 +450,9 @@ static dblast_status step_impl(StepCtx c, dblast_draft_out* dout, dblast_verify_
   cudaError_t e = side_stream(&ss);
   StepCtx side = c;
   if (e == cudaSuccess) side.stream = ss->s;
-  if (e == cudaSuccess)
-    e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t), c.stream);
   // the codes GEMM, then the codes reduction and the category prior in one
-  // launch, then the draft pass
+  // launch (which also starts the tie words and the draft-token counters),
+  // then the draft pass
   if (e == cudaSuccess) e = launch_codes(c);
   if (e == cudaSuccess) {
     pass_event_begin(0, c.stream);
@@ -610,9 +609,9 @@ dblast_status dblast_al_objective(const dblast_head* h, const dblast_block_args*
   c.target = al->target;
   c.Bt = a->B + vo.has_bonus;
   g_calls.fetch_add(1, std::memory_order_relaxed);
-  cudaError_t e = cudaMemsetAsync(c.ws + c.wl.off_ties, 0, (size_t)2 * c.wl.N * sizeof(uint32_t),
-                                  c.stream);
-  if (e == cudaSuccess) e = dbg(launch_codes(c), "codes", c.stream);
+  // the tie words and draft-token counters start in the launch that computes
+  // the prior (no memset: it would end the chain of dependent launches)
+  cudaError_t e = dbg(launch_codes(c), "codes", c.stream);
   if (e == cudaSuccess)
     e = dbg(c.tc ? launch_draft_pass_tc(c) : launch_draft_pass_simt(c), "draft_pass", c.stream);
   if (e == cudaSuccess) e = dbg(launch_draft_finalize(c, nullptr, al->tokens), "draft_finalize", c.stream);

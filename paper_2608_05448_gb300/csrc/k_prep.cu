@@ -180,7 +180,8 @@ __device__ __forceinline__ void prior_body(int n, const Tin* __restrict__ Wp,
                                            const uint32_t* __restrict__ rnd,
                                            int32_t* __restrict__ zhat_ws,
                                            float* __restrict__ log2pi_ws,
-                                           uint32_t* __restrict__ ties, float* ell) {
+                                           uint32_t* __restrict__ ties, uint32_t* __restrict__ done,
+                                           float* ell) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const Tin* a = anchor ? anchor + (size_t)n * H : hidden + (size_t)n * B * H;
   for (int z = warp; z < K; z += blockDim.x >> 5) {
@@ -244,8 +245,13 @@ __device__ __forceinline__ void prior_body(int n, const Tin* __restrict__ Wp,
     zh = posm ? 31 - __clz(posm) : 0;
   }
   if (lane == 0) {
-    if (zt != 0.f && margin < TIE_TOL) atomicOr(&ties[n], TIE_ZHAT);
-    if (zt != 0.f && margin < TIE_TOL + NEAR_DRAW) atomicOr(&ties[n], TIE_ZHAT << NEAR_SHIFT);
+    // this call's tie word of the sequence starts here (the kernels after
+    // this one add their bits), and so does the draft-token block counter
+    uint32_t bits = 0u;
+    if (zt != 0.f && margin < TIE_TOL) bits |= TIE_ZHAT;
+    if (zt != 0.f && margin < TIE_TOL + NEAR_DRAW) bits |= TIE_ZHAT << NEAR_SHIFT;
+    ties[n] = bits;
+    done[n] = 0u;
     zhat_ws[n] = zh;
   }
   if (on) log2pi_ws[n * K + lane] = pz > 0.f ? log2f(pz) : -INFINITY;
@@ -313,6 +319,7 @@ struct PriorArgs {
   int32_t* zhat;
   float* log2pi;
   uint32_t* ties;
+  uint32_t* done;  // draft-token block counters [N]
 };
 template <typename Tin>
 __global__ void __launch_bounds__(256)
@@ -330,7 +337,8 @@ __global__ void __launch_bounds__(256)
   }
   prior_body<Tin>((int)blockIdx.x - nfin, static_cast<const Tin*>(pa.Wp), pa.bp,
                   static_cast<const Tin*>(pa.anchor), static_cast<const Tin*>(pa.hidden), pa.H,
-                  pa.K, pa.B, pa.zt, pa.seed, pa.pos, pa.rnd, pa.zhat, pa.log2pi, pa.ties, ell);
+                  pa.K, pa.B, pa.zt, pa.seed, pa.pos, pa.rnd, pa.zhat, pa.log2pi, pa.ties, pa.done,
+                  ell);
 }
 
 template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
@@ -360,7 +368,8 @@ template <typename Tin> static cudaError_t codes_typed(const StepCtx& c) {
   const int nfin = ceil_div(warps * 32, 256);
   const PriorArgs pa{h->Wp, h->bp, a->anchor, a->hidden, h->H, h->K, a->B, a->z_temperature,
                      a->seed, a->pos, a->round, wsp<int32_t>(c, w.off_zhat),
-                     wsp<float>(c, w.off_log2pi), wsp<uint32_t>(c, w.off_ties)};
+                     wsp<float>(c, w.off_log2pi), wsp<uint32_t>(c, w.off_ties),
+                     wsp<uint32_t>(c, w.off_ties) + w.N};
   cudaError_t le = launch_dep(
       k_codes_prior<Tin>, dim3(nfin + a->N), dim3(256), 0, s, part, nsplit, w.M, w.Mpad, h->K,
       h->r, w.rr, w.rp, c.has_e, wsp<float>(c, w.off_codes), wsp<float>(c, w.off_cscale),
