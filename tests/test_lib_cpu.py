@@ -177,3 +177,16 @@ def test_al_objective_arguments_are_checked_before_launch(mutate, status):
     got = lib.dblast_al_objective(ctypes.byref(h), ctypes.byref(a), ctypes.byref(al), p,
                                   need - 1, None)
     assert got == status
+
+
+def test_no_cluster_multicast_copies_in_the_kernels():
+    # every CTA copies its own operand boxes: no bulk or tensor copy in the
+    # sources uses cluster multicast (the library also runs as independent
+    # replicas, one per GPU)
+    csrc = os.path.join(ROOT, "paper_2608_05448_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if not name.endswith((".cu", ".cuh")):
+            continue
+        for line in open(os.path.join(csrc, name)):
+            if "cp.async.bulk" in line:
+                assert "multicast" not in line, (name, line.strip())
